@@ -1,0 +1,308 @@
+/*
+ * pace.h - C ABI of the PACE hot path on GB300 (sm_103a).
+ *
+ * PACE (Pool-Aware Control of Effective Staleness) admits completed
+ * trajectories of an asynchronous RL pool into the trainer.  This library
+ * computes, on one GPU:
+ *   (a) per-trajectory staleness scores from per-token policy-version tags
+ *       (Lemma 1 / Eq. 2; Eqs. 7-10), the occupancy rejection budget
+ *       (Eqs. 3-4) and the deterministic rejection of the top-scored units
+ *       (Sec. 3.1 quantile rule; Algorithm 1, trainer side);
+ *   (b) for the accepted batch, each token's log-probability under the
+ *       current policy through a fused LM head (logits never reach memory)
+ *       and the asymmetric, dual-clipped token-mean surrogate of the
+ *       unchanged GRPO update (shared training settings of the appendix).
+ *
+ * Conventions shared by every entry point
+ *   - Pointers marked "device" are CUDA device pointers; "host" are host
+ *     pointers.  The caller owns every buffer; the library never allocates.
+ *   - Every call is asynchronous and ordered on `stream` (a cudaStream_t;
+ *     NULL is the legacy default stream).  Nothing is synchronised unless a
+ *     comment says so.
+ *   - Errors found from the arguments alone are returned at once, before any
+ *     launch.  Errors found in the data on the device (a version tag above
+ *     its completion version, a target outside the vocabulary, a wait that
+ *     ran out) are written to `*status_dev`, an int32 in device memory: the
+ *     first error wins (compare-and-swap from 0), so the caller sets it to 0
+ *     before the work and reads it after synchronising.  status_dev may be
+ *     NULL, in which case device-side errors are not reported.  After a
+ *     device-side error the outputs of that call are unspecified.
+ *   - `workspace` is caller-owned device scratch of at least the size the
+ *     matching *_workspace_size() query returns, 256-byte aligned; its
+ *     contents need not be initialised and are clobbered.
+ *   - bf16 arrays are passed as raw 16-bit storage (`const void*`).
+ */
+#ifndef PACE_H_
+#define PACE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define PACE_API __attribute__((visibility("default")))
+#else
+#define PACE_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  PACE_OK = 0,
+  PACE_ERR_INVALID_ARG = 1,       /* bad pointer, size, parameter or CSR offsets */
+  PACE_ERR_VERSION_ORDER = 2,     /* v_t > c(tau) or c(tau) > j: Lemma 1's premise fails */
+  PACE_ERR_NAN_INPUT = 3,         /* NaN in the prefix-score window or in unit scores */
+  PACE_ERR_UNSUPPORTED_SHAPE = 4, /* shape or alignment the kernels do not handle */
+  PACE_ERR_WORKSPACE = 5,         /* workspace missing, too small or misaligned */
+  PACE_ERR_TIMEOUT = 6,           /* a bounded on-device wait ran out (device-side only) */
+  PACE_ERR_CUDA = 7               /* a CUDA runtime call failed (no device, launch error) */
+} pace_status;
+
+/* Human-readable name of a status code (static storage). */
+PACE_API const char* pace_status_string(pace_status status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+PACE_API int32_t pace_version(void);
+
+/* ------------------------------------------------------------------------ */
+/* (a) Pool scoring                                                          */
+/* ------------------------------------------------------------------------ */
+
+/* Trajectory score M(tau; j) of Eq. 7 (Sec. 3.2):
+ *   PACE_SCORE_EFF  Effective Staleness, Eq. 8:  K_wait + F * K_gen
+ *   PACE_SCORE_RAW  PACE (Raw Staleness):         K_wait + K_gen
+ *   PACE_SCORE_GEN  PACE (Generation Staleness):  F * K_gen
+ * where F = phi_gamma(q) (Eq. 10) and q is the empirical percentile of the
+ * trajectory's prefix forgetting score in the window (Eq. 9). */
+typedef enum { PACE_SCORE_EFF = 0, PACE_SCORE_RAW = 1, PACE_SCORE_GEN = 2 } pace_score_mode;
+
+typedef struct {
+  int32_t mode;       /* pace_score_mode; default PACE_SCORE_EFF */
+  int32_t gamma;      /* integer sharpening exponent of Eq. 10, 1..64; default 4 */
+  int32_t min_obs;    /* window size below which F = 1 for all (falls back to Raw); default 32 */
+  int32_t group_size; /* G: trajectories g*G .. g*G+G-1 form unit g; default 8 (1 = per trajectory) */
+  double f_missing;   /* F of a trajectory without a prefix score (s_pre NaN); default 1.0 */
+} PaceScoreParams;
+
+/* Fill `p` with the defaults above (the paper's admission settings). */
+PACE_API void pace_score_params_default(PaceScoreParams* p);
+
+/* Score every trajectory of the pool (Lemma 1 / Eq. 2, Eqs. 7-10) and average
+ * the scores of each group of G ("mean aggregation within groups").
+ *
+ *   tags        device int32 [n_tokens], 16-byte aligned: policy version v_t
+ *               of each response token (Sec. 2), trajectory-major; -1 marks a
+ *               token the policy did not generate (tool output), which is left
+ *               out of K_gen.  Versions are below 2^31 - 1.
+ *   offsets     device int64 [n_traj+1]: tokens of trajectory i are
+ *               tags[offsets[i] .. offsets[i+1]); offsets[0] = 0,
+ *               non-decreasing, offsets[n_traj] = n_tokens.
+ *   c_version   device int32 [n_traj]: c(tau), the trainer version at which
+ *               the trajectory completed (= entered the pool), 0 <= c <= j.
+ *   s_pre       device float32 [n_traj]: prefix forgetting score (Eq. 6) or
+ *               NaN when no prefix was rescored.  May be NULL for RAW mode.
+ *   trainer_version  j, the step that consumes the pool.
+ *   window      device float32 [window_len]: W^pre, recent prefix scores
+ *               (Eq. 9); 0 <= window_len <= 4096; NaN is an error.  May be
+ *               NULL when window_len is 0.
+ * Outputs (device float64, may individually be NULL except score):
+ *   kgen, kwait, weight (F), score [n_traj]; unit_score [n_traj / G].
+ * Values are bit-identical to the fp64 definitions: K_gen = S / T with
+ * S = sum (c - v_t) summed exactly in integers (0 when T = 0); q = count of
+ * window values <= s_pre (float32 compare) / |W|; integer powers by repeated
+ * multiplication; no fused multiply-add anywhere.
+ * Device-side errors: PACE_ERR_VERSION_ORDER (v_t > c or c > j),
+ * PACE_ERR_INVALID_ARG (tag < -1, c < 0, bad offsets), PACE_ERR_NAN_INPUT.
+ * Host errors: PACE_ERR_INVALID_ARG when n_traj is not a multiple of G or a
+ * required pointer is NULL. */
+PACE_API pace_status pace_score_pool(const int32_t* tags, const int64_t* offsets,
+                            const int32_t* c_version, const float* s_pre, int64_t n_traj,
+                            int64_t n_tokens, int32_t trainer_version, const float* window,
+                            int64_t window_len, const PaceScoreParams* params, double* kgen,
+                            double* kwait, double* weight, double* score, double* unit_score,
+                            void* workspace, size_t workspace_bytes, int32_t* status_dev,
+                            void* stream);
+
+/* Workspace bytes pace_score_pool needs for a pool of n_traj trajectories. */
+PACE_API size_t pace_score_pool_workspace_size(int64_t n_traj, int64_t window_len);
+
+/* ------------------------------------------------------------------------ */
+/* (a) Rejection budget and selection                                        */
+/* ------------------------------------------------------------------------ */
+
+typedef struct {
+  int64_t n_target;  /* N^tar, desired buffer of ready trajectories (Eq. 3) */
+  double beta;       /* EMA coefficient of Eq. 4, in [0, 1); default 0 */
+  double r_max;      /* maximum rejection budget; default 0.9 (admission settings) */
+  double r_hat_prev; /* r-hat_{j-1}, the smoothed rate of the previous step; default 0 */
+} PaceBudgetParams;
+
+PACE_API void pace_budget_params_default(PaceBudgetParams* p);
+
+/* Host only, no device work.  Eq. 3 and Eq. 4:
+ *   r     = clip((N - N^tar) / max(N, 1), 0, 1)        N = n_traj
+ *   r_hat = beta * r_hat_prev + (1 - beta) * r
+ *   k     = min(floor(min(r_hat, r_max) * n_units + 1e-9), n_units)
+ * The 1e-9 nudge lands the floor on the exact surplus when fp64 rounding of
+ * the product falls just below an integer (N = 47, N^tar = 35 gives 12).
+ * Outputs are host pointers; r_out may be NULL. */
+PACE_API pace_status pace_budget(int64_t n_traj, int64_t n_units, const PaceBudgetParams* p,
+                        double* r_out, double* r_hat_out, int64_t* k_units_out);
+
+/* Budget + rejection (Sec. 3.1; Algorithm 1, trainer side).  Computes k on
+ * the host with pace_budget (no device synchronisation), then rejects on the
+ * device the k units with the largest unit score; equal scores reject the
+ * lower unit id first.  This is the quantile rule of Sec. 3.1 with the
+ * window taken as the current pool: it rejects exactly floor(r_hat * U)
+ * units, and ties are settled deterministically.
+ *   unit_score     device float64 [n_units], >= 0 (as pace_score_pool
+ *                  writes them); NaN gives PACE_ERR_NAN_INPUT on the device.
+ *   group_size     G; unit u is trajectories u*G .. u*G+G-1; n_traj = U*G.
+ *   r_hat_out, k_units_out   host outputs: r-hat_j (carry to the next step)
+ *                  and k.
+ *   accepted_ids   device int32, room for n_units*G entries: the
+ *                  (U-k)*G accepted trajectory ids, ascending.
+ *   rejected_ids   device int32, room for n_units*G entries (or NULL): the
+ *                  k*G rejected ids, ascending.
+ *   traj_accepted  device uint8 [n_units*G] or NULL: 1 accepted, 0 rejected. */
+PACE_API pace_status pace_select(const double* unit_score, int64_t n_units, int32_t group_size,
+                        const PaceBudgetParams* budget, double* r_hat_out,
+                        int64_t* k_units_out, int32_t* accepted_ids, int32_t* rejected_ids,
+                        uint8_t* traj_accepted, void* workspace, size_t workspace_bytes,
+                        int32_t* status_dev, void* stream);
+
+/* Same rejection with k given by the caller (0 <= k_units <= n_units). */
+PACE_API pace_status pace_select_k(const double* unit_score, int64_t n_units, int32_t group_size,
+                          int64_t k_units, int32_t* accepted_ids, int32_t* rejected_ids,
+                          uint8_t* traj_accepted, void* workspace, size_t workspace_bytes,
+                          int32_t* status_dev, void* stream);
+
+PACE_API size_t pace_select_workspace_size(int64_t n_units);
+
+/* ------------------------------------------------------------------------ */
+/* (b) Log-probabilities and the clipped surrogate                           */
+/* ------------------------------------------------------------------------ */
+
+typedef enum {
+  PACE_AGG_TOKEN_MEAN = 0,          /* sum_t m_t L_t / sum_t m_t ("Token mean") */
+  PACE_AGG_SEQ_MEAN_TOKEN_MEAN = 1  /* mean over sequences of each one's token mean */
+} pace_loss_agg;
+
+typedef struct {
+  float eps_low;      /* lower clip width; default 0.20 */
+  float eps_high;     /* upper clip width; default 0.28 */
+  float dual_clip;    /* dual-clip coefficient c (applies when A < 0); default 10 */
+  float adv_eps;      /* epsilon of the group standardisation; default 1e-6 */
+  int32_t agg;        /* pace_loss_agg; default PACE_AGG_TOKEN_MEAN */
+  int32_t std_unbiased; /* 1: sample std (n - 1), 0: population std; default 1 */
+} PaceLossParams;
+
+PACE_API void pace_loss_params_default(PaceLossParams* p);
+
+/* A batch of sequences laid out as rows (one row per token). */
+typedef struct {
+  const int64_t* seq_offsets;  /* device int64 [n_seq+1]: rows of sequence i are
+                                  [seq_offsets[i], seq_offsets[i+1]); 0 .. n_rows */
+  const uint8_t* seq_accepted; /* device uint8 [n_seq] or NULL (all accepted) */
+  const uint8_t* mask;         /* device uint8 [n_rows] or NULL (all rows): 1 = the
+                                  row is a policy token in the loss, 0 = prompt or
+                                  tool output (kept in context, masked from the loss) */
+  int64_t n_seq;
+  int64_t n_rows;
+} PaceBatch;
+
+/* The policy-objective inputs of the batch. */
+typedef struct {
+  const float* behav_lp; /* device float32 [n_rows]: ell^mu_t recorded at rollout */
+  const float* reward;   /* device float32 [n_seq] */
+  int32_t group_size;    /* G: sequences g*G .. g*G+G-1 are prompt group g; n_seq % G == 0 */
+  PaceLossParams params;
+  double* loss;          /* device float64 [1]: the loss (output) */
+  float* adv;            /* device float32 [n_seq] or NULL: advantages used (output) */
+  float* ratio;          /* device float32 [n_rows] or NULL: rho_t of rows in the loss,
+                            0 elsewhere (output) */
+} PaceLossArgs;
+
+/* GRPO within-group standardisation over the accepted members of each group:
+ *   A_i = (R_i - mean_g) / (std_g + adv_eps);  rejected members get 0; a
+ *   member whose reward equals the group mean gets 0.
+ * reward device float32 [n_seq]; seq_accepted device uint8 [n_seq] or NULL;
+ * adv device float32 [n_seq] (output).  Sums in fp64, lowest index first. */
+PACE_API pace_status pace_group_advantages(const float* reward, const uint8_t* seq_accepted,
+                                  int64_t n_seq, int32_t group_size, float adv_eps,
+                                  int32_t std_unbiased, float* adv, void* stream);
+
+/* Fused LM head: for every row r in the loss (mask[r] != 0 and its sequence
+ * accepted) compute
+ *   z_v     = h_r . W_v              bf16 x bf16, fp32 accumulation (tcgen05/TMEM)
+ *   lse_r   = log sum_v exp(z_v / temperature)   (online, over the whole vocabulary)
+ *   lp_r    = z_{y_r} / temperature - lse_r
+ * without writing any logit to memory.  Rows not in the loss get lp = 0 and
+ * lse = 0.  The hidden row r must be the state that predicts targets[r].
+ *   hidden     device bf16 [n_rows][hidden_size], row-major, 16-byte aligned.
+ *   w_vocab    device bf16 [vocab_size][hidden_size] (the lm_head.weight
+ *              layout), 16-byte aligned.
+ *   targets    device int32 [n_rows], 0 <= y < vocab_size for rows in the loss
+ *              (else PACE_ERR_INVALID_ARG on the device and lp = NaN).
+ *   hidden_size  multiple of 64, 64..16384; vocab_size 1..2^24; temperature > 0.
+ *   logprob    device float32 [n_rows] (output); lse device float32 [n_rows]
+ *              or NULL (output).
+ *   loss       NULL, or the surrogate inputs: the call then also computes
+ *              advantages (pace_group_advantages), the per-token clipped terms
+ *              and the aggregated loss exactly as pace_surrogate_loss does,
+ *              fused after the log-probs.
+ * Rows in the loss are first compacted (their hidden states gathered into the
+ * workspace) so the tensor cores only see rows that count. */
+PACE_API pace_status pace_token_logprob(const PaceBatch* batch, const void* hidden, const void* w_vocab,
+                               const int32_t* targets, int32_t hidden_size, int32_t vocab_size,
+                               float temperature, float* logprob, float* lse,
+                               const PaceLossArgs* loss, void* workspace, size_t workspace_bytes,
+                               int32_t* status_dev, void* stream);
+
+PACE_API size_t pace_token_logprob_workspace_size(int64_t n_rows, int64_t n_seq, int32_t hidden_size,
+                                         int32_t vocab_size);
+
+/* Clipped surrogate on given log-probabilities (shared training settings:
+ * asymmetric clip eps_low / eps_high, dual clip c, token-mean aggregation):
+ *   rho_t = exp(clamp(lp_t - ell^mu_t, -20, 20))
+ *   L_t   = max(-A rho_t, -A clip(rho_t, 1 - eps_low, 1 + eps_high)),
+ *           then min(L_t, -c A) when A < 0
+ *   loss  = sum_t m_t L_t / sum_t m_t  (TOKEN_MEAN), or the mean over
+ *           sequences with tokens of each sequence's token mean.
+ * A is the group-standardised advantage of the row's sequence.  Per-token
+ * terms in fp32, sums in fp64 in a fixed order (deterministic).  An empty
+ * loss is 0.  logprob is device float32 [n_rows]. */
+PACE_API pace_status pace_surrogate_loss(const PaceBatch* batch, const float* logprob,
+                                const PaceLossArgs* loss, void* workspace,
+                                size_t workspace_bytes, int32_t* status_dev, void* stream);
+
+PACE_API size_t pace_surrogate_loss_workspace_size(int64_t n_rows, int64_t n_seq);
+
+/* ------------------------------------------------------------------------ */
+/* Profiling                                                                 */
+/* ------------------------------------------------------------------------ */
+
+typedef enum {
+  PACE_PROFILE_LMHEAD = 0,     /* the fused LM-head kernel of pace_token_logprob */
+  PACE_PROFILE_TAG_REDUCE = 1  /* the tag-stream reduction of pace_score_pool */
+} pace_profile_kernel;
+
+/* Not part of the method: a measurement aid.  From now on, on the calling
+ * host thread, record the CUDA event `begin` (a cudaEvent_t) on the call's
+ * stream immediately before each launch of the given kernel and `end`
+ * immediately after it, so a caller can time that kernel alone with
+ * cudaEventElapsedTime.  NULL events turn it off.  The events stay owned by
+ * the caller.  Returns PACE_ERR_INVALID_ARG for an unknown kernel. */
+PACE_API pace_status pace_set_profile_events(int32_t kernel, void* begin, void* end);
+
+/* Not part of the method: the number of CUDA kernels this library has
+ * launched from the calling host thread since it was loaded (memsets and
+ * copies are not kernels and are not counted). */
+PACE_API uint64_t pace_kernel_launches(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PACE_H_ */

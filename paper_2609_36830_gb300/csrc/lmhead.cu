@@ -1,0 +1,483 @@
+// Fused LM head: per-token log-probabilities under the current policy
+// (Sec. 2: the policy factorises over tokens, log pi_theta(y_t | x, y_<t);
+// training temperature from the shared settings), without writing logits.
+//
+// lmhead_lse_kernel (sm_103a, one CTA per SM, 192 threads, warp-specialised):
+//   warp 0 / lane 0   TMA producer: 128x64 hidden tile + 256x64 vocabulary tile
+//                     per K step into a 4-stage shared-memory ring (128-byte
+//                     swizzle), completion tracked by mbarrier transaction bytes.
+//   warp 1 / lane 0   MMA issuer: tcgen05.mma kind::f16 (bf16 x bf16 -> fp32),
+//                     M=128, N=256, K=16 per instruction, accumulating a
+//                     128x256 logit tile in tensor memory; two accumulators
+//                     (512 TMEM columns) so the epilogue of tile n overlaps
+//                     the MMAs of tile n+1.
+//   warps 2..5        epilogue: each thread owns one row (one TMEM lane),
+//                     reads its 256 logits 32 columns at a time with
+//                     tcgen05.ld, keeps a running base-2 max and sum of
+//                     exponentials (online log-sum-exp) and picks out the
+//                     target's logit.
+// A CTA covers 128 rows and one of S contiguous vocabulary splits; it writes
+// one (max, sum) pair per row and split.  Consecutive CTAs share a row block,
+// so the hidden tile they re-read stays in L2 while the vocabulary streams.
+//
+// lse_merge_kernel: per row, merges the S partial pairs into the log-sum-exp
+//   and writes lp = z_y / tau - lse.
+//
+// Every mbarrier wait is bounded (2 s); on timeout the CTA reports
+// PACE_ERR_TIMEOUT, stops issuing, waits (bounded) for its in-flight copies
+// and MMAs, frees its tensor memory and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include <mutex>
+
+#include "pace_internal.cuh"
+#include "pace_loss.cuh"
+
+namespace pace {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = 64;
+constexpr int STAGES = 4;
+constexpr int kThreads = 192;
+constexpr uint32_t kStageA = BM * BK * 2;  // 16 KB
+constexpr uint32_t kStageB = BN * BK * 2;  // 32 KB
+constexpr uint32_t kStageBytes = kStageA + kStageB;
+constexpr uint32_t kTmemCols = 2 * BN;     // two fp32 accumulators of 256 columns
+constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
+constexpr size_t kSmemBytes = 1024 /* alignment slack */ + STAGES * kStageBytes + 256;
+
+struct LmArgs {
+  int64_t rows_cap;             // rows of the A tensor map
+  const long long* n_valid_dev; // rows actually present (device), or null = rows_cap
+  int32_t H, V;
+  int32_t n_vtiles, splits, tiles_per_split;
+  float scale_log2;             // log2(e) / temperature
+  const int32_t* targets;
+  const int32_t* rowidx;        // compact row -> original row, or null (identity)
+  float* part_m;                // [rows_cap * splits]
+  float* part_s;
+  float* tgt_logit;             // [rows_cap]
+  int32_t* status;
+};
+
+__device__ __forceinline__ uint64_t make_policy_evict_last() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+__device__ __forceinline__ uint64_t make_policy_evict_normal() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    lmhead_lse_kernel(const __grid_constant__ CUtensorMap tm_a,
+                      const __grid_constant__ CUtensorMap tm_b, LmArgs p) {
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  unsigned char* stage_base = smem;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * kStageBytes);
+  uint64_t* full = bars;                  // [STAGES]
+  uint64_t* empty = bars + STAGES;        // [STAGES]
+  uint64_t* tmem_full = bars + 2 * STAGES;   // [2]
+  uint64_t* tmem_empty = tmem_full + 2;      // [2]
+  uint64_t* mma_done = tmem_empty + 2;       // [1]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int64_t row_block = blockIdx.x / p.splits;
+  const int split = blockIdx.x % p.splits;
+  const int64_t row0 = row_block * BM;
+  const int64_t n_valid = p.n_valid_dev ? static_cast<int64_t>(*p.n_valid_dev) : p.rows_cap;
+  if (row0 >= n_valid) return;  // uniform: nothing allocated yet
+  // after a timeout anywhere in the grid, the remaining CTAs do not start waiting
+  if (p.status && *reinterpret_cast<volatile int32_t*>(p.status) == PACE_ERR_TIMEOUT) return;
+  const int tile0 = split * p.tiles_per_split;
+  const int tile1 = min(tile0 + p.tiles_per_split, p.n_vtiles);
+  if (tile0 >= tile1) return;
+  const int num_tiles = tile1 - tile0;
+  const int nkb = p.H / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tmem_full[b], 1);
+      mbar_init(&tmem_empty[b], 4 * 32);
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      tma_prefetch_desc(&tm_a);
+      tma_prefetch_desc(&tm_b);
+      const uint64_t pol_a = make_policy_evict_last();
+      const uint64_t pol_b = make_policy_evict_normal();
+      uint32_t it = 0;
+      bool ok = true;
+      for (int t = 0; t < num_tiles && ok; ++t) {
+        const int32_t n0 = (tile0 + t) * BN;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const uint32_t s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1u;
+          if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          unsigned char* sa = stage_base + s * kStageBytes;
+          unsigned char* sb = sa + kStageA;
+          mbar_arrive_expect_tx(&full[s], kStageBytes);
+          tma_load_2d(sa, &tm_a, &full[s], kb * BK, static_cast<int32_t>(row0), pol_a);
+          tma_load_2d(sb, &tm_b, &full[s], kb * BK, n0, pol_b);
+        }
+      }
+      if (!ok) {
+        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+        *abort_flag = 1;
+      }
+      // Drain: every copy issued must have landed before the CTA exits.
+      for (uint32_t s = 0; s < STAGES && s < it; ++s) {
+        const uint32_t last = it - 1 - ((it - 1 - s) % STAGES);  // last index with stage s
+        mbar_wait_bounded(&full[s], (last / STAGES) & 1u, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      uint32_t it = 0;
+      bool ok = true;
+      for (int t = 0; t < num_tiles && ok; ++t) {
+        const uint32_t acc = t & 1;
+        const uint32_t acc_ph = (t >> 1) & 1u;
+        if (!mbar_wait_bounded(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const uint32_t s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1u;
+          if (!mbar_wait_bounded(&full[s], ph, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(stage_base + s * kStageBytes);
+          const uint32_t sb = sa + kStageA;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            tc_mma_f16(d_tmem, smem_desc_k128(sa + k * 32), smem_desc_k128(sb + k * 32), kIdesc,
+                       (kb > 0 || k > 0) ? 1u : 0u);
+          }
+          tc_commit(&empty[s]);  // frees the stage once these MMAs have read it
+        }
+        if (!ok) break;
+        tc_commit(&tmem_full[acc]);
+      }
+      if (!ok) {
+        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+        *abort_flag = 1;
+      }
+      // all MMAs issued by this thread complete before tensor memory is freed
+      tc_commit(mma_done);
+      mbar_wait_bounded(mma_done, 0, nullptr);
+    }
+  } else {
+    // ------------------------------------------------ epilogue (4 warps)
+    const int quad = warp & 3;  // TMEM lanes this warp may access
+    const int r_local = quad * 32 + lane;
+    const int64_t row = row0 + r_local;
+    const bool row_ok = row < n_valid;
+    int32_t y = -1;
+    if (row_ok) {
+      const int64_t orig = p.rowidx ? static_cast<int64_t>(p.rowidx[row]) : row;
+      y = p.targets[orig];
+    }
+    const float scale = p.scale_log2;
+    float m = -INFINITY, s = 0.0f, tgt = 0.0f;
+    bool have_tgt = false;
+    for (int t = 0; t < num_tiles; ++t) {
+      const uint32_t acc = t & 1;
+      const uint32_t acc_ph = (t >> 1) & 1u;
+      if (!mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag)) {
+        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+        *abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const int32_t n0 = (tile0 + t) * BN;
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * BN;
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        float v[32];
+        tmem_ld_32x32b_x32(tbase + c, v);
+        tmem_wait_ld();
+        const int32_t col0 = n0 + c;
+        if (col0 + 32 > p.V) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (col0 + i >= p.V) v[i] = -INFINITY;
+        }
+        float cm = v[0];
+#pragma unroll
+        for (int i = 1; i < 32; ++i) cm = fmaxf(cm, v[i]);
+        const float m_new = fmaxf(m, cm * scale);
+        float acc_s = 0.0f;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) acc_s += ex2_approx(fmaf(v[i], scale, -m_new));
+        s = s * ex2_approx(m - m_new) + acc_s;
+        m = m_new;
+        const uint32_t off = static_cast<uint32_t>(y - col0);
+        if (off < 32u) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (off == static_cast<uint32_t>(i)) tgt = v[i];
+          have_tgt = true;
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&tmem_empty[acc]);
+    }
+    if (row_ok) {
+      const int64_t o = row * p.splits + split;
+      p.part_m[o] = m;
+      p.part_s[o] = s;
+      if (have_tgt) p.tgt_logit[row] = tgt;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
+}
+
+// Per row in the loss: log-sum-exp from the split partials, then
+// lp = z_y / tau - lse, scattered back to the original row.
+__global__ void lse_merge_kernel(int64_t rows_cap, const long long* __restrict__ n_valid_dev,
+                                 int splits, int32_t V, float inv_temp,
+                                 const float* __restrict__ part_m, const float* __restrict__ part_s,
+                                 const float* __restrict__ tgt_logit,
+                                 const int32_t* __restrict__ targets,
+                                 const int32_t* __restrict__ rowidx, float* __restrict__ logprob,
+                                 float* __restrict__ lse_out, int32_t* status) {
+  const int64_t n_valid = n_valid_dev ? static_cast<int64_t>(*n_valid_dev) : rows_cap;
+  for (int64_t r = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; r < n_valid;
+       r += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t orig = rowidx ? static_cast<int64_t>(rowidx[r]) : r;
+    float mm = -INFINITY;
+    for (int s = 0; s < splits; ++s) mm = fmaxf(mm, part_m[r * splits + s]);
+    float ss = 0.0f;
+    for (int s = 0; s < splits; ++s) ss += part_s[r * splits + s] * ex2_approx(part_m[r * splits + s] - mm);
+    const float lse = (mm + lg2_approx(ss)) * 0.69314718055994531f;
+    const int32_t y = targets[orig];
+    float lp;
+    if (y < 0 || y >= V) {
+      report(status, PACE_ERR_INVALID_ARG);
+      lp = __int_as_float(0x7fc00000);
+    } else {
+      lp = tgt_logit[r] * inv_temp - lse;
+    }
+    logprob[orig] = lp;
+    if (lse_out) lse_out[orig] = lse;
+  }
+}
+
+// ---------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor [rows][H] (row-major), boxes of box_rows x 64 with the
+// 128-byte swizzle the UMMA descriptors expect.
+pace_status encode_bf16_2d(CUtensorMap* tm, const void* ptr, int64_t rows, int H, int box_rows) {
+  auto enc = get_encode_fn();
+  if (!enc) return PACE_ERR_CUDA;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(H) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? PACE_OK : PACE_ERR_UNSUPPORTED_SHAPE;
+}
+
+int choose_splits(int n_vtiles) {
+  int s = 4;
+  if (s > n_vtiles) s = n_vtiles;
+  if (s < 1) s = 1;
+  return s;
+}
+
+struct LmWs {
+  CompactWs cw;
+  SurrogateWs sw;
+  void* hidden_c;  // gathered rows [n_rows][H] (null when no compaction)
+  float* part_m;
+  float* part_s;
+  float* tgt;
+};
+
+void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, bool compact,
+                 LmWs* w) {
+  const int n_vtiles = (V + BN - 1) / BN;
+  const int S = choose_splits(n_vtiles);
+  const int64_t rows_cap = n_rows > BM ? n_rows : BM;
+  carve_compact_ws(cv, n_seq, n_rows, &w->cw);
+  carve_surrogate_ws(cv, n_seq, &w->sw);
+  w->hidden_c = compact ? static_cast<void*>(cv.take<uint16_t>(static_cast<size_t>(rows_cap) * H))
+                        : nullptr;
+  w->part_m = cv.take<float>(static_cast<size_t>(rows_cap) * S);
+  w->part_s = cv.take<float>(static_cast<size_t>(rows_cap) * S);
+  w->tgt = cv.take<float>(static_cast<size_t>(rows_cap));
+}
+
+pace_status set_smem_attr() {
+  static int done_dev = -1;
+  static std::mutex mu;
+  int dev = 0;
+  PACE_TRY_CUDA(cudaGetDevice(&dev));
+  std::lock_guard<std::mutex> g(mu);
+  if (done_dev == dev) return PACE_OK;
+  PACE_TRY_CUDA(cudaFuncSetAttribute(lmhead_lse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(kSmemBytes)));
+  done_dev = dev;
+  return PACE_OK;
+}
+
+}  // namespace
+}  // namespace pace
+
+using namespace pace;
+
+extern "C" size_t pace_token_logprob_workspace_size(int64_t n_rows, int64_t n_seq,
+                                                    int32_t hidden_size, int32_t vocab_size) {
+  if (n_rows < 0 || n_seq < 0 || hidden_size <= 0 || vocab_size <= 0) return 0;
+  Carver cv;
+  LmWs w;
+  carve_lm_ws(cv, n_rows, n_seq, hidden_size, vocab_size, true, &w);
+  return cv.used;
+}
+
+extern "C" pace_status pace_token_logprob(const PaceBatch* batch, const void* hidden,
+                                          const void* w_vocab, const int32_t* targets,
+                                          int32_t hidden_size, int32_t vocab_size,
+                                          float temperature, float* logprob, float* lse,
+                                          const PaceLossArgs* loss, void* workspace,
+                                          size_t workspace_bytes, int32_t* status_dev,
+                                          void* stream) {
+  PACE_TRY(check_batch(batch));
+  if (loss) PACE_TRY(check_loss_args(batch, loss));
+  const int H = hidden_size, V = vocab_size;
+  if (H < 64 || H > 16384 || H % 64 != 0) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (V < 1 || V > (1 << 24)) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (!(temperature > 0.0f) || !isfinite(temperature)) return PACE_ERR_INVALID_ARG;
+  const int64_t n_rows = batch->n_rows;
+  if (n_rows > 0 && (!hidden || !w_vocab || !targets || !logprob)) return PACE_ERR_INVALID_ARG;
+  if (!aligned(hidden, 16) || !aligned(w_vocab, 16)) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
+  cudaStream_t st = as_stream(stream);
+  // Compaction is skipped only when every row is in the loss and there are
+  // enough rows for a full TMA box.
+  const bool compact = batch->mask || batch->seq_accepted || n_rows < BM;
+  Carver cv(workspace, workspace_bytes);
+  LmWs ws;
+  carve_lm_ws(cv, n_rows, batch->n_seq, H, V, compact, &ws);
+  if (!cv.fits()) return PACE_ERR_WORKSPACE;
+
+  if (n_rows > 0) {
+    PACE_TRY_CUDA(cudaMemsetAsync(logprob, 0, static_cast<size_t>(n_rows) * sizeof(float), st));
+    if (lse) PACE_TRY_CUDA(cudaMemsetAsync(lse, 0, static_cast<size_t>(n_rows) * sizeof(float), st));
+  }
+  const void* a_ptr = hidden;
+  const long long* n_valid_dev = nullptr;
+  const int32_t* rowidx = nullptr;
+  int64_t rows_cap = n_rows;
+  if (compact) {
+    PACE_TRY(run_compaction(batch, ws.cw, status_dev, st));
+    PACE_TRY(run_gather(hidden, H, n_rows, ws.cw, ws.hidden_c, st));
+    a_ptr = ws.hidden_c;
+    n_valid_dev = ws.cw.total;
+    rowidx = ws.cw.rowidx;
+    rows_cap = n_rows > BM ? n_rows : BM;
+  }
+  if (n_rows > 0) {
+    const int n_vtiles = (V + BN - 1) / BN;
+    const int S = choose_splits(n_vtiles);
+    const int tps = (n_vtiles + S - 1) / S;
+    CUtensorMap tm_a, tm_b;
+    PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, BM));
+    PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, BN));
+    PACE_TRY(set_smem_attr());
+    LmArgs a;
+    a.rows_cap = rows_cap;
+    a.n_valid_dev = n_valid_dev;
+    a.H = H;
+    a.V = V;
+    a.n_vtiles = n_vtiles;
+    a.splits = S;
+    a.tiles_per_split = tps;
+    a.scale_log2 = 1.4426950408889634f / temperature;
+    a.targets = targets;
+    a.rowidx = rowidx;
+    a.part_m = ws.part_m;
+    a.part_s = ws.part_s;
+    a.tgt_logit = ws.tgt;
+    a.status = status_dev;
+    const int64_t row_blocks = (rows_cap + BM - 1) / BM;
+    const int64_t grid = row_blocks * S;
+    if (grid > 0x7fffffff) return PACE_ERR_UNSUPPORTED_SHAPE;
+    const ProfileEvents& pe = profile_events(PACE_PROFILE_LMHEAD);
+    if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
+    lmhead_lse_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tm_a, tm_b, a);
+    PACE_TRY(last_launch_status());
+    if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
+    int64_t mblocks = (rows_cap + 255) / 256;
+    const int64_t cap = static_cast<int64_t>(sm_count()) * 8;
+    if (mblocks > cap) mblocks = cap;
+    lse_merge_kernel<<<static_cast<unsigned>(mblocks), 256, 0, st>>>(
+        rows_cap, n_valid_dev, S, V, 1.0f / temperature, ws.part_m, ws.part_s, ws.tgt, targets,
+        rowidx, logprob, lse, status_dev);
+    PACE_TRY(last_launch_status());
+  }
+  if (loss) PACE_TRY(run_surrogate(batch, logprob, loss, ws.sw, status_dev, st));
+  return PACE_OK;
+}

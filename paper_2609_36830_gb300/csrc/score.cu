@@ -1,0 +1,369 @@
+// Pool scoring: Lemma 1 / Eq. 2 staleness decomposition, Eqs. 7-10 scores and
+// the per-group mean, on sm_103a.
+//
+//   tag_reduce_kernel   one streaming pass over the int32 version tags (HBM
+//                       bound): per trajectory the count T of policy tokens,
+//                       the exact integer sum of their tags and the largest
+//                       tag (+1, for the Lemma 1 premise check).
+//   score_finalize_kernel  one thread per trajectory: K_gen, K_wait, the ECDF
+//                       percentile q against the window (Eq. 9), F = phi(q)
+//                       (Eq. 10), the mode's score (Eqs. 7-8), and the mean of
+//                       each group of G in fixed left-to-right order.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "pace_internal.cuh"
+
+namespace pace {
+namespace {
+
+constexpr int kReduceThreads = 256;  // 8 warps
+constexpr int kTileTokens = 128;     // one int4 per lane
+constexpr int kTilesPerBatch = 8;    // 1024 tokens (4 KB) per warp batch in flight
+constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
+constexpr int kMaxWindow = 4096;
+
+__device__ __forceinline__ int4 ld_stream_v4(const int32_t* p) {
+  int4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.s32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+struct LaneAcc {
+  long long sum;   // sum of policy tags seen by this lane for the current trajectory
+  unsigned cnt;    // number of policy tokens
+  unsigned maxp1;  // max over policy tokens of (unsigned)v + 1 (0 if none)
+};
+
+__device__ __forceinline__ void acc_elem(LaneAcc& a, int32_t v, bool in_range) {
+  const bool in = in_range && (v != -1);
+  a.sum += in ? static_cast<long long>(v) : 0ll;
+  a.cnt += in ? 1u : 0u;
+  const unsigned vp1 = static_cast<unsigned>(v) + 1u;
+  a.maxp1 = (in && vp1 > a.maxp1) ? vp1 : a.maxp1;
+}
+
+// Warp-reduce the lane partials and add them to trajectory `traj`'s totals.
+// Integer adds and max are order-independent, so the totals are exact and
+// deterministic however trajectories are split across warps.
+__device__ __forceinline__ void flush(LaneAcc& a, int64_t traj, unsigned long long* sumv,
+                                      unsigned* cnt, unsigned* maxp1) {
+  const unsigned full = 0xffffffffu;
+  const bool any = __any_sync(full, a.cnt != 0u);
+  if (any) {
+    long long s = a.sum;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(full, s, o);
+    const unsigned c = __reduce_add_sync(full, a.cnt);
+    const unsigned m = __reduce_max_sync(full, a.maxp1);
+    if ((threadIdx.x & 31) == 0) {
+      atomicAdd(&sumv[traj], static_cast<unsigned long long>(s));
+      atomicAdd(&cnt[traj], c);
+      atomicMax(&maxp1[traj], m);
+    }
+  }
+  a.sum = 0;
+  a.cnt = 0;
+  a.maxp1 = 0;
+}
+
+// Each warp owns a contiguous range of 1024-token batches of the flattened
+// tag stream and walks the CSR offsets forward through it, so trajectories of
+// any length mix are balanced across warps.  The walk never leaves
+// [0, n_traj) and loads only tags[0, n_tokens), whatever the offsets hold;
+// inconsistent offsets are reported by the finalize kernel.
+__global__ void __launch_bounds__(kReduceThreads)
+    tag_reduce_kernel(const int32_t* __restrict__ tags, const int64_t* __restrict__ offsets,
+                      int64_t n_traj, int64_t n_tokens, unsigned long long* __restrict__ sumv,
+                      unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t n_warps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
+  const int64_t b_begin = n_batches * warp / n_warps;
+  const int64_t b_end = n_batches * (warp + 1) / n_warps;
+  if (b_begin >= b_end) return;
+  const int64_t t_begin = b_begin * kBatchTokens;
+
+  // trajectory holding token t_begin: largest i < n_traj with offsets[i] <= t_begin
+  int64_t lo = 0, hi = n_traj;
+  while (hi - lo > 1) {
+    const int64_t mid = lo + (hi - lo) / 2;
+    if (offsets[mid] <= t_begin) lo = mid;
+    else hi = mid;
+  }
+  int64_t cur = lo;
+  int64_t cur_end = offsets[cur + 1];
+  LaneAcc acc{0, 0u, 0u};
+
+  for (int64_t b = b_begin; b < b_end; ++b) {
+    const int64_t bt0 = b * kBatchTokens;
+    const int64_t bt1 = (bt0 + kBatchTokens < n_tokens) ? bt0 + kBatchTokens : n_tokens;
+    int4 v[kTilesPerBatch];
+#pragma unroll
+    for (int u = 0; u < kTilesPerBatch; ++u) {
+      const int64_t t = bt0 + u * kTileTokens + lane * 4;
+      if (t + 3 < n_tokens) {
+        v[u] = ld_stream_v4(tags + t);
+      } else {
+        v[u].x = (t + 0 < n_tokens) ? tags[t + 0] : -1;
+        v[u].y = (t + 1 < n_tokens) ? tags[t + 1] : -1;
+        v[u].z = (t + 2 < n_tokens) ? tags[t + 2] : -1;
+        v[u].w = (t + 3 < n_tokens) ? tags[t + 3] : -1;
+      }
+    }
+    int64_t pos = bt0;
+    while (true) {
+      const int64_t seg_hi = cur_end < bt1 ? cur_end : bt1;
+      if (pos == bt0 && seg_hi == bt1) {
+        // whole batch inside one trajectory: no position tests
+#pragma unroll
+        for (int u = 0; u < kTilesPerBatch; ++u) {
+          acc_elem(acc, v[u].x, true);
+          acc_elem(acc, v[u].y, true);
+          acc_elem(acc, v[u].z, true);
+          acc_elem(acc, v[u].w, true);
+        }
+      } else if (seg_hi > pos) {
+#pragma unroll
+        for (int u = 0; u < kTilesPerBatch; ++u) {
+          const int64_t t = bt0 + u * kTileTokens + lane * 4;
+          acc_elem(acc, v[u].x, t + 0 >= pos && t + 0 < seg_hi);
+          acc_elem(acc, v[u].y, t + 1 >= pos && t + 1 < seg_hi);
+          acc_elem(acc, v[u].z, t + 2 >= pos && t + 2 < seg_hi);
+          acc_elem(acc, v[u].w, t + 3 >= pos && t + 3 < seg_hi);
+        }
+      }
+      if (cur_end > bt1) break;  // trajectory continues into the next batch
+      flush(acc, cur, sumv, cnt, maxp1);
+      if (seg_hi > pos) pos = seg_hi;
+      ++cur;
+      if (cur >= n_traj) return;  // tokens past the last trajectory: offsets are bad
+      cur_end = offsets[cur + 1];
+      // the next trajectory starts at the batch edge: continue in the next batch;
+      // otherwise loop (more of this batch, or empty trajectories to step over)
+      if (pos >= bt1 && cur_end > bt1) break;
+    }
+  }
+  if (cur < n_traj) flush(acc, cur, sumv, cnt, maxp1);
+}
+
+struct FinalizeArgs {
+  const int64_t* offsets;
+  const int32_t* c_version;
+  const float* s_pre;
+  const float* window;
+  const unsigned long long* sumv;
+  const unsigned* cnt;
+  const unsigned* maxp1;
+  int64_t n_traj;
+  int64_t n_tokens;
+  int32_t j;
+  int32_t window_len;
+  int32_t window_ready;
+  int32_t mode;
+  int32_t gamma;
+  int32_t group_size;
+  double f_missing;
+  double* kgen;
+  double* kwait;
+  double* weight;
+  double* score;
+  double* unit_score;
+  int32_t* status;
+};
+
+// phi_gamma(q) of Eq. 10 with integer gamma, powers by repeated
+// multiplication, every operation rounded once (no FMA).
+__device__ __forceinline__ double sharpen(double q, int gamma) {
+  const double omq = __dsub_rn(1.0, q);
+  double a = q, b = omq;
+  for (int g = 1; g < gamma; ++g) {
+    a = __dmul_rn(a, q);
+    b = __dmul_rn(b, omq);
+  }
+  return __ddiv_rn(a, __dadd_rn(a, b));
+}
+
+__global__ void score_finalize_kernel(FinalizeArgs p) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int wpad = (p.window_len + 3) & ~3;
+  float* swin = reinterpret_cast<float*>(smem_raw);
+  double* sscore = reinterpret_cast<double*>(smem_raw + align_up(wpad * sizeof(float), 16));
+
+  if (p.window_ready) {
+    for (int k = threadIdx.x; k < wpad; k += blockDim.x) {
+      const float w = k < p.window_len ? p.window[k] : __int_as_float(0x7fc00000);  // NaN pad
+      swin[k] = w;
+      if (k < p.window_len && isnan(w)) report(p.status, PACE_ERR_NAN_INPUT);
+    }
+  }
+  __syncthreads();
+
+  const int G = p.group_size;
+  const int64_t per_block = blockDim.x;  // whole groups per block
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * per_block + threadIdx.x;
+  if (i < p.n_traj) {
+    const int64_t o0 = p.offsets[i], o1 = p.offsets[i + 1];
+    if (o1 < o0 || (i == 0 && o0 != 0) || (i == p.n_traj - 1 && o1 != p.n_tokens))
+      report(p.status, PACE_ERR_INVALID_ARG);
+    const int64_t c = p.c_version[i];
+    const unsigned t_count = p.cnt[i];
+    const unsigned mp1 = p.maxp1[i];
+    const long long tag_sum = static_cast<long long>(p.sumv[i]);
+    if (c < 0 || mp1 >= 0x80000000u) report(p.status, PACE_ERR_INVALID_ARG);
+    if (c > p.j || (mp1 != 0u && static_cast<int64_t>(mp1) - 1 > c))
+      report(p.status, PACE_ERR_VERSION_ORDER);
+    // Lemma 1: K_gen = (1/T) sum (c - v_t) = (c T - sum v_t) / T, exact integers
+    const long long gen_sum = static_cast<long long>(c) * static_cast<long long>(t_count) - tag_sum;
+    const double kgen =
+        t_count > 0u ? __ddiv_rn(__ll2double_rn(gen_sum), __ull2double_rn(t_count)) : 0.0;
+    const double kwait = __ll2double_rn(static_cast<long long>(p.j) - c);
+    double f;
+    if (!p.window_ready) {
+      f = 1.0;
+    } else {
+      const float s = p.s_pre ? p.s_pre[i] : __int_as_float(0x7fc00000);
+      if (isnan(s)) {
+        f = p.f_missing;
+      } else {
+        int count = 0;
+        const float4* w4 = reinterpret_cast<const float4*>(swin);
+        for (int k = 0; k < wpad / 4; ++k) {
+          const float4 w = w4[k];
+          count += (w.x <= s) + (w.y <= s) + (w.z <= s) + (w.w <= s);
+        }
+        const double q = __ddiv_rn(static_cast<double>(count), static_cast<double>(p.window_len));
+        f = sharpen(q, p.gamma);
+      }
+    }
+    double sc;
+    if (p.mode == PACE_SCORE_EFF) sc = __dadd_rn(kwait, __dmul_rn(f, kgen));
+    else if (p.mode == PACE_SCORE_RAW) sc = __dadd_rn(kwait, kgen);
+    else sc = __dmul_rn(f, kgen);
+    if (p.kgen) p.kgen[i] = kgen;
+    if (p.kwait) p.kwait[i] = kwait;
+    if (p.weight) p.weight[i] = f;
+    p.score[i] = sc;
+    sscore[threadIdx.x] = sc;
+  }
+  __syncthreads();
+  if (p.unit_score && i < p.n_traj && (threadIdx.x % G) == 0) {
+    double acc = 0.0;
+    for (int g = 0; g < G; ++g) acc = __dadd_rn(acc, sscore[threadIdx.x + g]);
+    p.unit_score[i / G] = __ddiv_rn(acc, static_cast<double>(G));
+  }
+}
+
+struct ScoreWs {
+  unsigned long long* sumv;
+  unsigned* cnt;
+  unsigned* maxp1;
+};
+
+ScoreWs carve_score_ws(Carver& cv, int64_t n_traj) {
+  ScoreWs w;
+  // one contiguous block so a single memset clears it
+  w.sumv = cv.take<unsigned long long>(static_cast<size_t>(n_traj) * 2);
+  w.cnt = w.sumv ? reinterpret_cast<unsigned*>(w.sumv + n_traj) : nullptr;
+  w.maxp1 = w.cnt ? w.cnt + n_traj : nullptr;
+  return w;
+}
+
+}  // namespace
+}  // namespace pace
+
+using namespace pace;
+
+extern "C" void pace_score_params_default(PaceScoreParams* p) {
+  if (!p) return;
+  p->mode = PACE_SCORE_EFF;
+  p->gamma = 4;
+  p->min_obs = 32;
+  p->group_size = 8;
+  p->f_missing = 1.0;
+}
+
+extern "C" size_t pace_score_pool_workspace_size(int64_t n_traj, int64_t window_len) {
+  (void)window_len;
+  if (n_traj < 0) return 0;
+  Carver cv;
+  carve_score_ws(cv, n_traj);
+  return cv.used;
+}
+
+extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offsets,
+                                       const int32_t* c_version, const float* s_pre,
+                                       int64_t n_traj, int64_t n_tokens, int32_t trainer_version,
+                                       const float* window, int64_t window_len,
+                                       const PaceScoreParams* params, double* kgen,
+                                       double* kwait, double* weight, double* score,
+                                       double* unit_score, void* workspace,
+                                       size_t workspace_bytes, int32_t* status_dev,
+                                       void* stream) {
+  if (!params || !offsets || !c_version || !score) return PACE_ERR_INVALID_ARG;
+  if (n_traj < 0 || n_tokens < 0 || n_traj > (int64_t(1) << 31)) return PACE_ERR_INVALID_ARG;
+  if (n_tokens > 0 && !tags) return PACE_ERR_INVALID_ARG;
+  const int G = params->group_size;
+  if (G < 1 || G > 1024 || n_traj % G != 0) return PACE_ERR_INVALID_ARG;
+  if (params->gamma < 1 || params->gamma > 64) return PACE_ERR_INVALID_ARG;
+  if (params->mode != PACE_SCORE_EFF && params->mode != PACE_SCORE_RAW &&
+      params->mode != PACE_SCORE_GEN)
+    return PACE_ERR_INVALID_ARG;
+  if (window_len < 0 || window_len > kMaxWindow) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (window_len > 0 && !window) return PACE_ERR_INVALID_ARG;
+  if (tags && !aligned(tags, 16)) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (n_traj == 0) return PACE_OK;
+  if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
+  Carver cv(workspace, workspace_bytes);
+  ScoreWs ws = carve_score_ws(cv, n_traj);
+  if (!cv.fits()) return PACE_ERR_WORKSPACE;
+
+  cudaStream_t st = as_stream(stream);
+  PACE_TRY_CUDA(cudaMemsetAsync(ws.sumv, 0, static_cast<size_t>(n_traj) * 16, st));
+  if (n_tokens > 0) {
+    const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
+    const int warps_per_block = kReduceThreads / 32;
+    int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
+    const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
+    if (blocks > cap) blocks = cap;
+    const ProfileEvents& pe = profile_events(PACE_PROFILE_TAG_REDUCE);
+    if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
+    tag_reduce_kernel<<<static_cast<unsigned>(blocks), kReduceThreads, 0, st>>>(
+        tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1);
+    PACE_TRY(last_launch_status());
+    if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
+  }
+  FinalizeArgs a;
+  a.offsets = offsets;
+  a.c_version = c_version;
+  a.s_pre = s_pre;
+  a.window = window;
+  a.sumv = ws.sumv;
+  a.cnt = ws.cnt;
+  a.maxp1 = ws.maxp1;
+  a.n_traj = n_traj;
+  a.n_tokens = n_tokens;
+  a.j = trainer_version;
+  a.window_len = static_cast<int32_t>(window_len);
+  a.window_ready = (window_len > 0 && window_len >= params->min_obs) ? 1 : 0;
+  a.mode = params->mode;
+  a.gamma = params->gamma;
+  a.group_size = G;
+  a.f_missing = params->f_missing;
+  a.kgen = kgen;
+  a.kwait = kwait;
+  a.weight = weight;
+  a.score = score;
+  a.unit_score = unit_score;
+  a.status = status_dev;
+  const int units_per_block = G >= 256 ? 1 : 256 / G;
+  const int threads = units_per_block * G;
+  const int64_t blocks = (n_traj + threads - 1) / threads;
+  const size_t smem = align_up(((window_len + 3) & ~3) * sizeof(float), 16) +
+                      static_cast<size_t>(threads) * sizeof(double);
+  score_finalize_kernel<<<static_cast<unsigned>(blocks), threads, smem, st>>>(a);
+  return last_launch_status();
+}

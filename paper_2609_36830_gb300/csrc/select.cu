@@ -1,0 +1,442 @@
+// Rejection budget (Eqs. 3-4, host) and deterministic top-k rejection of
+// units (Sec. 3.1 quantile rule read as "reject the r-hat fraction of the
+// current pool with the largest scores"; Algorithm 1, trainer side).
+//
+// Order: score descending, then unit id ascending.  The k first units in that
+// order are rejected; outputs list trajectory ids ascending.
+//
+//   small pools (U <= 512): one block ranks every unit against every other
+//     unit in shared memory and compacts the ids (one launch).
+//   large pools: MSB-first radix select over order-preserving 64-bit keys
+//     (six 11/10-bit digit passes, each a histogram + a one-block pick), then
+//     a three-phase scan compaction that rejects the units above the pivot
+//     and the lowest-id units equal to it.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "pace_internal.cuh"
+
+namespace pace {
+namespace {
+
+constexpr int kSmallMax = 512;
+constexpr int kSmallThreads = 512;
+constexpr int kHistBins = 2048;
+constexpr int kTile = 2048;  // units per compaction block
+constexpr int kTileThreads = 256;
+constexpr int kPerThread = kTile / kTileThreads;
+constexpr int kPasses = 6;
+__constant__ int c_shift[kPasses] = {53, 42, 31, 20, 10, 0};
+__constant__ int c_width[kPasses] = {11, 11, 11, 11, 10, 10};
+
+// Order-preserving map of a double to uint64 (after folding -0.0 into +0.0),
+// so unsigned key order equals numeric order for every non-NaN value.
+__device__ __forceinline__ uint64_t order_key(double x) {
+  uint64_t b = static_cast<uint64_t>(__double_as_longlong(x));
+  if (b == 0x8000000000000000ull) b = 0;
+  return (b & 0x8000000000000000ull) ? ~b : (b | 0x8000000000000000ull);
+}
+
+struct SelectState {
+  unsigned long long prefix;
+  unsigned long long mask;
+  long long k_rem;
+  int done;
+  int pad;
+};
+
+// Block-wide exclusive scan of one value per thread (blockDim.x a multiple of
+// 32, <= 1024).  Returns the exclusive prefix; *total gets the block sum.
+template <typename T>
+__device__ T block_exclusive_scan(T v, T* total) {
+  __shared__ T warp_sums[32];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  T x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const T y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sums[wid] = x;
+  __syncthreads();
+  const int nw = blockDim.x >> 5;
+  if (wid == 0) {
+    T w = lane < nw ? warp_sums[lane] : T(0);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const T y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < nw) warp_sums[lane] = w;  // inclusive
+  }
+  __syncthreads();
+  const T before = wid > 0 ? warp_sums[wid - 1] : T(0);
+  if (total) *total = warp_sums[nw - 1];
+  __syncthreads();
+  return before + x - v;
+}
+
+__device__ __forceinline__ void write_unit(int64_t u, bool rejected, int64_t rej_pos,
+                                           int64_t acc_pos, int G, int32_t* accepted_ids,
+                                           int32_t* rejected_ids, uint8_t* flags) {
+  for (int g = 0; g < G; ++g) {
+    const int64_t id = u * G + g;
+    if (rejected) {
+      if (rejected_ids) rejected_ids[rej_pos * G + g] = static_cast<int32_t>(id);
+    } else {
+      accepted_ids[acc_pos * G + g] = static_cast<int32_t>(id);
+    }
+    if (flags) flags[id] = rejected ? 0 : 1;
+  }
+}
+
+// U <= 512: rank of u = number of units ordered before it.
+__global__ void __launch_bounds__(kSmallThreads)
+    select_small_kernel(const double* __restrict__ score, int n_units, int G, int64_t k,
+                        int32_t* accepted_ids, int32_t* rejected_ids, uint8_t* flags,
+                        int32_t* status) {
+  __shared__ double s[kSmallMax];
+  for (int u = threadIdx.x; u < n_units; u += blockDim.x) {
+    double x = score[u];
+    if (isnan(x)) report(status, PACE_ERR_NAN_INPUT);
+    s[u] = x;
+  }
+  __syncthreads();
+  const int u = threadIdx.x;
+  int rejected = 0;
+  if (u < n_units) {
+    const double x = s[u];
+    int rank = 0;
+    for (int w = 0; w < n_units; ++w) {
+      const double y = s[w];
+      rank += (y > x) || (y == x && w < u);
+    }
+    rejected = rank < k;
+  }
+  int n_rej = 0;
+  const int rej_before = block_exclusive_scan<int>(rejected, &n_rej);
+  if (u < n_units)
+    write_unit(u, rejected, rej_before, u - rej_before, G, accepted_ids, rejected_ids, flags);
+}
+
+__global__ void radix_hist_kernel(const double* __restrict__ score, int64_t n_units, int pass,
+                                  const SelectState* __restrict__ state,
+                                  unsigned* __restrict__ hist, int32_t* status) {
+  __shared__ unsigned h[kHistBins];
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) h[b] = 0;
+  __syncthreads();
+  const unsigned long long prefix = state->prefix, mask = state->mask;
+  const int shift = c_shift[pass];
+  const unsigned dmask = (1u << c_width[pass]) - 1u;
+  for (int64_t u = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; u < n_units;
+       u += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const double x = score[u];
+    if (pass == 0 && isnan(x)) report(status, PACE_ERR_NAN_INPUT);
+    const uint64_t key = order_key(x);
+    if ((key & mask) == prefix) atomicAdd(&h[(key >> shift) & dmask], 1u);
+  }
+  __syncthreads();
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x)
+    if (h[b]) atomicAdd(&hist[b], h[b]);
+}
+
+// One block of 1024 threads: find the digit holding the k_rem-th largest key
+// among those matching the prefix, narrow the prefix, clear the histogram.
+// Thread t owns digits nbins-1-2t and nbins-2-2t, so an exclusive scan in
+// thread order counts the matching keys with larger digits.
+__global__ void __launch_bounds__(1024) radix_pick_kernel(int pass, SelectState* state,
+                                                          unsigned* hist) {
+  __shared__ long long s_krem;
+  const int shift = c_shift[pass];
+  const int nbins = 1 << c_width[pass];
+  const int d1 = nbins - 1 - 2 * static_cast<int>(threadIdx.x);
+  const int d2 = d1 - 1;
+  const long long h1 = d1 >= 0 ? hist[d1] : 0;
+  const long long h2 = d2 >= 0 ? hist[d2] : 0;
+  if (threadIdx.x == 0) s_krem = state->k_rem;
+  __syncthreads();
+  const long long k_rem = s_krem;
+  const long long above = block_exclusive_scan<long long>(h1 + h2, nullptr);
+  int digit = -1;
+  long long left = 0;
+  if (d1 >= 0 && above < k_rem && k_rem <= above + h1) {
+    digit = d1;
+    left = k_rem - above;
+  } else if (d2 >= 0 && above + h1 < k_rem && k_rem <= above + h1 + h2) {
+    digit = d2;
+    left = k_rem - above - h1;
+  }
+  if (digit >= 0) {  // exactly one thread
+    state->prefix |= static_cast<unsigned long long>(digit) << shift;
+    state->mask |= static_cast<unsigned long long>(nbins - 1) << shift;
+    state->k_rem = left;
+  }
+  if (d1 >= 0) hist[d1] = 0;
+  if (d2 >= 0) hist[d2] = 0;
+}
+
+// Phase 1: per tile, units equal to the pivot and above it.
+__global__ void __launch_bounds__(kTileThreads)
+    count_tile_kernel(const double* __restrict__ score, int64_t n_units,
+                      const SelectState* __restrict__ state, int* eq_cnt, int* gt_cnt) {
+  const unsigned long long pivot = state->prefix;
+  int eq = 0, gt = 0;
+  const int64_t base = static_cast<int64_t>(blockIdx.x) * kTile + threadIdx.x * kPerThread;
+  for (int i = 0; i < kPerThread; ++i) {
+    const int64_t u = base + i;
+    if (u < n_units) {
+      const uint64_t key = order_key(score[u]);
+      eq += key == pivot;
+      gt += key > pivot;
+    }
+  }
+  int te = 0, tg = 0;
+  block_exclusive_scan<int>(eq, &te);
+  block_exclusive_scan<int>(gt, &tg);
+  if (threadIdx.x == 0) {
+    eq_cnt[blockIdx.x] = te;
+    gt_cnt[blockIdx.x] = tg;
+  }
+}
+
+// Phase 2 (one block): per tile, ties before it and rejections before it.
+__global__ void __launch_bounds__(1024)
+    scan_tiles_kernel(int n_tiles, const SelectState* __restrict__ state, const int* eq_cnt,
+                      const int* gt_cnt, long long* eq_before, long long* rej_before) {
+  __shared__ long long carry_eq, carry_rej;
+  if (threadIdx.x == 0) {
+    carry_eq = 0;
+    carry_rej = 0;
+  }
+  __syncthreads();
+  const long long k_rem = state->k_rem;
+  for (int t0 = 0; t0 < n_tiles; t0 += blockDim.x) {
+    const int t = t0 + threadIdx.x;
+    const int e = t < n_tiles ? eq_cnt[t] : 0;
+    int te = 0;
+    const int eb = block_exclusive_scan<int>(e, &te);
+    const long long eq_b = carry_eq + eb;
+    long long take = k_rem - eq_b;
+    take = take < 0 ? 0 : (take > e ? e : take);
+    const int r = t < n_tiles ? gt_cnt[t] + static_cast<int>(take) : 0;
+    int tr = 0;
+    const int rb = block_exclusive_scan<int>(r, &tr);
+    if (t < n_tiles) {
+      eq_before[t] = eq_b;
+      rej_before[t] = carry_rej + rb;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      carry_eq += te;
+      carry_rej += tr;
+    }
+    __syncthreads();
+  }
+}
+
+// Phase 3: flags and output positions inside each tile.
+__global__ void __launch_bounds__(kTileThreads)
+    write_tile_kernel(const double* __restrict__ score, int64_t n_units, int G,
+                      const SelectState* __restrict__ state, const long long* eq_before,
+                      const long long* rej_before, int32_t* accepted_ids,
+                      int32_t* rejected_ids, uint8_t* flags) {
+  const unsigned long long pivot = state->prefix;
+  const long long k_rem = state->k_rem;
+  const int64_t base = static_cast<int64_t>(blockIdx.x) * kTile + threadIdx.x * kPerThread;
+  uint64_t keys[kPerThread];
+  int eq = 0;
+  for (int i = 0; i < kPerThread; ++i) {
+    const int64_t u = base + i;
+    keys[i] = u < n_units ? order_key(score[u]) : 0;
+    eq += (u < n_units) && keys[i] == pivot;
+  }
+  const long long tie0 = eq_before[blockIdx.x] + block_exclusive_scan<int>(eq, nullptr);
+  bool rej[kPerThread];
+  int nrej = 0;
+  long long tie = tie0;
+  for (int i = 0; i < kPerThread; ++i) {
+    const int64_t u = base + i;
+    bool r = false;
+    if (u < n_units) {
+      if (keys[i] > pivot) r = true;
+      else if (keys[i] == pivot) r = (tie++) < k_rem;
+    }
+    rej[i] = r;
+    nrej += r;
+  }
+  long long rpos = rej_before[blockIdx.x] + block_exclusive_scan<int>(nrej, nullptr);
+  for (int i = 0; i < kPerThread; ++i) {
+    const int64_t u = base + i;
+    if (u >= n_units) break;
+    const long long apos = u - rpos;
+    write_unit(u, rej[i], rpos, apos, G, accepted_ids, rejected_ids, flags);
+    rpos += rej[i];
+  }
+}
+
+__global__ void fill_identity_kernel(int64_t n_units, int G, bool accept, int32_t* accepted_ids,
+                                     int32_t* rejected_ids, uint8_t* flags) {
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_units * G;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    if (accept) accepted_ids[i] = static_cast<int32_t>(i);
+    else if (rejected_ids) rejected_ids[i] = static_cast<int32_t>(i);
+    if (flags) flags[i] = accept ? 1 : 0;
+  }
+}
+
+__global__ void nan_check_kernel(const double* __restrict__ score, int64_t n, int32_t* status) {
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    if (isnan(score[i])) report(status, PACE_ERR_NAN_INPUT);
+}
+
+struct SelectWs {
+  SelectState* state;
+  unsigned* hist;
+  int* eq_cnt;
+  int* gt_cnt;
+  long long* eq_before;
+  long long* rej_before;
+};
+
+SelectWs carve_select_ws(Carver& cv, int64_t n_units) {
+  const int64_t n_tiles = (n_units + kTile - 1) / kTile;
+  SelectWs w;
+  w.state = cv.take<SelectState>(1);
+  w.hist = cv.take<unsigned>(kHistBins);
+  w.eq_cnt = cv.take<int>(n_tiles);
+  w.gt_cnt = cv.take<int>(n_tiles);
+  w.eq_before = cv.take<long long>(n_tiles);
+  w.rej_before = cv.take<long long>(n_tiles);
+  return w;
+}
+
+int grid_for(int64_t n, int threads, int per_sm) {
+  int64_t b = (n + threads - 1) / threads;
+  const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;
+  if (b > cap) b = cap;
+  if (b < 1) b = 1;
+  return static_cast<int>(b);
+}
+
+}  // namespace
+}  // namespace pace
+
+using namespace pace;
+
+extern "C" void pace_budget_params_default(PaceBudgetParams* p) {
+  if (!p) return;
+  p->n_target = 0;
+  p->beta = 0.0;
+  p->r_max = 0.9;
+  p->r_hat_prev = 0.0;
+}
+
+extern "C" pace_status pace_budget(int64_t n_traj, int64_t n_units, const PaceBudgetParams* p,
+                                   double* r_out, double* r_hat_out, int64_t* k_units_out) {
+  if (!p || !r_hat_out || !k_units_out) return PACE_ERR_INVALID_ARG;
+  if (n_traj < 0 || n_units < 0 || p->n_target < 0) return PACE_ERR_INVALID_ARG;
+  if (!(p->beta >= 0.0 && p->beta < 1.0)) return PACE_ERR_INVALID_ARG;
+  if (!(p->r_max >= 0.0 && p->r_max <= 1.0)) return PACE_ERR_INVALID_ARG;
+  if (!(p->r_hat_prev >= 0.0 && p->r_hat_prev <= 1.0)) return PACE_ERR_INVALID_ARG;
+  // Eq. 3: surplus fraction of the pool above its target occupancy
+  const int64_t denom = n_traj > 1 ? n_traj : 1;
+  volatile double r = static_cast<double>(n_traj - p->n_target) / static_cast<double>(denom);
+  double rr = r;
+  if (rr < 0.0) rr = 0.0;
+  if (rr > 1.0) rr = 1.0;
+  // Eq. 4: EMA smoothing; each product rounded on its own (no contraction)
+  volatile double t1 = p->beta * p->r_hat_prev;
+  volatile double one_minus_beta = 1.0 - p->beta;
+  volatile double t2 = one_minus_beta * rr;
+  const double r_hat = t1 + t2;
+  const double r_eff = r_hat < p->r_max ? r_hat : p->r_max;
+  volatile double prod = r_eff * static_cast<double>(n_units);
+  int64_t k = static_cast<int64_t>(floor(prod + 1e-9));
+  if (k > n_units) k = n_units;
+  if (k < 0) k = 0;
+  if (r_out) *r_out = rr;
+  *r_hat_out = r_hat;
+  *k_units_out = k;
+  return PACE_OK;
+}
+
+extern "C" size_t pace_select_workspace_size(int64_t n_units) {
+  if (n_units < 0) return 0;
+  Carver cv;
+  carve_select_ws(cv, n_units);
+  return cv.used;
+}
+
+extern "C" pace_status pace_select_k(const double* unit_score, int64_t n_units, int32_t group_size,
+                                     int64_t k, int32_t* accepted_ids, int32_t* rejected_ids,
+                                     uint8_t* traj_accepted, void* workspace,
+                                     size_t workspace_bytes, int32_t* status_dev, void* stream) {
+  if (n_units < 0 || group_size < 1 || k < 0 || k > n_units) return PACE_ERR_INVALID_ARG;
+  if (n_units > (int64_t(1) << 30) ||
+      n_units * static_cast<int64_t>(group_size) > (int64_t(1) << 31) - 1)
+    return PACE_ERR_INVALID_ARG;
+  if (n_units == 0) return PACE_OK;
+  if (!unit_score || (!accepted_ids && k < n_units)) return PACE_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream);
+  const int G = group_size;
+  if (k == 0 || k == n_units) {
+    nan_check_kernel<<<grid_for(n_units, 256, 4), 256, 0, st>>>(unit_score, n_units, status_dev);
+    PACE_TRY(last_launch_status());
+    fill_identity_kernel<<<grid_for(n_units * G, 256, 8), 256, 0, st>>>(
+        n_units, G, k == 0, accepted_ids, rejected_ids, traj_accepted);
+    return last_launch_status();
+  }
+  if (n_units <= kSmallMax) {
+    select_small_kernel<<<1, kSmallThreads, 0, st>>>(unit_score, static_cast<int>(n_units), G, k,
+                                                     accepted_ids, rejected_ids, traj_accepted,
+                                                     status_dev);
+    return last_launch_status();
+  }
+  if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
+  Carver cv(workspace, workspace_bytes);
+  SelectWs ws = carve_select_ws(cv, n_units);
+  if (!cv.fits()) return PACE_ERR_WORKSPACE;
+  SelectState init{0ull, 0ull, static_cast<long long>(k), 0, 0};
+  PACE_TRY_CUDA(cudaMemcpyAsync(ws.state, &init, sizeof(init), cudaMemcpyHostToDevice, st));
+  PACE_TRY_CUDA(cudaMemsetAsync(ws.hist, 0, kHistBins * sizeof(unsigned), st));
+  const int hist_grid = grid_for(n_units, 256, 2);
+  for (int pass = 0; pass < kPasses; ++pass) {
+    radix_hist_kernel<<<hist_grid, 256, 0, st>>>(unit_score, n_units, pass, ws.state, ws.hist,
+                                                 status_dev);
+    PACE_TRY(last_launch_status());
+    radix_pick_kernel<<<1, 1024, 0, st>>>(pass, ws.state, ws.hist);
+    PACE_TRY(last_launch_status());
+  }
+  const int64_t n_tiles = (n_units + kTile - 1) / kTile;
+  count_tile_kernel<<<static_cast<unsigned>(n_tiles), kTileThreads, 0, st>>>(
+      unit_score, n_units, ws.state, ws.eq_cnt, ws.gt_cnt);
+  PACE_TRY(last_launch_status());
+  scan_tiles_kernel<<<1, 1024, 0, st>>>(static_cast<int>(n_tiles), ws.state, ws.eq_cnt,
+                                        ws.gt_cnt, ws.eq_before, ws.rej_before);
+  PACE_TRY(last_launch_status());
+  write_tile_kernel<<<static_cast<unsigned>(n_tiles), kTileThreads, 0, st>>>(
+      unit_score, n_units, G, ws.state, ws.eq_before, ws.rej_before, accepted_ids, rejected_ids,
+      traj_accepted);
+  return last_launch_status();
+}
+
+extern "C" pace_status pace_select(const double* unit_score, int64_t n_units, int32_t group_size,
+                                   const PaceBudgetParams* budget, double* r_hat_out,
+                                   int64_t* k_units_out, int32_t* accepted_ids,
+                                   int32_t* rejected_ids, uint8_t* traj_accepted,
+                                   void* workspace, size_t workspace_bytes, int32_t* status_dev,
+                                   void* stream) {
+  if (!budget || !r_hat_out || !k_units_out || group_size < 1 || n_units < 0)
+    return PACE_ERR_INVALID_ARG;
+  double r_hat = 0.0;
+  int64_t k = 0;
+  PACE_TRY(pace_budget(n_units * static_cast<int64_t>(group_size), n_units, budget, nullptr,
+                       &r_hat, &k));
+  PACE_TRY(pace_select_k(unit_score, n_units, group_size, k, accepted_ids, rejected_ids,
+                         traj_accepted, workspace, workspace_bytes, status_dev, stream));
+  *r_hat_out = r_hat;
+  *k_units_out = k;
+  return PACE_OK;
+}

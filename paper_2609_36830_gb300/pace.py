@@ -1,0 +1,324 @@
+"""Python binding of libpace (include/pace.h): argument marshalling only.
+
+Every step of the path runs in the library's CUDA kernels; torch provides the
+device memory (outputs and workspace are allocated here, never by the library)
+and the current stream.  Loading fails loudly if the library was not built:
+there is no fallback of any kind.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Optional
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libpace.so")
+_lock = threading.Lock()
+_lib = None
+
+# status codes (include/pace.h)
+OK = 0
+ERR_INVALID_ARG = 1
+ERR_VERSION_ORDER = 2
+ERR_NAN_INPUT = 3
+ERR_UNSUPPORTED_SHAPE = 4
+ERR_WORKSPACE = 5
+ERR_TIMEOUT = 6
+ERR_CUDA = 7
+
+SCORE_EFF, SCORE_RAW, SCORE_GEN = 0, 1, 2
+PROFILE_LMHEAD, PROFILE_TAG_REDUCE = 0, 1
+AGG_TOKEN_MEAN, AGG_SEQ_MEAN_TOKEN_MEAN = 0, 1
+
+_P = ctypes.c_void_p
+_I32, _I64, _F32, _F64 = ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_double
+_SZ = ctypes.c_size_t
+
+
+class PaceScoreParams(ctypes.Structure):
+    _fields_ = [("mode", _I32), ("gamma", _I32), ("min_obs", _I32), ("group_size", _I32),
+                ("f_missing", _F64)]
+
+
+class PaceBudgetParams(ctypes.Structure):
+    _fields_ = [("n_target", _I64), ("beta", _F64), ("r_max", _F64), ("r_hat_prev", _F64)]
+
+
+class PaceLossParams(ctypes.Structure):
+    _fields_ = [("eps_low", _F32), ("eps_high", _F32), ("dual_clip", _F32), ("adv_eps", _F32),
+                ("agg", _I32), ("std_unbiased", _I32)]
+
+
+class PaceBatch(ctypes.Structure):
+    _fields_ = [("seq_offsets", _P), ("seq_accepted", _P), ("mask", _P), ("n_seq", _I64),
+                ("n_rows", _I64)]
+
+
+class PaceLossArgs(ctypes.Structure):
+    _fields_ = [("behav_lp", _P), ("reward", _P), ("group_size", _I32),
+                ("params", PaceLossParams), ("loss", _P), ("adv", _P), ("ratio", _P)]
+
+
+# every symbol include/pace.h declares, with its C signature
+SIGNATURES = {
+    "pace_status_string": ([_I32], ctypes.c_char_p),
+    "pace_version": ([], _I32),
+    "pace_score_params_default": ([_P], None),
+    "pace_score_pool": ([_P, _P, _P, _P, _I64, _I64, _I32, _P, _I64, _P, _P, _P, _P, _P, _P, _P,
+                         _SZ, _P, _P], _I32),
+    "pace_score_pool_workspace_size": ([_I64, _I64], _SZ),
+    "pace_budget_params_default": ([_P], None),
+    "pace_budget": ([_I64, _I64, _P, _P, _P, _P], _I32),
+    "pace_select": ([_P, _I64, _I32, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P], _I32),
+    "pace_select_k": ([_P, _I64, _I32, _I64, _P, _P, _P, _P, _SZ, _P, _P], _I32),
+    "pace_select_workspace_size": ([_I64], _SZ),
+    "pace_loss_params_default": ([_P], None),
+    "pace_group_advantages": ([_P, _P, _I64, _I32, _F32, _I32, _P, _P], _I32),
+    "pace_token_logprob": ([_P, _P, _P, _P, _I32, _I32, _F32, _P, _P, _P, _P, _SZ, _P, _P],
+                           _I32),
+    "pace_token_logprob_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
+    "pace_surrogate_loss": ([_P, _P, _P, _P, _SZ, _P, _P], _I32),
+    "pace_surrogate_loss_workspace_size": ([_I64, _I64], _SZ),
+    "pace_set_profile_events": ([_I32, _P, _P], _I32),
+    "pace_kernel_launches": ([], ctypes.c_uint64),
+}
+
+
+class PaceError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+def lib():
+    """The loaded libpace.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(
+                    f"{LIB_PATH} is missing: build it with "
+                    "`python -c 'import __graft_entry__ as g; g.build()'` "
+                    "(there is no fallback implementation)")
+            L = ctypes.CDLL(LIB_PATH)
+            for name, (args, res) in SIGNATURES.items():
+                fn = getattr(L, name)
+                fn.argtypes = args
+                fn.restype = res
+            _lib = L
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return lib().pace_status_string(int(status)).decode()
+
+
+def _check(st: int, where: str):
+    if st != OK:
+        raise PaceError(st, where)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dev(t: torch.Tensor):
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return t
+
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    """A caller-owned workspace buffer (torch's allocator aligns to >= 256 bytes)."""
+    return torch.empty(max(int(nbytes), 1), dtype=torch.uint8, device=device)
+
+
+def new_status(device) -> torch.Tensor:
+    return torch.zeros(1, dtype=torch.int32, device=device)
+
+
+def check_status(status: torch.Tensor, where: str = "device"):
+    """Synchronises and raises if a device-side error was recorded."""
+    v = int(status.item())
+    _check(v, where)
+
+
+# ---------------------------------------------------------------- (a) pool
+
+def score_params(mode=SCORE_EFF, gamma=4, min_obs=32, group_size=8, f_missing=1.0):
+    return PaceScoreParams(int(mode), int(gamma), int(min_obs), int(group_size),
+                           float(f_missing))
+
+
+def score_pool(tags, offsets, c_version, s_pre, trainer_version, window, params=None,
+               out=None, ws=None, status=None, stream=None):
+    """pace_score_pool.  Returns dict kgen, kwait, weight, score, unit_score (float64)."""
+    p = params or score_params()
+    dev = offsets.device
+    n = offsets.numel() - 1
+    if out is None:
+        out = {k: torch.empty(n, dtype=torch.float64, device=dev)
+               for k in ("kgen", "kwait", "weight", "score")}
+        out["unit_score"] = torch.empty(n // max(p.group_size, 1), dtype=torch.float64,
+                                        device=dev)
+    wl = 0 if window is None else window.numel()
+    if ws is None:
+        ws = workspace(lib().pace_score_pool_workspace_size(n, wl), dev)
+    st = lib().pace_score_pool(
+        _ptr(tags), _ptr(_dev(offsets)), _ptr(_dev(c_version)), _ptr(s_pre), n, tags.numel(),
+        int(trainer_version), _ptr(window), wl, ctypes.byref(p), _ptr(out.get("kgen")),
+        _ptr(out.get("kwait")), _ptr(out.get("weight")), _ptr(out["score"]),
+        _ptr(out.get("unit_score")), _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    _check(st, "pace_score_pool")
+    return out
+
+
+def budget_params(n_target, beta=0.0, r_max=0.9, r_hat_prev=0.0):
+    return PaceBudgetParams(int(n_target), float(beta), float(r_max), float(r_hat_prev))
+
+
+def budget(n_traj, n_units, params):
+    """pace_budget (host only): (r, r_hat, k_units)."""
+    r, rh, k = _F64(), _F64(), _I64()
+    st = lib().pace_budget(int(n_traj), int(n_units), ctypes.byref(params), ctypes.byref(r),
+                           ctypes.byref(rh), ctypes.byref(k))
+    _check(st, "pace_budget")
+    return r.value, rh.value, k.value
+
+
+def select(unit_score, group_size, params, out=None, ws=None, status=None, stream=None):
+    """pace_select: budget on the host, rejection on the device.
+
+    Returns (r_hat, k_units, accepted_ids, rejected_ids, traj_accepted) where the id
+    tensors are views of the first (U-k)*G / k*G entries of full-size buffers.
+    """
+    dev = unit_score.device
+    u = unit_score.numel()
+    n = u * group_size
+    if out is None:
+        out = {"accepted": torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               "rejected": torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               "flags": torch.empty(max(n, 1), dtype=torch.uint8, device=dev)}
+    if ws is None:
+        ws = workspace(lib().pace_select_workspace_size(u), dev)
+    rh, k = _F64(), _I64()
+    st = lib().pace_select(_ptr(_dev(unit_score)), u, int(group_size), ctypes.byref(params),
+                           ctypes.byref(rh), ctypes.byref(k), _ptr(out["accepted"]),
+                           _ptr(out["rejected"]), _ptr(out["flags"]), _ptr(ws), ws.numel(),
+                           _ptr(status), _stream(stream))
+    _check(st, "pace_select")
+    kk = k.value
+    return (rh.value, kk, out["accepted"][:(u - kk) * group_size],
+            out["rejected"][:kk * group_size], out["flags"][:n])
+
+
+def select_k(unit_score, group_size, k, out=None, ws=None, status=None, stream=None):
+    dev = unit_score.device
+    u = unit_score.numel()
+    n = u * group_size
+    if out is None:
+        out = {"accepted": torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               "rejected": torch.empty(max(n, 1), dtype=torch.int32, device=dev),
+               "flags": torch.empty(max(n, 1), dtype=torch.uint8, device=dev)}
+    if ws is None:
+        ws = workspace(lib().pace_select_workspace_size(u), dev)
+    st = lib().pace_select_k(_ptr(_dev(unit_score)), u, int(group_size), int(k),
+                             _ptr(out["accepted"]), _ptr(out["rejected"]), _ptr(out["flags"]),
+                             _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    _check(st, "pace_select_k")
+    return (out["accepted"][:(u - k) * group_size], out["rejected"][:k * group_size],
+            out["flags"][:n])
+
+
+# ---------------------------------------------------------------- (b) batch
+
+def loss_params(eps_low=0.2, eps_high=0.28, dual_clip=10.0, adv_eps=1e-6,
+                agg=AGG_TOKEN_MEAN, std_unbiased=True):
+    return PaceLossParams(float(eps_low), float(eps_high), float(dual_clip), float(adv_eps),
+                          int(agg), int(bool(std_unbiased)))
+
+
+def make_batch(seq_offsets, n_rows, seq_accepted=None, mask=None):
+    b = PaceBatch(_ptr(_dev(seq_offsets)), _ptr(seq_accepted), _ptr(mask),
+                  seq_offsets.numel() - 1, int(n_rows))
+    b._keep = (seq_offsets, seq_accepted, mask)  # keep the tensors alive with the struct
+    return b
+
+
+def make_loss_args(behav_lp, reward, group_size, params, loss_out, adv_out=None,
+                   ratio_out=None):
+    a = PaceLossArgs(_ptr(_dev(behav_lp)), _ptr(_dev(reward)), int(group_size), params,
+                     _ptr(loss_out), _ptr(adv_out), _ptr(ratio_out))
+    a._keep = (behav_lp, reward, loss_out, adv_out, ratio_out)
+    return a
+
+
+def group_advantages(reward, group_size, seq_accepted=None, adv_eps=1e-6, std_unbiased=True,
+                     out=None, stream=None):
+    n = reward.numel()
+    if out is None:
+        out = torch.empty(n, dtype=torch.float32, device=reward.device)
+    st = lib().pace_group_advantages(_ptr(_dev(reward)), _ptr(seq_accepted), n, int(group_size),
+                                     float(adv_eps), int(bool(std_unbiased)), _ptr(out),
+                                     _stream(stream))
+    _check(st, "pace_group_advantages")
+    return out
+
+
+def token_logprob_workspace_size(n_rows, n_seq, hidden, vocab):
+    return lib().pace_token_logprob_workspace_size(int(n_rows), int(n_seq), int(hidden),
+                                                   int(vocab))
+
+
+def token_logprob(batch: PaceBatch, hidden, w_vocab, targets, temperature=1.0, loss=None,
+                  logprob=None, lse=None, ws=None, status=None, stream=None):
+    """pace_token_logprob.  hidden [n_rows, H] and w_vocab [V, H] are bf16 tensors."""
+    if hidden.dtype != torch.bfloat16 or w_vocab.dtype != torch.bfloat16:
+        raise ValueError("hidden and w_vocab must be bf16")
+    n_rows, H = hidden.shape
+    V = w_vocab.shape[0]
+    dev = hidden.device
+    if logprob is None:
+        logprob = torch.empty(n_rows, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(token_logprob_workspace_size(n_rows, batch.n_seq, H, V), dev)
+    st = lib().pace_token_logprob(ctypes.byref(batch), _ptr(_dev(hidden)), _ptr(_dev(w_vocab)),
+                                  _ptr(_dev(targets)), int(H), int(V), float(temperature),
+                                  _ptr(logprob), _ptr(lse),
+                                  ctypes.byref(loss) if loss is not None else None, _ptr(ws),
+                                  ws.numel(), _ptr(status), _stream(stream))
+    _check(st, "pace_token_logprob")
+    return logprob
+
+
+def surrogate_loss(batch: PaceBatch, logprob, loss: PaceLossArgs, ws=None, status=None,
+                   stream=None):
+    dev = logprob.device
+    if ws is None:
+        ws = workspace(lib().pace_surrogate_loss_workspace_size(batch.n_rows, batch.n_seq), dev)
+    st = lib().pace_surrogate_loss(ctypes.byref(batch), _ptr(_dev(logprob)), ctypes.byref(loss),
+                                   _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    _check(st, "pace_surrogate_loss")
+
+
+def set_profile_events(kernel: int, begin=None, end=None):
+    """Record torch.cuda.Event ``begin`` / ``end`` around every launch of ``kernel``
+    (PROFILE_LMHEAD or PROFILE_TAG_REDUCE) on this thread; None turns it off."""
+    b = ctypes.c_void_p(begin.cuda_event) if begin is not None else None
+    e = ctypes.c_void_p(end.cuda_event) if end is not None else None
+    _check(lib().pace_set_profile_events(int(kernel), b, e), "pace_set_profile_events")
+
+
+def kernel_launches() -> int:
+    """Kernels the library has launched from this thread so far."""
+    return int(lib().pace_kernel_launches())

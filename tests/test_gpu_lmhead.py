@@ -1,0 +1,179 @@
+"""Fused LM-head log-probs on the GPU vs the oracle's fp64 log-softmax.
+
+Tolerance |lp_gpu - lp_oracle| <= 5e-3 (absolute) per row, on every row of
+small shapes (ragged row blocks, partial vocabulary tiles, compacted and
+uncompacted paths), on the tiny workload in full, and on seeded row samples
+of the 7B-shaped, multi-turn and MoE-shaped heads at full size."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from pace_cases import DEV, as_np, bf16_dev, to_dev
+from paper_2609_36830_gb300 import pace, workloads
+
+pytestmark = pytest.mark.gpu
+TOL = 5e-3
+
+
+def _bits(t):
+    return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def _run(hidden, w, targets, seq_offsets=None, seq_accepted=None, mask=None, temperature=1.0,
+         expect_status=0):
+    n_rows = hidden.shape[0]
+    if seq_offsets is None:
+        seq_offsets = torch.tensor([0, n_rows], dtype=torch.int64, device=DEV)
+    b = pace.make_batch(seq_offsets, n_rows, seq_accepted=seq_accepted, mask=mask)
+    lse = torch.empty(n_rows, dtype=torch.float32, device=DEV)
+    status = pace.new_status(DEV)
+    lp = pace.token_logprob(b, hidden, w, targets, temperature, lse=lse, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == expect_status, pace.status_string(int(status.item()))
+    return as_np(lp), as_np(lse)
+
+
+@pytest.mark.parametrize("rows,H,V", [(1, 64, 256), (5, 64, 300), (127, 128, 1000),
+                                      (128, 64, 256), (129, 192, 513), (300, 256, 2048),
+                                      (1000, 512, 4099), (2048, 1024, 8192)])
+@pytest.mark.parametrize("masked", [False, True])
+def test_small_shapes_all_rows(rows, H, V, masked):
+    rng = np.random.default_rng(rows * 7 + H + V)
+    hb = workloads.bf16_normal_host((rows, H), 1.0, rows + H)
+    wb = workloads.bf16_normal_host((V, H), 1.0 / math.sqrt(H) * 2.0, V + H)
+    y = rng.integers(0, V, size=rows).astype(np.int32)
+    hidden = bf16_dev(hb)
+    w = bf16_dev(wb)
+    mask = None
+    if masked:
+        m = (rng.random(rows) < 0.6).astype(np.uint8)
+        mask = to_dev(m)
+    lp, lse = _run(hidden, w, to_dev(y), mask=mask)
+    st, olp, olse = oracle.token_logprob(hb, wb, y)
+    assert st == 0
+    sel = np.ones(rows, bool) if mask is None else as_np(mask).astype(bool)
+    err = np.abs(lp[sel] - olp[sel])
+    assert err.max(initial=0) <= TOL, err.max()
+    assert np.abs(lse[sel] - olse[sel]).max(initial=0) <= TOL
+    assert (lp[~sel] == 0).all() and (lse[~sel] == 0).all()
+
+
+def test_vocab_smaller_than_one_tile():
+    rng = np.random.default_rng(1)
+    rows, H, V = 200, 64, 100
+    hb = workloads.bf16_normal_host((rows, H), 1.0, 3)
+    wb = workloads.bf16_normal_host((V, H), 0.125, 4)
+    y = rng.integers(0, V, size=rows).astype(np.int32)
+    lp, _ = _run(bf16_dev(hb), bf16_dev(wb), to_dev(y))
+    st, olp, _ = oracle.token_logprob(hb, wb, y)
+    assert np.abs(lp - olp).max() <= TOL
+
+
+def test_temperature():
+    rng = np.random.default_rng(2)
+    rows, H, V = 333, 128, 3000
+    hb = workloads.bf16_normal_host((rows, H), 1.0, 5)
+    wb = workloads.bf16_normal_host((V, H), 0.09, 6)
+    y = rng.integers(0, V, size=rows).astype(np.int32)
+    for tau in (0.7, 1.3):
+        lp, _ = _run(bf16_dev(hb), bf16_dev(wb),
+                     to_dev(y), temperature=tau)
+        st, olp, _ = oracle.token_logprob(hb, wb, y, temperature=float(np.float32(tau)))
+        assert np.abs(lp - olp).max() <= TOL
+
+
+def test_zero_weights_give_uniform():
+    rows, H, V = 130, 64, 1000
+    hb = workloads.bf16_normal_host((rows, H), 1.0, 7)
+    w = torch.zeros(V, H, dtype=torch.bfloat16, device=DEV)
+    y = torch.randint(0, V, (rows,), dtype=torch.int32, device=DEV)
+    lp, _ = _run(bf16_dev(hb), w, y)
+    assert np.abs(lp + math.log(V)).max() <= 1e-5
+
+
+def test_bad_target_reported():
+    rows, H, V = 140, 64, 512
+    hb = workloads.bf16_normal_host((rows, H), 1.0, 8)
+    wb = workloads.bf16_normal_host((V, H), 0.125, 9)
+    y = np.zeros(rows, np.int32)
+    y[17] = V
+    lp, _ = _run(bf16_dev(hb), bf16_dev(wb), to_dev(y),
+                 expect_status=pace.ERR_INVALID_ARG)
+    assert math.isnan(lp[17]) and np.isfinite(np.delete(lp, 17)).all()
+
+
+def _tiny_case():
+    pool = workloads.make_pool("tiny")
+    rw = workloads.make_rows(pool)
+    H, V = pool.spec.hidden, pool.spec.vocab
+    hb = workloads.bf16_normal_host((rw.n_rows, H), 1.0, pool.seed + 1)
+    wb = workloads.bf16_normal_host((V, H), 1.0 / math.sqrt(H), pool.seed + 2)
+    return pool, rw, hb, wb
+
+
+@pytest.mark.parametrize("agg", [pace.AGG_TOKEN_MEAN, pace.AGG_SEQ_MEAN_TOKEN_MEAN])
+def test_tiny_workload_full_with_fused_loss(agg):
+    pool, rw, hb, wb = _tiny_case()
+    st, olp, _ = oracle.token_logprob(hb, wb, rw.targets)
+    assert st == 0
+    # behaviour = current + N(0, 0.05 * staleness), current from the oracle
+    behav = workloads.behaviour_logprob(rw, pool.trainer_version, olp, pool.seed)
+    rng = np.random.default_rng(3)
+    acc = (rng.random(pool.n_traj) < 0.75).astype(np.uint8)
+    eps_l, eps_h = np.float32(pool.spec.eps_low), np.float32(pool.spec.eps_high)
+    params = pace.loss_params(eps_low=eps_l, eps_high=eps_h, agg=agg)
+    loss = torch.zeros(1, dtype=torch.float64, device=DEV)
+    la = pace.make_loss_args(to_dev(behav), to_dev(pool.reward), pool.group_size, params, loss)
+    b = pace.make_batch(to_dev(rw.row_offsets), rw.n_rows, seq_accepted=to_dev(acc),
+                        mask=to_dev(rw.mask))
+    status = pace.new_status(DEV)
+    lp = pace.token_logprob(b, bf16_dev(hb), bf16_dev(wb),
+                            to_dev(rw.targets), 1.0, loss=la, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    in_loss = np.repeat(acc, np.diff(rw.row_offsets)).astype(bool) & rw.mask.astype(bool)
+    lp = as_np(lp)
+    assert np.abs(lp[in_loss] - olp[in_loss]).max() <= TOL
+    assert (lp[~in_loss] == 0).all()
+    st, oadv = oracle.group_advantages(pool.reward, pool.group_size, seq_accepted=acc,
+                                       eps=float(np.float32(1e-6)))
+    st, oloss, _, _ = oracle.surrogate(olp, behav, rw.row_offsets, oadv, mask=rw.mask,
+                                       seq_accepted=acc, eps_low=float(eps_l),
+                                       eps_high=float(eps_h), agg=agg)
+    gl = float(loss.item())
+    assert abs(gl - oloss) <= 1e-3 * abs(oloss), (gl, oloss)
+
+
+@pytest.mark.parametrize("name", ["math7b", "multiturn", "moe"])
+def test_full_size_heads_sampled_rows(name):
+    """Full-size heads in the benchmark's launch configuration (all pool rows,
+    accepted flags and loss mask applied by the library's compaction); the
+    oracle recomputes a seeded sample of the rows in the loss."""
+    pool = workloads.make_pool(name)
+    rw = workloads.make_rows(pool)
+    H, V = pool.spec.hidden, pool.spec.vocab
+    hidden = workloads.bf16_normal_device((rw.n_rows, H), 1.0, pool.seed + 11)
+    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), pool.seed + 12)
+    rng = np.random.default_rng(pool.seed)
+    acc = np.repeat((rng.random(pool.n_traj // 8) < 0.75).astype(np.uint8), 8)
+    b = pace.make_batch(to_dev(rw.row_offsets), rw.n_rows, seq_accepted=to_dev(acc),
+                        mask=to_dev(rw.mask))
+    status = pace.new_status(DEV)
+    lp = pace.token_logprob(b, hidden, w, to_dev(rw.targets), 1.0, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    lp = as_np(lp)
+    in_loss = np.repeat(acc, np.diff(rw.row_offsets)).astype(bool) & rw.mask.astype(bool)
+    assert (lp[~in_loss] == 0).all() and np.isfinite(lp).all()
+    cand = np.nonzero(in_loss)[0]
+    sample = np.sort(rng.choice(cand, size=48, replace=False))
+    sample = np.concatenate([sample, cand[:2], cand[-2:]])  # first and last rows of the loss
+    hb = _bits(hidden[torch.from_numpy(sample).to(DEV)])
+    wb = _bits(w)
+    st, olp, _ = oracle.token_logprob(hb, wb, rw.targets[sample])
+    assert st == 0
+    err = np.abs(lp[sample] - olp)
+    assert err.max() <= TOL, err.max()

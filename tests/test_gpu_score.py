@@ -1,0 +1,174 @@
+"""Pool scoring on the GPU vs the oracle: fp64 bits must be identical
+(K_gen, K_wait, F, score, unit score) on every workload, mode and edge case."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from pace_cases import (DEV, as_np, assert_bits_equal, gpu_score, oracle_score,
+                        pool_score_case, to_dev)
+from paper_2609_36830_gb300 import pace, workloads
+
+pytestmark = pytest.mark.gpu
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "hand_pool.json")
+
+
+def _check(g, o, what):
+    for k in ("kgen", "kwait", "weight", "score", "unit_score"):
+        assert_bits_equal(g[k], o[k], f"{what}:{k}")
+
+
+@pytest.mark.parametrize("mode", ["eff", "raw", "gen"])
+def test_hand_pool(mode):
+    h = json.load(open(GOLDEN))
+    tr = h["trajectories"]
+    tags = np.concatenate([np.array(t["tags"], np.int32) for t in tr])
+    offsets = np.concatenate([[0], np.cumsum([len(t["tags"]) for t in tr])]).astype(np.int64)
+    c = np.array([t["c"] for t in tr], np.int32)
+    s_pre = np.array([np.nan if t["s_pre"] is None else t["s_pre"] for t in tr], np.float32)
+    window = np.array(h["window"], np.float32)
+    for G in (1, 2, 3, 6):
+        g = gpu_score(tags, offsets, c, s_pre, 10, window, mode=mode, min_obs=1, group_size=G)
+        o = oracle_score(tags, offsets, c, s_pre, 10, window, mode=mode, min_obs=1, group_size=G)
+        _check(g, o, f"hand G={G}")
+
+
+@pytest.mark.parametrize("name,n", [("tiny", None), ("math7b", 384), ("math7b", 512),
+                                    ("math7b", 768), ("multiturn", 256), ("multiturn", 480),
+                                    ("moe", None), ("sweep", 1024), ("sweep", 16384)])
+@pytest.mark.parametrize("mode", ["eff", "raw", "gen"])
+def test_workloads(name, n, mode):
+    pool = workloads.make_pool(name, n_traj=n)
+    g, o = pool_score_case(pool, mode=mode)
+    _check(g, o, f"{name}/{n}/{mode}")
+
+
+def test_group_sizes_and_gammas():
+    pool = workloads.make_pool("math7b", n_traj=768)
+    for G in (1, 12, 16, 96):
+        for gamma in (1, 2, 4, 7):
+            args = (pool.tags, pool.meta["offsets_host"], pool.c_version, pool.s_pre,
+                    pool.trainer_version, pool.window)
+            g = gpu_score(*args, group_size=G, gamma=gamma)
+            o = oracle_score(*args, group_size=G, gamma=gamma)
+            _check(g, o, f"G={G} gamma={gamma}")
+
+
+def test_sweep_128k_full_and_1m_sampled():
+    # 128k pool (~0.44 G tags) checked in full
+    pool = workloads.make_pool("sweep", n_traj=131072, device=DEV)
+    tags_h = pool.tags.cpu().numpy()
+    args = (pool.tags, pool.meta["offsets_host"], pool.c_version, pool.s_pre,
+            pool.trainer_version, pool.window)
+    g = gpu_score(*args, group_size=8)
+    o = oracle_score(tags_h, *args[1:], group_size=8)
+    _check(g, o, "sweep128k")
+    del pool, tags_h
+    torch.cuda.empty_cache()
+    # 1M pool (~3.4 G tags): the launch the benchmark times; the oracle scores a
+    # seeded sample of whole groups from their own tags.
+    pool = workloads.make_pool("sweep", n_traj=1048576, device=DEV)
+    off = pool.meta["offsets_host"]
+    g = gpu_score(pool.tags, off, pool.c_version, pool.s_pre, pool.trainer_version, pool.window,
+                  group_size=8)
+    rng = np.random.default_rng(5)
+    units = np.sort(rng.choice(1048576 // 8, size=256, replace=False))
+    ids = (units[:, None] * 8 + np.arange(8)[None, :]).ravel()
+    seg = [pool.tags[off[i]:off[i + 1]].cpu().numpy() for i in ids]
+    sub_off = np.concatenate([[0], np.cumsum([s.size for s in seg])]).astype(np.int64)
+    o = oracle_score(np.concatenate(seg), sub_off, pool.c_version[ids], pool.s_pre[ids],
+                     pool.trainer_version, pool.window, group_size=8)
+    for k in ("kgen", "kwait", "weight", "score"):
+        assert_bits_equal(g[k][ids], o[k], f"sweep1m:{k}")
+    assert_bits_equal(g["unit_score"][units], o["unit_score"], "sweep1m:unit")
+    # identities over the whole pool: score = K_wait + F K_gen, all finite, >= 0
+    assert np.isfinite(g["score"]).all() and (g["score"] >= 0).all()
+    np.testing.assert_array_equal(g["score"], g["kwait"] + g["weight"] * g["kgen"])
+
+
+def _mk(lens, rng, j=50, tool=0.0):
+    offsets = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    n = len(lens)
+    c = rng.integers(0, j + 1, size=n).astype(np.int32)
+    tags = np.empty(int(offsets[-1]), np.int32)
+    for i in range(n):
+        t = np.sort(rng.integers(0, c[i] + 1, size=lens[i])).astype(np.int32)
+        t[rng.random(lens[i]) < tool] = -1
+        tags[offsets[i]:offsets[i + 1]] = t
+    s_pre = np.where(rng.random(n) < 0.5, rng.random(n), np.nan).astype(np.float32)
+    window = rng.random(100).astype(np.float32)
+    return tags, offsets, c, s_pre, j, window
+
+
+@pytest.mark.parametrize("case", ["empty_traj", "ragged", "one_long", "tiny_many", "all_tool",
+                                  "single"])
+def test_edge_cases(case):
+    rng = np.random.default_rng(hash(case) % 1000)
+    if case == "empty_traj":
+        lens = [0, 5, 0, 0, 130, 0, 1, 0]
+    elif case == "ragged":
+        lens = list(rng.integers(1, 3000, size=64))
+        lens[-1] = 1027
+    elif case == "one_long":
+        lens = [3, 5_000_003, 17, 0, 1, 2, 9, 100]
+    elif case == "tiny_many":
+        lens = list(rng.integers(0, 4, size=40000))
+    elif case == "all_tool":
+        lens = [10, 20, 30, 40]
+    else:
+        lens = [1]
+    lens = list(lens)
+    while len(lens) % 4:
+        lens.append(int(rng.integers(0, 9)))
+    tool = 1.0 if case == "all_tool" else 0.2
+    tags, offsets, c, s_pre, j, window = _mk(lens, rng, tool=tool)
+    for G in (1, 4):
+        g = gpu_score(tags, offsets, c, s_pre, j, window, group_size=G, min_obs=10)
+        o = oracle_score(tags, offsets, c, s_pre, j, window, group_size=G, min_obs=10)
+        _check(g, o, f"{case}/G={G}")
+
+
+def test_window_below_min_obs_and_no_window():
+    pool = workloads.make_pool("tiny")
+    args = (pool.tags, pool.meta["offsets_host"], pool.c_version, pool.s_pre,
+            pool.trainer_version)
+    g = gpu_score(*args, pool.window[:20], min_obs=32)
+    o = oracle_score(*args, pool.window[:20], min_obs=32)
+    _check(g, o, "short window")
+    assert (g["weight"] == 1.0).all()
+    g = gpu_score(*args, None, min_obs=0)
+    o = oracle_score(*args, np.zeros(0, np.float32), min_obs=0)
+    _check(g, o, "no window")
+
+
+def test_empty_pool():
+    out = gpu_score(np.zeros(0, np.int32), np.zeros(1, np.int64), np.zeros(0, np.int32),
+                    np.zeros(0, np.float32), 5, np.ones(4, np.float32), group_size=1)
+    assert out["score"].size == 0
+
+
+@pytest.mark.parametrize("what,code", [("v_gt_c", pace.ERR_VERSION_ORDER),
+                                       ("c_gt_j", pace.ERR_VERSION_ORDER),
+                                       ("tag_below_sentinel", pace.ERR_INVALID_ARG),
+                                       ("nan_window", pace.ERR_NAN_INPUT),
+                                       ("bad_offsets", pace.ERR_INVALID_ARG)])
+def test_device_side_errors(what, code):
+    pool = workloads.make_pool("tiny")
+    tags = pool.tags.copy()
+    off = pool.meta["offsets_host"].copy()
+    c = pool.c_version.copy()
+    w = pool.window.copy()
+    j = pool.trainer_version
+    if what == "v_gt_c":
+        tags[off[3] + 1] = c[3] + 1
+    elif what == "c_gt_j":
+        c[5] = j + 1
+    elif what == "tag_below_sentinel":
+        tags[7] = -3
+    elif what == "nan_window":
+        w[100] = np.nan
+    else:
+        off[10] = off[11] + 1  # not non-decreasing
+    gpu_score(tags, off, c, pool.s_pre, j, w, expect_status=code)

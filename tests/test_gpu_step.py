@@ -1,0 +1,61 @@
+"""One whole PACE step (score -> budget/select -> fused log-prob + loss) at
+the 7B-shaped single-turn workload, in exactly the launch configuration
+bench.py times: the selection must match the oracle id for id, sampled
+log-probs within 5e-3, and the fused loss must equal the standalone
+surrogate on the same log-probs (whose parity with the oracle is pinned in
+test_gpu_loss.py at these sizes)."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from pace_cases import DEV, as_np
+from paper_2609_36830_gb300 import pace, step, workloads
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("n_traj", [512, 768])
+def test_math7b_step(n_traj):
+    pool = workloads.make_pool("math7b", n_traj=n_traj)
+    rw = workloads.make_rows(pool)
+    H, V = pool.spec.hidden, pool.spec.vocab
+    hidden = workloads.bf16_normal_device((rw.n_rows, H), 1.0, pool.seed + 11)
+    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), pool.seed + 12)
+    behav = workloads.behaviour_logprob(rw, pool.trainer_version, workloads.uniform_center(V),
+                                        pool.seed)
+    x = step.build_inputs(pool, rw, hidden, w, behav)
+    lp_params = pace.loss_params(eps_low=pool.spec.eps_low, eps_high=pool.spec.eps_high)
+    st = step.PaceStep(x, loss_params=lp_params)
+    k, r_hat = st.run()
+    torch.cuda.synchronize()
+    assert int(st.status.item()) == 0
+    # selection parity
+    ost, *_, ous = oracle.score_pool(pool.tags, pool.meta["offsets_host"], pool.c_version,
+                                     pool.s_pre, pool.trainer_version, pool.window,
+                                     group_size=pool.group_size)
+    U = pool.n_traj // pool.group_size
+    _, _, orh, ok = oracle.budget(pool.n_traj, pool.n_target, 0.0, 0.9, 0.0, U)
+    assert (k, r_hat) == (ok, orh)
+    _, oacc, orej, oflag = oracle.select(ous, pool.group_size, ok)
+    np.testing.assert_array_equal(as_np(st.sel_out["flags"]), oflag)
+    # sampled log-probs
+    lp = as_np(st.logprob)
+    in_loss = np.repeat(oflag, np.diff(rw.row_offsets)).astype(bool) & rw.mask.astype(bool)
+    assert (lp[~in_loss] == 0).all() and np.isfinite(lp).all()
+    rng = np.random.default_rng(17)
+    sample = np.sort(rng.choice(np.nonzero(in_loss)[0], size=32, replace=False))
+    hb = hidden[torch.from_numpy(sample).to(DEV)].view(torch.int16).cpu().numpy().view(np.uint16)
+    wb = w.view(torch.int16).cpu().numpy().view(np.uint16)
+    _, olp, _ = oracle.token_logprob(hb, wb, rw.targets[sample])
+    assert np.abs(lp[sample] - olp).max() <= 5e-3
+    # fused loss == standalone surrogate on the same log-probs (same stream)
+    loss2 = torch.zeros(1, dtype=torch.float64, device=DEV)
+    la = pace.make_loss_args(x.behav_lp, x.reward, pool.group_size, lp_params, loss2)
+    pace.surrogate_loss(st.batch, st.logprob, la)
+    torch.cuda.synchronize()
+    assert float(st.loss.item()) == float(loss2.item())
+    assert math.isfinite(float(st.loss.item()))
+    assert st.rows_in_loss() == int(in_loss.sum())
