@@ -289,8 +289,9 @@ def run_gpu(args):
 
     pool, rows, x, st = _make_step(rank, device)
     H, V = x.hidden.shape[1], x.w_vocab.shape[0]
+    k_units = None
     for _ in range(args.warmup):
-        st.run()
+        k_units, _ = st.run()
     torch.cuda.synchronize()
     assert int(st.status.item()) == 0, pace.status_string(int(st.status.item()))
     M = st.rows_in_loss()
@@ -380,7 +381,7 @@ def run_gpu(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": _workload_name(), "global_batch": pool.n_traj * ws,
                        "rows_in_loss_per_step": M, "rows_total": int(rows.n_rows),
-                       "k_units_rejected": st.k_units if hasattr(st, "k_units") else None,
+                       "k_units_rejected": k_units,
                        "parallelism": f"{ws} independent pool replica(s), no collective",
                        "l2": "inputs larger than L2 (hidden states 10.7 GB per step)"},
             "roofline": {"bound": "tensor", "kernel": "lmhead_lse_kernel", "achieved": achieved,
@@ -401,6 +402,61 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
+def run_case(args):
+    """One kernel's launch configuration on a small case (for profiler captures)."""
+    import torch
+    from paper_2609_36830_gb300 import pace, workloads
+    device = "cuda:0"
+    torch.cuda.set_device(0)
+    peaks, _ = _peaks()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    if args.case == "lmhead":
+        spec = workloads.SPECS[WORKLOAD]
+        H, V, rows = spec.hidden, spec.vocab, args.case_rows
+        hidden = workloads.bf16_normal_device((rows, H), 1.0, 101, device)
+        w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), 102, device)
+        gen = torch.Generator(device=device)
+        gen.manual_seed(103)
+        targets = torch.randint(0, V, (rows,), generator=gen, device=device, dtype=torch.int32)
+        b = pace.make_batch(torch.tensor([0, rows], dtype=torch.int64, device=device), rows)
+        lp = torch.empty(rows, dtype=torch.float32, device=device)
+        ws = pace.workspace(pace.token_logprob_workspace_size(rows, 1, H, V), device)
+        status = pace.new_status(device)
+        for i in range(args.warmup + args.steps):
+            if i >= args.warmup:
+                pace.set_profile_events(pace.PROFILE_LMHEAD, *evs[i - args.warmup])
+            pace.token_logprob(b, hidden, w, targets, 1.0, logprob=lp, ws=ws, status=status)
+        pace.set_profile_events(pace.PROFILE_LMHEAD)
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0
+        ms = statistics.mean(a.elapsed_time(z) for a, z in evs)
+        tf = 2.0 * rows * H * V / (ms / 1e3) / 1e12
+        print(json.dumps({"case": "lmhead", "rows": rows, "H": H, "V": V, "kernel_ms": ms,
+                          "tflops": tf, "frac_burst": tf / peaks["bf16_tflops"]}), flush=True)
+    else:
+        pool = workloads.make_pool("sweep", n_traj=args.case_traj, device=device)
+        n = pool.n_traj
+        tok = int(pool.meta["offsets_host"][-1])
+        c = torch.from_numpy(pool.c_version).to(device)
+        sp = torch.from_numpy(pool.s_pre).to(device)
+        win = torch.from_numpy(pool.window).to(device)
+        status = pace.new_status(device)
+        for i in range(args.warmup + args.steps):
+            if i >= args.warmup:
+                pace.set_profile_events(pace.PROFILE_TAG_REDUCE, *evs[i - args.warmup])
+            out = pace.score_pool(pool.tags, pool.offsets, c, sp, pool.trainer_version, win,
+                                  pace.score_params(group_size=8), status=status)
+        pace.set_profile_events(pace.PROFILE_TAG_REDUCE)
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0
+        ms = statistics.mean(a.elapsed_time(z) for a, z in evs)
+        nbytes = 4 * tok + 8 * (n + 1) + 16 * n
+        print(json.dumps({"case": "tagreduce", "n_traj": n, "tokens": tok, "kernel_ms": ms,
+                          "gbs": nbytes / (ms / 1e3) / 1e9,
+                          "frac_hbm": nbytes / (ms / 1e3) / 1e9 / peaks["hbm_gbs"]}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -410,6 +466,10 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=64)
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--case", choices=["lmhead", "tagreduce"], default=None,
+                    help="time one kernel on a small case (profiler captures)")
+    ap.add_argument("--case-rows", type=int, default=4864)
+    ap.add_argument("--case-traj", type=int, default=16384)
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -418,6 +478,9 @@ def main():
         return
     from paper_2609_36830_gb300 import build as pace_build
     pace_build.build()
+    if args.case:
+        run_case(args)
+        return
     run_gpu(args)
 
 

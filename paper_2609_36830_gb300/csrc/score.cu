@@ -303,8 +303,9 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
                                        double* unit_score, void* workspace,
                                        size_t workspace_bytes, int32_t* status_dev,
                                        void* stream) {
-  if (!params || !offsets || !c_version || !score) return PACE_ERR_INVALID_ARG;
+  if (!params) return PACE_ERR_INVALID_ARG;
   if (n_traj < 0 || n_tokens < 0 || n_traj > (int64_t(1) << 31)) return PACE_ERR_INVALID_ARG;
+  if (n_traj > 0 && (!offsets || !c_version || !score)) return PACE_ERR_INVALID_ARG;
   if (n_tokens > 0 && !tags) return PACE_ERR_INVALID_ARG;
   const int G = params->group_size;
   if (G < 1 || G > 1024 || n_traj % G != 0) return PACE_ERR_INVALID_ARG;
@@ -315,7 +316,7 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   if (window_len < 0 || window_len > kMaxWindow) return PACE_ERR_UNSUPPORTED_SHAPE;
   if (window_len > 0 && !window) return PACE_ERR_INVALID_ARG;
   if (tags && !aligned(tags, 16)) return PACE_ERR_UNSUPPORTED_SHAPE;
-  if (n_traj == 0) return PACE_OK;
+  if (n_traj == 0) return n_tokens == 0 ? PACE_OK : PACE_ERR_INVALID_ARG;
   if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
   Carver cv(workspace, workspace_bytes);
   ScoreWs ws = carve_score_ws(cv, n_traj);

@@ -314,8 +314,13 @@ def surrogate_loss(batch: PaceBatch, logprob, loss: PaceLossArgs, ws=None, statu
 def set_profile_events(kernel: int, begin=None, end=None):
     """Record torch.cuda.Event ``begin`` / ``end`` around every launch of ``kernel``
     (PROFILE_LMHEAD or PROFILE_TAG_REDUCE) on this thread; None turns it off."""
-    b = ctypes.c_void_p(begin.cuda_event) if begin is not None else None
-    e = ctypes.c_void_p(end.cuda_event) if end is not None else None
+    def handle(ev):
+        if ev is None:
+            return None
+        if not ev.cuda_event:  # torch creates the CUDA event on its first record
+            ev.record()
+        return ctypes.c_void_p(ev.cuda_event)
+    b, e = handle(begin), handle(end)
     _check(lib().pace_set_profile_events(int(kernel), b, e), "pace_set_profile_events")
 
 
