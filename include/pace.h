@@ -180,6 +180,29 @@ PACE_API pace_status pace_select_k(const double* unit_score, int64_t n_units, in
 
 PACE_API size_t pace_select_workspace_size(int64_t n_units);
 
+/* pace_select_k for callers that cannot allocate device memory.  The paper has
+ * no counterpart: this exists for code that must not call cudaMalloc, such as
+ * a plugin running inside a host framework whose memory pool owns all device
+ * memory, or a latency-critical loop where an allocation could synchronise
+ * the device.  Such a caller still passes its inputs and outputs; the scratch
+ * the radix path needs comes from a fixed array of 32 KB inside the library,
+ * which every GPU that loads the library keeps until the process exits.
+ *   - n_units must be at most 2^20 (1,048,576); larger pools get
+ *     PACE_ERR_UNSUPPORTED_SHAPE and nothing is launched.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current) and caches it; make that first call before any
+ *     stream capture.
+ *   - All calls on a device share the one array and each call re-initialises
+ *     what it needs, so results do not depend on earlier calls; but calls
+ *     that overlap on the GPU (different streams, or threads) race on it.
+ * Arguments and outputs are those of pace_select_k; no cudaMalloc, cudaFree or
+ * other allocating routine is called. */
+PACE_API pace_status pace_select_k_noalloc(const double* unit_score, int64_t n_units,
+                                           int32_t group_size, int64_t k_units,
+                                           int32_t* accepted_ids, int32_t* rejected_ids,
+                                           uint8_t* traj_accepted, int32_t* status_dev,
+                                           void* stream);
+
 /* ------------------------------------------------------------------------ */
 /* (b) Log-probabilities and the clipped surrogate                           */
 /* ------------------------------------------------------------------------ */

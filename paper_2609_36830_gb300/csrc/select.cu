@@ -15,6 +15,8 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "pace_internal.cuh"
 
 namespace pace {
@@ -439,4 +441,59 @@ extern "C" pace_status pace_select(const double* unit_score, int64_t n_units, in
   *r_hat_out = r_hat;
   *k_units_out = k;
   return PACE_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Selection without a caller-provided workspace.
+//
+// For callers that may not allocate device memory themselves, the radix path's
+// scratch lives in this file-scope array instead of a workspace.  Every GPU
+// that loads the library holds it (32 KB) until the process exits; every call
+// on a device shares it, so calls that overlap on that device race.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+constexpr int64_t kNoAllocMaxUnits = int64_t(1) << 20;
+constexpr size_t kNoAllocScratchBytes = 32768;
+
+}  // namespace
+
+static __device__ __align__(256) unsigned char g_select_scratch[kNoAllocScratchBytes];
+
+namespace {
+
+// Device address of g_select_scratch on the current device.  In host code the
+// array's name is only a host-side stand-in, so the address is asked from the
+// runtime once per device (with that device current) and cached.
+pace_status select_scratch_address(void** out) {
+  constexpr int kMaxDevices = 64;
+  static void* addr[kMaxDevices] = {};
+  static std::mutex mu;
+  int dev = 0;
+  PACE_TRY_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return PACE_ERR_CUDA;
+  std::lock_guard<std::mutex> g(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_select_scratch) != cudaSuccess || !p) return PACE_ERR_CUDA;
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return PACE_OK;
+}
+
+}  // namespace
+
+extern "C" pace_status pace_select_k_noalloc(const double* unit_score, int64_t n_units,
+                                             int32_t group_size, int64_t k_units,
+                                             int32_t* accepted_ids, int32_t* rejected_ids,
+                                             uint8_t* traj_accepted, int32_t* status_dev,
+                                             void* stream) {
+  if (n_units > kNoAllocMaxUnits) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (pace_select_workspace_size(n_units) > kNoAllocScratchBytes) return PACE_ERR_UNSUPPORTED_SHAPE;
+  void* scratch = nullptr;
+  PACE_TRY(select_scratch_address(&scratch));
+  return pace_select_k(unit_score, n_units, group_size, k_units, accepted_ids, rejected_ids,
+                       traj_accepted, scratch, kNoAllocScratchBytes, status_dev, stream);
 }

@@ -75,6 +75,7 @@ SIGNATURES = {
     "pace_select": ([_P, _I64, _I32, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P], _I32),
     "pace_select_k": ([_P, _I64, _I32, _I64, _P, _P, _P, _P, _SZ, _P, _P], _I32),
     "pace_select_workspace_size": ([_I64], _SZ),
+    "pace_select_k_noalloc": ([_P, _I64, _I32, _I64, _P, _P, _P, _P, _P], _I32),
     "pace_loss_params_default": ([_P], None),
     "pace_group_advantages": ([_P, _P, _I64, _I32, _F32, _I32, _P, _P], _I32),
     "pace_token_logprob": ([_P, _P, _P, _P, _I32, _I32, _F32, _P, _P, _P, _P, _SZ, _P, _P],
