@@ -321,7 +321,8 @@ def run_gpu(args):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
         dist.barrier()
-    lm_ms = statistics.mean(b.elapsed_time(e) for b, e in zip(k_b, k_e))
+    lm_each = [b.elapsed_time(e) for b, e in zip(k_b, k_e)]
+    lm_ms = statistics.mean(lm_each)
     flops = 2.0 * H * V * M
     achieved = flops / (lm_ms / 1e3) / 1e12
     peak_s = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
@@ -389,7 +390,8 @@ def run_gpu(args):
                          "peak_source": f"{peak_src} bf16_tflops_sustained",
                          "frac_of_burst": achieved / peaks["bf16_tflops"],
                          "frac_of_nominal_2250": achieved / 2250.0,
-                         "kernel_ms": lm_ms, "flops_per_launch": flops, "traffic": None},
+                         "kernel_ms": lm_ms, "kernel_ms_each": lm_each,
+                         "flops_per_launch": flops, "traffic": None},
             "cpu_baseline": cpu,
             "e2e": {"value": M * ws / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e_ms},

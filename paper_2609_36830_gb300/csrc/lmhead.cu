@@ -44,12 +44,15 @@ constexpr int BM = 128;
 constexpr int BN = 256;
 constexpr int BK = 64;
 constexpr int STAGES = 4;
+constexpr int CLUSTER = 2;                      // CTAs sharing each vocabulary tile
 constexpr int kThreads = 192;
-constexpr uint32_t kStageA = BM * BK * 2;  // 16 KB
-constexpr uint32_t kStageB = BN * BK * 2;  // 32 KB
+constexpr uint32_t kStageA = BM * BK * 2;       // 16 KB: this CTA's 128 hidden rows
+constexpr uint32_t kStageB = BN * BK * 2;       // 32 KB: 256 vocabulary rows
+constexpr uint32_t kHalfB = kStageB / CLUSTER;  // each CTA of the pair loads one half
 constexpr uint32_t kStageBytes = kStageA + kStageB;
-constexpr uint32_t kTmemCols = 2 * BN;     // two fp32 accumulators of 256 columns
+constexpr uint32_t kTmemCols = 2 * BN;          // two fp32 accumulators of 256 columns
 constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
+constexpr uint16_t kPairMask = 0x3;
 constexpr size_t kSmemBytes = 1024 /* alignment slack */ + STAGES * kStageBytes + 256;
 
 struct LmArgs {
@@ -66,19 +69,27 @@ struct LmArgs {
   int32_t* status;
 };
 
-__device__ __forceinline__ uint64_t make_policy_evict_last() {
-  uint64_t pol;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
-  return pol;
-}
-
 __device__ __forceinline__ uint64_t make_policy_evict_normal() {
   uint64_t pol;
   asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
   return pol;
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+// A work item is (row pair, vocabulary split): the two CTAs of a cluster take
+// the two 128-row blocks of the pair and sweep the same vocabulary tiles, each
+// loading half of every 256-row vocabulary tile and multicasting it to both.
+// Clusters are persistent and take items round-robin, so all clusters sweep
+// their splits in step and each vocabulary tile is read from HBM about once per
+// round of items.
+struct ItemCursor {
+  int64_t item, n_items;
+  int n_clusters;
+  __device__ ItemCursor(int cid, int nc, int64_t ni) : item(cid), n_items(ni), n_clusters(nc) {}
+  __device__ bool valid() const { return item < n_items; }
+  __device__ void next() { item += n_clusters; }
+};
+
+__global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
     lmhead_lse_kernel(const __grid_constant__ CUtensorMap tm_a,
                       const __grid_constant__ CUtensorMap tm_b, LmArgs p) {
   extern __shared__ unsigned char smem_raw[];
@@ -86,8 +97,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* stage_base = smem;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * kStageBytes);
-  uint64_t* full = bars;                  // [STAGES]
-  uint64_t* empty = bars + STAGES;        // [STAGES]
+  uint64_t* full = bars;                     // [STAGES] this CTA's A + both halves of B landed
+  uint64_t* empty = bars + STAGES;           // [STAGES] both CTAs' MMAs done with the stage
   uint64_t* tmem_full = bars + 2 * STAGES;   // [2]
   uint64_t* tmem_empty = tmem_full + 2;      // [2]
   uint64_t* mma_done = tmem_empty + 2;       // [1]
@@ -96,23 +107,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int64_t row_block = blockIdx.x / p.splits;
-  const int split = blockIdx.x % p.splits;
-  const int64_t row0 = row_block * BM;
+  const uint32_t crank = cluster_ctarank();
+  const int n_clusters = static_cast<int>(gridDim.x) / CLUSTER;
+  const int cid = static_cast<int>(blockIdx.x) / CLUSTER;
   const int64_t n_valid = p.n_valid_dev ? static_cast<int64_t>(*p.n_valid_dev) : p.rows_cap;
-  if (row0 >= n_valid) return;  // uniform: nothing allocated yet
-  // after a timeout anywhere in the grid, the remaining CTAs do not start waiting
-  if (p.status && *reinterpret_cast<volatile int32_t*>(p.status) == PACE_ERR_TIMEOUT) return;
-  const int tile0 = split * p.tiles_per_split;
-  const int tile1 = min(tile0 + p.tiles_per_split, p.n_vtiles);
-  if (tile0 >= tile1) return;
-  const int num_tiles = tile1 - tile0;
+  const int64_t row_pairs = (n_valid + 2 * BM - 1) / (2 * BM);
+  const int64_t n_items = row_pairs * p.splits;
+  // both CTAs of a cluster read the same n_valid and cid: the exit is uniform
+  if (cid >= n_items) return;
   const int nkb = p.H / BK;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], CLUSTER);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tmem_full[b], 1);
@@ -127,7 +135,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_relinquish();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();  // both CTAs' barriers exist before any multicast reaches them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -136,24 +144,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ------------------------------------------------ TMA producer
       tma_prefetch_desc(&tm_a);
       tma_prefetch_desc(&tm_b);
-      const uint64_t pol_a = make_policy_evict_last();
-      const uint64_t pol_b = make_policy_evict_normal();
+      const uint64_t pol = make_policy_evict_normal();
       uint32_t it = 0;
       bool ok = true;
-      for (int t = 0; t < num_tiles && ok; ++t) {
-        const int32_t n0 = (tile0 + t) * BN;
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const uint32_t s = it % STAGES;
-          const uint32_t ph = (it / STAGES) & 1u;
-          if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
-            ok = false;
-            break;
+      for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
+        const int64_t rp = c.item / p.splits;
+        const int split = static_cast<int>(c.item % p.splits);
+        const int32_t row0 = static_cast<int32_t>((rp * CLUSTER + crank) * BM);
+        const int tile0 = split * p.tiles_per_split;
+        const int tile1 = min(tile0 + p.tiles_per_split, p.n_vtiles);
+        for (int t = tile0; t < tile1 && ok; ++t) {
+          const int32_t nb = t * BN + static_cast<int32_t>(crank) * (BN / CLUSTER);
+          for (int kb = 0; kb < nkb; ++kb, ++it) {
+            const uint32_t s = it % STAGES;
+            const uint32_t ph = (it / STAGES) & 1u;
+            if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
+              ok = false;
+              break;
+            }
+            unsigned char* sa = stage_base + s * kStageBytes;
+            unsigned char* sb = sa + kStageA;
+            mbar_arrive_expect_tx(&full[s], kStageBytes);
+            tma_load_2d(sa, &tm_a, &full[s], kb * BK, row0, pol);
+            tma_load_2d_multicast(sb + crank * kHalfB, &tm_b, &full[s], kb * BK, nb, kPairMask,
+                                  pol);
           }
-          unsigned char* sa = stage_base + s * kStageBytes;
-          unsigned char* sb = sa + kStageA;
-          mbar_arrive_expect_tx(&full[s], kStageBytes);
-          tma_load_2d(sa, &tm_a, &full[s], kb * BK, static_cast<int32_t>(row0), pol_a);
-          tma_load_2d(sb, &tm_b, &full[s], kb * BK, n0, pol_b);
         }
       }
       if (!ok) {
@@ -169,36 +184,43 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------ MMA issuer
-      uint32_t it = 0;
+      uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int t = 0; t < num_tiles && ok; ++t) {
-        const uint32_t acc = t & 1;
-        const uint32_t acc_ph = (t >> 1) & 1u;
-        if (!mbar_wait_bounded(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t d_tmem = tmem_base + acc * BN;
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const uint32_t s = it % STAGES;
-          const uint32_t ph = (it / STAGES) & 1u;
-          if (!mbar_wait_bounded(&full[s], ph, abort_flag)) {
+      for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
+        const int split = static_cast<int>(c.item % p.splits);
+        const int tile0 = split * p.tiles_per_split;
+        const int tile1 = min(tile0 + p.tiles_per_split, p.n_vtiles);
+        for (int t = tile0; t < tile1 && ok; ++t, ++tcount) {
+          const uint32_t acc = tcount & 1u;
+          const uint32_t acc_ph = (tcount >> 1) & 1u;
+          if (!mbar_wait_bounded(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(stage_base + s * kStageBytes);
-          const uint32_t sb = sa + kStageA;
+          const uint32_t d_tmem = tmem_base + acc * BN;
+          for (int kb = 0; kb < nkb; ++kb, ++it) {
+            const uint32_t s = it % STAGES;
+            const uint32_t ph = (it / STAGES) & 1u;
+            if (!mbar_wait_bounded(&full[s], ph, abort_flag)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_u32(stage_base + s * kStageBytes);
+            const uint32_t sb = sa + kStageA;
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {
-            tc_mma_f16(d_tmem, smem_desc_k128(sa + k * 32), smem_desc_k128(sb + k * 32), kIdesc,
-                       (kb > 0 || k > 0) ? 1u : 0u);
+            for (int k = 0; k < BK / 16; ++k) {
+              tc_mma_f16(d_tmem, smem_desc_k128(sa + k * 32), smem_desc_k128(sb + k * 32),
+                         kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
+            }
+            // frees the stage in both CTAs once these MMAs have read it: the peer
+            // multicasts its half of B into this CTA's stage too
+            tc_commit_multicast(&empty[s], kPairMask);
           }
-          tc_commit(&empty[s]);  // frees the stage once these MMAs have read it
+          if (!ok) break;
+          tc_commit(&tmem_full[acc]);
         }
-        if (!ok) break;
-        tc_commit(&tmem_full[acc]);
       }
       if (!ok) {
         if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
@@ -212,68 +234,79 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ epilogue (4 warps)
     const int quad = warp & 3;  // TMEM lanes this warp may access
     const int r_local = quad * 32 + lane;
-    const int64_t row = row0 + r_local;
-    const bool row_ok = row < n_valid;
-    int32_t y = -1;
-    if (row_ok) {
-      const int64_t orig = p.rowidx ? static_cast<int64_t>(p.rowidx[row]) : row;
-      y = p.targets[orig];
-    }
     const float scale = p.scale_log2;
-    float m = -INFINITY, s = 0.0f, tgt = 0.0f;
-    bool have_tgt = false;
-    for (int t = 0; t < num_tiles; ++t) {
-      const uint32_t acc = t & 1;
-      const uint32_t acc_ph = (t >> 1) & 1u;
-      if (!mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag)) {
-        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
-        *abort_flag = 1;
-        break;
+    uint32_t tcount = 0;
+    bool ok = true;
+    for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
+      const int64_t rp = c.item / p.splits;
+      const int split = static_cast<int>(c.item % p.splits);
+      const int tile0 = split * p.tiles_per_split;
+      const int tile1 = min(tile0 + p.tiles_per_split, p.n_vtiles);
+      const int64_t row = (rp * CLUSTER + crank) * BM + r_local;
+      const bool row_ok = row < n_valid;
+      int32_t y = -1;
+      if (row_ok) {
+        const int64_t orig = p.rowidx ? static_cast<int64_t>(p.rowidx[row]) : row;
+        y = p.targets[orig];
       }
-      tc_fence_after();
-      const int32_t n0 = (tile0 + t) * BN;
-      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * BN;
+      float m = -INFINITY, s = 0.0f, tgt = 0.0f;
+      bool have_tgt = false;
+      for (int t = tile0; t < tile1; ++t, ++tcount) {
+        const uint32_t acc = tcount & 1u;
+        const uint32_t acc_ph = (tcount >> 1) & 1u;
+        if (!mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag)) {
+          if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+          *abort_flag = 1;
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int32_t n0 = t * BN;
+        const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * BN;
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        float v[32];
-        tmem_ld_32x32b_x32(tbase + c, v);
-        tmem_wait_ld();
-        const int32_t col0 = n0 + c;
-        if (col0 + 32 > p.V) {
+        for (int cc = 0; cc < BN; cc += 32) {
+          float v[32];
+          tmem_ld_32x32b_x32(tbase + cc, v);
+          tmem_wait_ld();
+          const int32_t col0 = n0 + cc;
+          if (col0 + 32 > p.V) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (col0 + i >= p.V) v[i] = -INFINITY;
+            for (int i = 0; i < 32; ++i)
+              if (col0 + i >= p.V) v[i] = -INFINITY;
+          }
+          float cm = v[0];
+#pragma unroll
+          for (int i = 1; i < 32; ++i) cm = fmaxf(cm, v[i]);
+          const float m_new = fmaxf(m, cm * scale);
+          float acc_s = 0.0f;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) acc_s += ex2_approx(fmaf(v[i], scale, -m_new));
+          s = s * ex2_approx(m - m_new) + acc_s;
+          m = m_new;
+          const uint32_t off = static_cast<uint32_t>(y - col0);
+          if (off < 32u) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (off == static_cast<uint32_t>(i)) tgt = v[i];
+            have_tgt = true;
+          }
         }
-        float cm = v[0];
-#pragma unroll
-        for (int i = 1; i < 32; ++i) cm = fmaxf(cm, v[i]);
-        const float m_new = fmaxf(m, cm * scale);
-        float acc_s = 0.0f;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) acc_s += ex2_approx(fmaf(v[i], scale, -m_new));
-        s = s * ex2_approx(m - m_new) + acc_s;
-        m = m_new;
-        const uint32_t off = static_cast<uint32_t>(y - col0);
-        if (off < 32u) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (off == static_cast<uint32_t>(i)) tgt = v[i];
-          have_tgt = true;
-        }
+        tc_fence_before();
+        mbar_arrive(&tmem_empty[acc]);
       }
-      tc_fence_before();
-      mbar_arrive(&tmem_empty[acc]);
-    }
-    if (row_ok) {
-      const int64_t o = row * p.splits + split;
-      p.part_m[o] = m;
-      p.part_s[o] = s;
-      if (have_tgt) p.tgt_logit[row] = tgt;
+      if (row_ok && ok) {
+        const int64_t o = row * p.splits + split;
+        p.part_m[o] = m;
+        p.part_s[o] = s;
+        if (have_tgt) p.tgt_logit[row] = tgt;
+      }
     }
   }
 
   tc_fence_before();
   __syncthreads();
+  // neither CTA leaves while its peer may still multicast into it or arrive on it
+  cluster_sync();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
 }
@@ -370,16 +403,41 @@ void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, bool c
   w->tgt = cv.take<float>(static_cast<size_t>(rows_cap));
 }
 
-pace_status set_smem_attr() {
-  static int done_dev = -1;
+struct LmLaunchInfo {
+  int max_clusters = 0;
+};
+
+// Dynamic shared memory opt-in and the number of 2-CTA clusters that can be
+// resident at once on the current device (cached per device).
+pace_status lm_launch_info(LmLaunchInfo* out) {
+  constexpr int kMaxDevices = 64;
+  static LmLaunchInfo info[kMaxDevices];
   static std::mutex mu;
   int dev = 0;
   PACE_TRY_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return PACE_ERR_CUDA;
   std::lock_guard<std::mutex> g(mu);
-  if (done_dev == dev) return PACE_OK;
-  PACE_TRY_CUDA(cudaFuncSetAttribute(lmhead_lse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(kSmemBytes)));
-  done_dev = dev;
+  if (info[dev].max_clusters == 0) {
+    PACE_TRY_CUDA(cudaFuncSetAttribute(lmhead_lse_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(kSmemBytes)));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(sm_count()), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = CLUSTER;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, lmhead_lse_kernel, &cfg) != cudaSuccess || n < 1)
+      n = sm_count() / CLUSTER;
+    info[dev].max_clusters = n;
+  }
+  *out = info[dev];
   return PACE_OK;
 }
 
@@ -445,8 +503,9 @@ extern "C" pace_status pace_token_logprob(const PaceBatch* batch, const void* hi
     const int tps = (n_vtiles + S - 1) / S;
     CUtensorMap tm_a, tm_b;
     PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, BM));
-    PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, BN));
-    PACE_TRY(set_smem_attr());
+    PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, BN / CLUSTER));
+    LmLaunchInfo li;
+    PACE_TRY(lm_launch_info(&li));
     LmArgs a;
     a.rows_cap = rows_cap;
     a.n_valid_dev = n_valid_dev;
@@ -462,9 +521,10 @@ extern "C" pace_status pace_token_logprob(const PaceBatch* batch, const void* hi
     a.part_s = ws.part_s;
     a.tgt_logit = ws.tgt;
     a.status = status_dev;
-    const int64_t row_blocks = (rows_cap + BM - 1) / BM;
-    const int64_t grid = row_blocks * S;
-    if (grid > 0x7fffffff) return PACE_ERR_UNSUPPORTED_SHAPE;
+    // persistent: at most one wave of 2-CTA clusters, never more clusters than items
+    const int64_t items = (rows_cap + 2 * BM - 1) / (2 * BM) * S;
+    const int64_t clusters = items < li.max_clusters ? items : li.max_clusters;
+    const int64_t grid = clusters * CLUSTER;
     const ProfileEvents& pe = profile_events(PACE_PROFILE_LMHEAD);
     if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
     lmhead_lse_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tm_a, tm_b, a);

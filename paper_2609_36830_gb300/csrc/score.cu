@@ -69,12 +69,33 @@ __device__ __forceinline__ void flush(LaneAcc& a, int64_t traj, unsigned long lo
   a.maxp1 = 0;
 }
 
+// Sum, count and max of a batch that lies inside one trajectory and holds only
+// policy tags below 2^26: then 32 tags fit a 32-bit sum.  Returns false (and
+// leaves acc untouched) when the batch needs the general per-element path.
+__device__ __forceinline__ bool acc_batch_fast(LaneAcc& a, const int4 (&v)[kTilesPerBatch]) {
+  int mx = v[0].x, mn = v[0].x;
+#pragma unroll
+  for (int u = 0; u < kTilesPerBatch; ++u) {
+    mx = max(max(mx, v[u].x), max(v[u].y, max(v[u].z, v[u].w)));
+    mn = min(min(mn, v[u].x), min(v[u].y, min(v[u].z, v[u].w)));
+  }
+  if (mn < 0 || mx >= (1 << 26)) return false;
+  int s = 0;
+#pragma unroll
+  for (int u = 0; u < kTilesPerBatch; ++u) s += (v[u].x + v[u].y) + (v[u].z + v[u].w);
+  a.sum += s;
+  a.cnt += 4 * kTilesPerBatch;
+  const unsigned mp1 = static_cast<unsigned>(mx) + 1u;
+  a.maxp1 = mp1 > a.maxp1 ? mp1 : a.maxp1;
+  return true;
+}
+
 // Each warp owns a contiguous range of 1024-token batches of the flattened
 // tag stream and walks the CSR offsets forward through it, so trajectories of
 // any length mix are balanced across warps.  The walk never leaves
 // [0, n_traj) and loads only tags[0, n_tokens), whatever the offsets hold;
 // inconsistent offsets are reported by the finalize kernel.
-__global__ void __launch_bounds__(kReduceThreads)
+__global__ void __launch_bounds__(kReduceThreads, 3)
     tag_reduce_kernel(const int32_t* __restrict__ tags, const int64_t* __restrict__ offsets,
                       int64_t n_traj, int64_t n_tokens, unsigned long long* __restrict__ sumv,
                       unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1) {
@@ -102,12 +123,14 @@ __global__ void __launch_bounds__(kReduceThreads)
     const int64_t bt0 = b * kBatchTokens;
     const int64_t bt1 = (bt0 + kBatchTokens < n_tokens) ? bt0 + kBatchTokens : n_tokens;
     int4 v[kTilesPerBatch];
+    if (bt0 + kBatchTokens <= n_tokens) {
 #pragma unroll
-    for (int u = 0; u < kTilesPerBatch; ++u) {
-      const int64_t t = bt0 + u * kTileTokens + lane * 4;
-      if (t + 3 < n_tokens) {
-        v[u] = ld_stream_v4(tags + t);
-      } else {
+      for (int u = 0; u < kTilesPerBatch; ++u)
+        v[u] = ld_stream_v4(tags + bt0 + u * kTileTokens + lane * 4);
+    } else {
+#pragma unroll
+      for (int u = 0; u < kTilesPerBatch; ++u) {
+        const int64_t t = bt0 + u * kTileTokens + lane * 4;
         v[u].x = (t + 0 < n_tokens) ? tags[t + 0] : -1;
         v[u].y = (t + 1 < n_tokens) ? tags[t + 1] : -1;
         v[u].z = (t + 2 < n_tokens) ? tags[t + 2] : -1;
@@ -117,23 +140,27 @@ __global__ void __launch_bounds__(kReduceThreads)
     int64_t pos = bt0;
     while (true) {
       const int64_t seg_hi = cur_end < bt1 ? cur_end : bt1;
-      if (pos == bt0 && seg_hi == bt1) {
+      if (pos == bt0 && seg_hi == bt0 + kBatchTokens) {
         // whole batch inside one trajectory: no position tests
+        if (!acc_batch_fast(acc, v)) {
 #pragma unroll
-        for (int u = 0; u < kTilesPerBatch; ++u) {
-          acc_elem(acc, v[u].x, true);
-          acc_elem(acc, v[u].y, true);
-          acc_elem(acc, v[u].z, true);
-          acc_elem(acc, v[u].w, true);
+          for (int u = 0; u < kTilesPerBatch; ++u) {
+            acc_elem(acc, v[u].x, true);
+            acc_elem(acc, v[u].y, true);
+            acc_elem(acc, v[u].z, true);
+            acc_elem(acc, v[u].w, true);
+          }
         }
       } else if (seg_hi > pos) {
+        // batch-relative bounds fit 32 bits
+        const int lo_r = static_cast<int>(pos - bt0), hi_r = static_cast<int>(seg_hi - bt0);
 #pragma unroll
         for (int u = 0; u < kTilesPerBatch; ++u) {
-          const int64_t t = bt0 + u * kTileTokens + lane * 4;
-          acc_elem(acc, v[u].x, t + 0 >= pos && t + 0 < seg_hi);
-          acc_elem(acc, v[u].y, t + 1 >= pos && t + 1 < seg_hi);
-          acc_elem(acc, v[u].z, t + 2 >= pos && t + 2 < seg_hi);
-          acc_elem(acc, v[u].w, t + 3 >= pos && t + 3 < seg_hi);
+          const int t = u * kTileTokens + lane * 4;
+          acc_elem(acc, v[u].x, t + 0 >= lo_r && t + 0 < hi_r);
+          acc_elem(acc, v[u].y, t + 1 >= lo_r && t + 1 < hi_r);
+          acc_elem(acc, v[u].z, t + 2 >= lo_r && t + 2 < hi_r);
+          acc_elem(acc, v[u].w, t + 3 >= lo_r && t + 3 < hi_r);
         }
       }
       if (cur_end > bt1) break;  // trajectory continues into the next batch
@@ -328,7 +355,7 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
     const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
     const int warps_per_block = kReduceThreads / 32;
     int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
-    const int64_t cap = static_cast<int64_t>(sm_count()) * 4;
+    const int64_t cap = static_cast<int64_t>(sm_count()) * 3;  // one wave at 3 blocks / SM
     if (blocks > cap) blocks = cap;
     const ProfileEvents& pe = profile_events(PACE_PROFILE_TAG_REDUCE);
     if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
