@@ -99,18 +99,16 @@ class ClockSampler:
 
 
 def _dist():
-    ws = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return ws, rank, local
+    from paper_2609_36830_gb300 import replicas
+    return replicas.rank_env()
 
 
 def _make_step(seed_offset, device):
     import torch
     from paper_2609_36830_gb300 import pace, step, workloads
     spec = workloads.SPECS[WORKLOAD]
-    pool = workloads.make_pool(WORKLOAD, seed=workloads.SEED_BASE + spec.index + 1000 * seed_offset
-                               if seed_offset else None)
+    from paper_2609_36830_gb300 import replicas
+    pool = workloads.make_pool(WORKLOAD, seed=replicas.replica_seed(WORKLOAD, seed_offset))
     rows = workloads.make_rows(pool)
     H, V = spec.hidden, spec.vocab
     hidden = workloads.bf16_normal_device((rows.n_rows, H), 1.0, pool.seed + 11, device=device)
@@ -316,17 +314,16 @@ def run_gpu(args):
     launches = pace.kernel_launches() - launches0
     assert int(st.status.item()) == 0, pace.status_string(int(st.status.item()))
     ms = t_b.elapsed_time(t_e) / K
+    from paper_2609_36830_gb300 import replicas
+    job_rows, ms = replicas.job_totals(M, ms, device)
     if ws > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
         dist.barrier()
     lm_each = [b.elapsed_time(e) for b, e in zip(k_b, k_e)]
     lm_ms = statistics.mean(lm_each)
     flops = 2.0 * H * V * M
     achieved = flops / (lm_ms / 1e3) / 1e12
     peak_s = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
-    value = M * ws / (ms / 1e3)
+    value = job_rows / (ms / 1e3)
 
     # end to end through the same C ABI with host buffers: pinned host copies of
     # every input, copied in each step; the loss and log-probs copied out.
@@ -355,10 +352,7 @@ def run_gpu(args):
     e_e.record()
     torch.cuda.synchronize()
     e_ms = e_b.elapsed_time(e_e) / e_steps
-    if ws > 1:
-        t = torch.tensor([e_ms], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e_ms = float(t.item())
+    _, e_ms = replicas.job_totals(M, e_ms, device)
     del host
 
     sweep = None
@@ -393,7 +387,7 @@ def run_gpu(args):
                          "kernel_ms": lm_ms, "kernel_ms_each": lm_each,
                          "flops_per_launch": flops, "traffic": None},
             "cpu_baseline": cpu,
-            "e2e": {"value": M * ws / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "e2e": {"value": job_rows / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e_ms},
             "gpu_launches": launches,
             "clocks": clk.summary(),
@@ -462,8 +456,8 @@ def run_case(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
-    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--cpu-rows", type=int, default=64)
     ap.add_argument("--no-sweep", action="store_true")
