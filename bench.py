@@ -34,6 +34,12 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOAD = "math7b"
+# DRAM bytes per unit from the committed ncu captures of the current kernels
+# (profiles/lmhead_lse_kernel_one_wave.md: 1.135 GB for one full round of 4864 rows, W read
+# once per round, so traffic grows with the rows processed; profiles/tag_reduce_kernel_sweep16k.md:
+# 223.2 MB for 54.93 M tags).  Set to None when a kernel changes until it is captured again.
+LMHEAD_DRAM_BYTES_PER_ROW = 1.135e9 / 4864
+TAG_REDUCE_DRAM_BYTES_PER_TAG = 223.155e6 / 54929421
 SWEEP_N = 1048576
 METRIC = "accepted tokens/sec (logprob+loss) and % bf16 tensor peak; pool scoring traj/s + HBM GB/s"
 UNIT = "tokens/s"
@@ -171,9 +177,63 @@ def _sweep_scoring(steps, warmup, device):
     # the 16-byte per-trajectory accumulators written once
     k_bytes = 4 * tok + 8 * (n + 1) + 16 * n
     res = {"workload": f"sweep pool {n} trajectories, {tok} tags", "traj_per_s": n / (s_ms / 1e3),
+           "tag_reduce_traffic": (TAG_REDUCE_DRAM_BYTES_PER_TAG * tok
+                                  if TAG_REDUCE_DRAM_BYTES_PER_TAG else None),
            "ms_per_call": s_ms, "tag_reduce_ms": k_ms,
            "tag_reduce_gbs": k_bytes / (k_ms / 1e3) / 1e9, "tag_reduce_bytes": k_bytes}
     del pool, flush
+    torch.cuda.empty_cache()
+    return res
+
+
+def _prefix_scoring(steps, warmup, device):
+    """pace_prefix_score (Eq. 6) on every interrupted prefix of the math pool: the
+    rollout-side overhead the paper measures for PACE (prefix rescoring)."""
+    import torch
+    from paper_2609_36830_gb300 import pace, workloads
+    spec = workloads.SPECS[WORKLOAD]
+    pool = workloads.make_pool(WORKLOAD)
+    rows = workloads.make_rows(pool)
+    pre = workloads.make_prefixes(pool, rows)
+    H, V = spec.hidden, spec.vocab
+    hidden = workloads.bf16_normal_device((pre.n_rows, H), 1.0, pool.seed + 31, device=device)
+    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), pool.seed + 32, device=device)
+    targets = torch.from_numpy(rows.targets[pre.rows]).to(device)
+    behav = torch.from_numpy((workloads.uniform_center(V) + np.random.default_rng(3)
+                              .standard_normal(pre.n_rows) * 0.3).astype(np.float32)).to(device)
+    b = pace.make_batch(torch.from_numpy(pre.seq_offsets).to(device), pre.n_rows,
+                        mask=torch.from_numpy(pre.mask).to(device))
+    s_pre = torch.empty(len(pre.traj), dtype=torch.float32, device=device)
+    lp = torch.empty(pre.n_rows, dtype=torch.float32, device=device)
+    ws = pace.workspace(pace.lib().pace_prefix_score_workspace_size(pre.n_rows, len(pre.traj),
+                                                                    H, V), device)
+    status = pace.new_status(device)
+    for _ in range(warmup):
+        pace.prefix_score(b, hidden, w, targets, behav, cap_tokens=1024, s_pre=s_pre, logprob=lp,
+                          ws=ws, status=status)
+    torch.cuda.synchronize()
+    scored = int((lp != 0).sum().item())
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    kv = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    for i in range(steps):
+        pace.set_profile_events(pace.PROFILE_LMHEAD, *kv[i])
+        ev[i][0].record()
+        pace.prefix_score(b, hidden, w, targets, behav, cap_tokens=1024, s_pre=s_pre, logprob=lp,
+                          ws=ws, status=status)
+        ev[i][1].record()
+    pace.set_profile_events(pace.PROFILE_LMHEAD)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0, pace.status_string(int(status.item()))
+    ms = statistics.mean(a.elapsed_time(z) for a, z in ev)
+    k_ms = statistics.mean(a.elapsed_time(z) for a, z in kv)
+    res = {"workload": f"{len(pre.traj)} interrupted prefixes of the {WORKLOAD} pool, "
+                       f"{pre.n_rows} rows, first 1024 eligible tokens scored",
+           "prefixes": len(pre.traj), "rows_scored": scored, "ms_per_call": ms,
+           "rows_scored_per_s": scored / (ms / 1e3), "lmhead_ms": k_ms,
+           "lmhead_tflops": 2.0 * H * V * scored / (k_ms / 1e3) / 1e12}
+    del hidden, w, ws
     torch.cuda.empty_cache()
     return res
 
@@ -363,6 +423,10 @@ def run_gpu(args):
         sweep["tag_reduce_frac_of_hbm"] = sweep["tag_reduce_gbs"] / peaks["hbm_gbs"]
         sweep["hbm_peak_gbs"] = peaks["hbm_gbs"]
 
+    prefix = None
+    if not args.no_sweep and rank == 0:
+        prefix = _prefix_scoring(max(3, min(K, 5)), 3, device)
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         if sweep is not None:
@@ -385,13 +449,18 @@ def run_gpu(args):
                          "frac_of_burst": achieved / peaks["bf16_tflops"],
                          "frac_of_nominal_2250": achieved / 2250.0,
                          "kernel_ms": lm_ms, "kernel_ms_each": lm_each,
-                         "flops_per_launch": flops, "traffic": None},
+                         "flops_per_launch": flops,
+                         "traffic": (LMHEAD_DRAM_BYTES_PER_ROW * M
+                                     if LMHEAD_DRAM_BYTES_PER_ROW else None),
+                         "traffic_note": "dram read+write bytes per launch, scaled by rows from "
+                                         "the one-round ncu capture"},
             "cpu_baseline": cpu,
             "e2e": {"value": job_rows / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e_ms},
             "gpu_launches": launches,
             "clocks": clk.summary(),
             "pool_scoring": sweep,
+            "prefix_scoring": prefix,
         }
         print(json.dumps(line), flush=True)
     if ws > 1:

@@ -302,6 +302,38 @@ PACE_API pace_status pace_surrogate_loss(const PaceBatch* batch, const float* lo
 
 PACE_API size_t pace_surrogate_loss_workspace_size(int64_t n_rows, int64_t n_seq);
 
+/* Prefix Forgetting Score (Eq. 6, Sec. 3.2) with the collection rules of the
+ * admission settings.  Each sequence of the batch is an interrupted rollout's
+ * prefix (prompt plus the response tokens generated before a weight sync),
+ * whose hidden states come from a forward pass of the updated rollout policy
+ * u.  For each prefix,
+ *   s_pre = (1/m) sum |log pi_u(y_t | x, y_<t) - l^mu_t|
+ * over its first m = min(#eligible, cap_tokens) eligible rows (row order),
+ * with log pi_u from the same fused LM head as pace_token_logprob; s_pre is NaN
+ * when fewer than min_tokens rows are eligible (the paper requires 32; its caps
+ * are 1,024 response tokens for math and 2,048 for ReTool).
+ *   batch      seq_offsets over the prefix rows; mask marks eligible rows (policy
+ *              response tokens; prompt and tool rows 0); NULL = every row;
+ *              seq_accepted, if given, makes unaccepted prefixes empty.
+ *   hidden, w_vocab, targets, hidden_size, vocab_size, temperature: as for
+ *              pace_token_logprob, under policy u.
+ *   behav_lp   device float32 [n_rows]: recorded behaviour log-probs l^mu_t.
+ *   s_pre      device float32 [n_seq] (output), the input pace_score_pool takes.
+ *   logprob    device float32 [n_rows] (output: log pi_u of the scored rows, 0
+ *              elsewhere) or NULL (kept in the workspace).
+ * The mean is an fp64 sum in a fixed order; device-side errors as for
+ * pace_token_logprob. */
+PACE_API pace_status pace_prefix_score(const PaceBatch* batch, const void* hidden,
+                                       const void* w_vocab, const int32_t* targets,
+                                       const float* behav_lp, int32_t hidden_size,
+                                       int32_t vocab_size, float temperature, int32_t min_tokens,
+                                       int32_t cap_tokens, float* s_pre, float* logprob,
+                                       void* workspace, size_t workspace_bytes,
+                                       int32_t* status_dev, void* stream);
+
+PACE_API size_t pace_prefix_score_workspace_size(int64_t n_rows, int64_t n_seq,
+                                                 int32_t hidden_size, int32_t vocab_size);
+
 /* ------------------------------------------------------------------------ */
 /* Profiling                                                                 */
 /* ------------------------------------------------------------------------ */

@@ -64,6 +64,7 @@ def _load():
                 "oracle_group_advantages": [_P, _P, _I64, _I32, _F64, _I32, _P],
                 "oracle_surrogate": [_P, _P, _P, _P, _P, _I64, _P, _F64, _F64, _F64, _I32, _P,
                                      _P, _P],
+                "oracle_prefix_score": [_P, _P, _P, _P, _I64, _I32, _I32, _P],
             }
             for name, args in sig.items():
                 fn = getattr(lib, name)
@@ -200,3 +201,13 @@ def surrogate(logprob, behav_lp, seq_offsets, adv, mask=None, seq_accepted=None,
                                   _ptr(a), float(eps_low), float(eps_high), float(dual_clip),
                                   int(agg), ctypes.byref(loss), _ptr(ratio), _ptr(term))
     return st, loss.value, ratio, term
+
+
+def prefix_score(logprob, behav_lp, seq_offsets, mask=None, min_tokens=32, cap_tokens=1024):
+    """Eq. 6 Prefix Forgetting Score per prefix: (status, s_pre fp64, NaN = not scored)."""
+    lp, bl = _c(logprob, np.float64), _c(behav_lp, np.float64)
+    so, m = _c(seq_offsets, np.int64), _c(mask, np.uint8)
+    out = np.zeros(so.size - 1, np.float64)
+    st = _load().oracle_prefix_score(_ptr(lp), _ptr(bl), _ptr(m), _ptr(so), so.size - 1,
+                                     int(min_tokens), int(cap_tokens), _ptr(out))
+    return st, out

@@ -380,29 +380,6 @@ int choose_splits(int n_vtiles) {
   return s;
 }
 
-struct LmWs {
-  CompactWs cw;
-  SurrogateWs sw;
-  void* hidden_c;  // gathered rows [n_rows][H] (null when no compaction)
-  float* part_m;
-  float* part_s;
-  float* tgt;
-};
-
-void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, bool compact,
-                 LmWs* w) {
-  const int n_vtiles = (V + BN - 1) / BN;
-  const int S = choose_splits(n_vtiles);
-  const int64_t rows_cap = n_rows > BM ? n_rows : BM;
-  carve_compact_ws(cv, n_seq, n_rows, &w->cw);
-  carve_surrogate_ws(cv, n_seq, &w->sw);
-  w->hidden_c = compact ? static_cast<void*>(cv.take<uint16_t>(static_cast<size_t>(rows_cap) * H))
-                        : nullptr;
-  w->part_m = cv.take<float>(static_cast<size_t>(rows_cap) * S);
-  w->part_s = cv.take<float>(static_cast<size_t>(rows_cap) * S);
-  w->tgt = cv.take<float>(static_cast<size_t>(rows_cap));
-}
-
 struct LmLaunchInfo {
   int max_clusters = 0;
 };
@@ -442,6 +419,103 @@ pace_status lm_launch_info(LmLaunchInfo* out) {
 }
 
 }  // namespace
+
+void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, bool compact,
+                 LmWs* w) {
+  const int n_vtiles = (V + BN - 1) / BN;
+  const int S = choose_splits(n_vtiles);
+  const int64_t rows_cap = n_rows > BM ? n_rows : BM;
+  carve_compact_ws(cv, n_seq, n_rows, &w->cw);
+  carve_surrogate_ws(cv, n_seq, &w->sw);
+  w->hidden_c = compact ? static_cast<void*>(cv.take<uint16_t>(static_cast<size_t>(rows_cap) * H))
+                        : nullptr;
+  w->part_m = cv.take<float>(static_cast<size_t>(rows_cap) * S);
+  w->part_s = cv.take<float>(static_cast<size_t>(rows_cap) * S);
+  w->tgt = cv.take<float>(static_cast<size_t>(rows_cap));
+}
+
+bool lm_needs_compaction(const PaceBatch* b) {
+  return b->mask || b->seq_accepted || b->n_rows < BM;
+}
+
+pace_status check_lm_args(const PaceBatch* batch, const void* hidden, const void* w_vocab,
+                          const int32_t* targets, int H, int V, float temperature,
+                          const float* logprob) {
+  PACE_TRY(check_batch(batch));
+  if (H < 64 || H > 16384 || H % 64 != 0) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (V < 1 || V > (1 << 24)) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (!(temperature > 0.0f) || !isfinite(temperature)) return PACE_ERR_INVALID_ARG;
+  if (batch->n_rows > 0 && (!hidden || !w_vocab || !targets || !logprob))
+    return PACE_ERR_INVALID_ARG;
+  if (!aligned(hidden, 16) || !aligned(w_vocab, 16)) return PACE_ERR_UNSUPPORTED_SHAPE;
+  return PACE_OK;
+}
+
+// Compaction, gather, fused LM head and merge: lp (and lse) for every row in
+// the batch's loss, 0 elsewhere.
+pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* w_vocab,
+                        const int32_t* targets, int H, int V, float temperature, float* logprob,
+                        float* lse, const LmWs& ws, int32_t* status_dev, cudaStream_t st) {
+  const int64_t n_rows = batch->n_rows;
+  const bool compact = lm_needs_compaction(batch);
+  if (n_rows > 0) {
+    PACE_TRY_CUDA(cudaMemsetAsync(logprob, 0, static_cast<size_t>(n_rows) * sizeof(float), st));
+    if (lse) PACE_TRY_CUDA(cudaMemsetAsync(lse, 0, static_cast<size_t>(n_rows) * sizeof(float), st));
+  }
+  const void* a_ptr = hidden;
+  const long long* n_valid_dev = nullptr;
+  const int32_t* rowidx = nullptr;
+  int64_t rows_cap = n_rows;
+  if (compact) {
+    PACE_TRY(run_compaction(batch, ws.cw, status_dev, st));
+    PACE_TRY(run_gather(hidden, H, n_rows, ws.cw, ws.hidden_c, st));
+    a_ptr = ws.hidden_c;
+    n_valid_dev = ws.cw.total;
+    rowidx = ws.cw.rowidx;
+    rows_cap = n_rows > BM ? n_rows : BM;
+  }
+  if (n_rows == 0) return PACE_OK;
+  const int n_vtiles = (V + BN - 1) / BN;
+  const int S = choose_splits(n_vtiles);
+  const int tps = (n_vtiles + S - 1) / S;
+  CUtensorMap tm_a, tm_b;
+  PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, BM));
+  PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, BN / CLUSTER));
+  LmLaunchInfo li;
+  PACE_TRY(lm_launch_info(&li));
+  LmArgs a;
+  a.rows_cap = rows_cap;
+  a.n_valid_dev = n_valid_dev;
+  a.H = H;
+  a.V = V;
+  a.n_vtiles = n_vtiles;
+  a.splits = S;
+  a.tiles_per_split = tps;
+  a.scale_log2 = 1.4426950408889634f / temperature;
+  a.targets = targets;
+  a.rowidx = rowidx;
+  a.part_m = ws.part_m;
+  a.part_s = ws.part_s;
+  a.tgt_logit = ws.tgt;
+  a.status = status_dev;
+  // persistent: at most one wave of 2-CTA clusters, never more clusters than items
+  const int64_t items = (rows_cap + 2 * BM - 1) / (2 * BM) * S;
+  const int64_t clusters = items < li.max_clusters ? items : li.max_clusters;
+  const int64_t grid = clusters * CLUSTER;
+  const ProfileEvents& pe = profile_events(PACE_PROFILE_LMHEAD);
+  if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
+  lmhead_lse_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tm_a, tm_b, a);
+  PACE_TRY(last_launch_status());
+  if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
+  int64_t mblocks = (rows_cap + 255) / 256;
+  const int64_t cap = static_cast<int64_t>(sm_count()) * 8;
+  if (mblocks > cap) mblocks = cap;
+  lse_merge_kernel<<<static_cast<unsigned>(mblocks), 256, 0, st>>>(
+      rows_cap, n_valid_dev, S, V, 1.0f / temperature, ws.part_m, ws.part_s, ws.tgt, targets,
+      rowidx, logprob, lse, status_dev);
+  return last_launch_status();
+}
+
 }  // namespace pace
 
 using namespace pace;
@@ -462,82 +536,18 @@ extern "C" pace_status pace_token_logprob(const PaceBatch* batch, const void* hi
                                           const PaceLossArgs* loss, void* workspace,
                                           size_t workspace_bytes, int32_t* status_dev,
                                           void* stream) {
-  PACE_TRY(check_batch(batch));
+  PACE_TRY(check_lm_args(batch, hidden, w_vocab, targets, hidden_size, vocab_size, temperature,
+                         logprob));
   if (loss) PACE_TRY(check_loss_args(batch, loss));
-  const int H = hidden_size, V = vocab_size;
-  if (H < 64 || H > 16384 || H % 64 != 0) return PACE_ERR_UNSUPPORTED_SHAPE;
-  if (V < 1 || V > (1 << 24)) return PACE_ERR_UNSUPPORTED_SHAPE;
-  if (!(temperature > 0.0f) || !isfinite(temperature)) return PACE_ERR_INVALID_ARG;
-  const int64_t n_rows = batch->n_rows;
-  if (n_rows > 0 && (!hidden || !w_vocab || !targets || !logprob)) return PACE_ERR_INVALID_ARG;
-  if (!aligned(hidden, 16) || !aligned(w_vocab, 16)) return PACE_ERR_UNSUPPORTED_SHAPE;
   if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
-  cudaStream_t st = as_stream(stream);
-  // Compaction is skipped only when every row is in the loss and there are
-  // enough rows for a full TMA box.
-  const bool compact = batch->mask || batch->seq_accepted || n_rows < BM;
   Carver cv(workspace, workspace_bytes);
   LmWs ws;
-  carve_lm_ws(cv, n_rows, batch->n_seq, H, V, compact, &ws);
+  carve_lm_ws(cv, batch->n_rows, batch->n_seq, hidden_size, vocab_size,
+              lm_needs_compaction(batch), &ws);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
-
-  if (n_rows > 0) {
-    PACE_TRY_CUDA(cudaMemsetAsync(logprob, 0, static_cast<size_t>(n_rows) * sizeof(float), st));
-    if (lse) PACE_TRY_CUDA(cudaMemsetAsync(lse, 0, static_cast<size_t>(n_rows) * sizeof(float), st));
-  }
-  const void* a_ptr = hidden;
-  const long long* n_valid_dev = nullptr;
-  const int32_t* rowidx = nullptr;
-  int64_t rows_cap = n_rows;
-  if (compact) {
-    PACE_TRY(run_compaction(batch, ws.cw, status_dev, st));
-    PACE_TRY(run_gather(hidden, H, n_rows, ws.cw, ws.hidden_c, st));
-    a_ptr = ws.hidden_c;
-    n_valid_dev = ws.cw.total;
-    rowidx = ws.cw.rowidx;
-    rows_cap = n_rows > BM ? n_rows : BM;
-  }
-  if (n_rows > 0) {
-    const int n_vtiles = (V + BN - 1) / BN;
-    const int S = choose_splits(n_vtiles);
-    const int tps = (n_vtiles + S - 1) / S;
-    CUtensorMap tm_a, tm_b;
-    PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, BM));
-    PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, BN / CLUSTER));
-    LmLaunchInfo li;
-    PACE_TRY(lm_launch_info(&li));
-    LmArgs a;
-    a.rows_cap = rows_cap;
-    a.n_valid_dev = n_valid_dev;
-    a.H = H;
-    a.V = V;
-    a.n_vtiles = n_vtiles;
-    a.splits = S;
-    a.tiles_per_split = tps;
-    a.scale_log2 = 1.4426950408889634f / temperature;
-    a.targets = targets;
-    a.rowidx = rowidx;
-    a.part_m = ws.part_m;
-    a.part_s = ws.part_s;
-    a.tgt_logit = ws.tgt;
-    a.status = status_dev;
-    // persistent: at most one wave of 2-CTA clusters, never more clusters than items
-    const int64_t items = (rows_cap + 2 * BM - 1) / (2 * BM) * S;
-    const int64_t clusters = items < li.max_clusters ? items : li.max_clusters;
-    const int64_t grid = clusters * CLUSTER;
-    const ProfileEvents& pe = profile_events(PACE_PROFILE_LMHEAD);
-    if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
-    lmhead_lse_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tm_a, tm_b, a);
-    PACE_TRY(last_launch_status());
-    if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
-    int64_t mblocks = (rows_cap + 255) / 256;
-    const int64_t cap = static_cast<int64_t>(sm_count()) * 8;
-    if (mblocks > cap) mblocks = cap;
-    lse_merge_kernel<<<static_cast<unsigned>(mblocks), 256, 0, st>>>(
-        rows_cap, n_valid_dev, S, V, 1.0f / temperature, ws.part_m, ws.part_s, ws.tgt, targets,
-        rowidx, logprob, lse, status_dev);
-    PACE_TRY(last_launch_status());
-  }
+  cudaStream_t st = as_stream(stream);
+  PACE_TRY(run_logprob(batch, hidden, w_vocab, targets, hidden_size, vocab_size, temperature,
+                       logprob, lse, ws, status_dev, st));
   if (loss) PACE_TRY(run_surrogate(batch, logprob, loss, ws.sw, status_dev, st));
   return PACE_OK;
 }

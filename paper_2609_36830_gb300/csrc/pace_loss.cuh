@@ -19,7 +19,26 @@ struct CompactWs {
   int32_t* rowidx;      // [n_rows]: compact row -> original row
 };
 
+// Workspace of the log-prob pipeline (compaction, gathered rows, split partials).
+struct LmWs {
+  CompactWs cw;
+  SurrogateWs sw;
+  void* hidden_c;  // gathered rows [max(n_rows, 128)][H] (null when no compaction)
+  float* part_m;
+  float* part_s;
+  float* tgt;
+};
+
 void carve_surrogate_ws(Carver& cv, int64_t n_seq, SurrogateWs* w);
+void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, bool compact,
+                 LmWs* w);
+bool lm_needs_compaction(const PaceBatch* b);
+pace_status check_lm_args(const PaceBatch* batch, const void* hidden, const void* w_vocab,
+                          const int32_t* targets, int H, int V, float temperature,
+                          const float* logprob);
+pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* w_vocab,
+                        const int32_t* targets, int H, int V, float temperature, float* logprob,
+                        float* lse, const LmWs& ws, int32_t* status_dev, cudaStream_t st);
 void carve_compact_ws(Carver& cv, int64_t n_seq, int64_t n_rows, CompactWs* w);
 pace_status check_batch(const PaceBatch* b);
 pace_status check_loss_args(const PaceBatch* b, const PaceLossArgs* l);

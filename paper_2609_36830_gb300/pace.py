@@ -83,6 +83,9 @@ SIGNATURES = {
     "pace_token_logprob_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
     "pace_surrogate_loss": ([_P, _P, _P, _P, _SZ, _P, _P], _I32),
     "pace_surrogate_loss_workspace_size": ([_I64, _I64], _SZ),
+    "pace_prefix_score": ([_P, _P, _P, _P, _P, _I32, _I32, _F32, _I32, _I32, _P, _P, _P, _SZ,
+                           _P, _P], _I32),
+    "pace_prefix_score_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
     "pace_set_profile_events": ([_I32, _P, _P], _I32),
     "pace_kernel_launches": ([], ctypes.c_uint64),
 }
@@ -328,3 +331,25 @@ def set_profile_events(kernel: int, begin=None, end=None):
 def kernel_launches() -> int:
     """Kernels the library has launched from this thread so far."""
     return int(lib().pace_kernel_launches())
+
+
+def prefix_score(batch: PaceBatch, hidden, w_vocab, targets, behav_lp, temperature=1.0,
+                 min_tokens=32, cap_tokens=1024, s_pre=None, logprob=None, ws=None, status=None,
+                 stream=None):
+    """pace_prefix_score (Eq. 6): float32 s_pre per prefix (NaN = not scored)."""
+    if hidden.dtype != torch.bfloat16 or w_vocab.dtype != torch.bfloat16:
+        raise ValueError("hidden and w_vocab must be bf16")
+    n_rows, H = hidden.shape
+    V = w_vocab.shape[0]
+    dev = hidden.device
+    if s_pre is None:
+        s_pre = torch.empty(batch.n_seq, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(lib().pace_prefix_score_workspace_size(n_rows, batch.n_seq, H, V), dev)
+    st = lib().pace_prefix_score(ctypes.byref(batch), _ptr(_dev(hidden)), _ptr(_dev(w_vocab)),
+                                 _ptr(_dev(targets)), _ptr(_dev(behav_lp)), int(H), int(V),
+                                 float(temperature), int(min_tokens), int(cap_tokens),
+                                 _ptr(s_pre), _ptr(logprob), _ptr(ws), ws.numel(), _ptr(status),
+                                 _stream(stream))
+    _check(st, "pace_prefix_score")
+    return s_pre

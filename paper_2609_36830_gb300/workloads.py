@@ -218,7 +218,7 @@ def make_pool(name: str, seed: Optional[int] = None, n_traj: Optional[int] = Non
     return Pool(spec, seed, n, j, G, _target_for(spec, n), offsets if device is None else
                 _to_device(offsets, device), tags, c.astype(np.int32), s_pre_v, window, reward,
                 lens, np.full(n, spec.prompt_len, np.int64), n_int,
-                meta={"offsets_host": offsets})
+                meta={"offsets_host": offsets, "last_interrupt": last.astype(np.int64)})
 
 
 def _target_for(spec, n):
@@ -310,7 +310,8 @@ def _make_multiturn(spec, seed, n, r_len, r_ver, r_int, r_pre, r_win, r_rew, dev
     return Pool(spec, seed, n, j, spec.group_size, spec.n_target,
                 offsets if device is None else _to_device(offsets, device), tags,
                 np.array(c, np.int32), s_pre_v, window, reward, lens,
-                np.zeros(n, np.int64), n_int, meta={"offsets_host": offsets})
+                np.zeros(n, np.int64), n_int,
+                meta={"offsets_host": offsets, "last_interrupt": last})
 
 
 # ---------------------------------------------------------------------------
@@ -401,3 +402,29 @@ def bf16_normal_device(shape, std: float, seed: int, device="cuda", chunk_rows: 
             x.mul_(std)
         out[r0:r1].copy_(x)
     return out
+
+
+@dataclass
+class PrefixBatch:
+    """Prefixes of the pool's interrupted rollouts, for re-scoring (Eq. 6).
+
+    Prefix i is trajectory ``traj[i]``'s prompt plus the response tokens generated
+    before its last weight-sync interruption; ``rows`` are its row indices in the
+    pool's row layout and ``mask`` marks the eligible (policy-generated) rows.
+    """
+    traj: np.ndarray         # int64 [n_prefix]
+    seq_offsets: np.ndarray  # int64 [n_prefix+1]
+    rows: np.ndarray         # int64 [n_rows] pool row of each prefix row
+    mask: np.ndarray         # uint8 [n_rows]
+    n_rows: int
+
+
+def make_prefixes(pool: Pool, rows: Rows) -> PrefixBatch:
+    last = pool.meta["last_interrupt"]
+    traj = np.nonzero(last >= 1)[0].astype(np.int64)
+    plen = pool.prompt_len[traj] + last[traj]
+    seq_offsets = np.concatenate([[0], np.cumsum(plen)]).astype(np.int64)
+    starts = rows.row_offsets[traj]
+    idx = np.repeat(starts, plen) + _ramp(plen)
+    return PrefixBatch(traj, seq_offsets, idx.astype(np.int64), rows.mask[idx].copy(),
+                       int(seq_offsets[-1]))
