@@ -302,6 +302,61 @@ PACE_API pace_status pace_surrogate_loss(const PaceBatch* batch, const float* lo
 
 PACE_API size_t pace_surrogate_loss_workspace_size(int64_t n_rows, int64_t n_seq);
 
+/* The literal admission rule of Sec. 3.1 and Algorithm 1 (trainer side), kept
+ * across steps with a sliding window of recently observed unit scores:
+ *   kappa = Quantile_{1 - r}(W^M)  (inverted-CDF: the k-th smallest window
+ *           score, k = max(ceil((1 - r) |W| - 1e-9), 1); +inf while the window
+ *           holds fewer than min_obs scores),
+ * then candidates are drawn in the given order: score > kappa is rejected
+ * (decision 0), the rest retained (1) until batch_units are retained, and the
+ * candidates after that are not drawn (2; batch_units <= 0 draws all).  Every
+ * drawn score then enters the window.
+ *   unit_score   device float64 [n_cand], in draw order.
+ *   r_hat        host: the budget, min(r-hat_j, r_max) from pace_budget.
+ *   window       device float64 [capacity], capacity <= 4096 (the paper uses 512
+ *                groups); window_state device int64 [2] = {count, next slot},
+ *                zero-initialised by the caller once; both updated in place.
+ *   decision     device uint8 [n_cand] (output); kappa device float64 [1] (output).
+ * pace_select is the same rule with the window taken as the current pool. */
+PACE_API pace_status pace_quantile_admit(const double* unit_score, int64_t n_cand,
+                                         double r_hat, int64_t batch_units, int32_t min_obs,
+                                         double* window, int64_t capacity,
+                                         int64_t* window_state, uint8_t* decision,
+                                         double* kappa, int32_t* status_dev, void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* Stale-k admission and staleness diagnostics                               */
+/* ------------------------------------------------------------------------ */
+
+/* Stale-k admission, the prior-work baseline of Sec. 2 ("Controlled Stale-k
+ * Analysis"): trajectory tau is admitted when its token-weighted policy lag
+ *   kbar(tau; j) = (1/T) sum_t (j - v_t)                      (Eq. 1)
+ * is at most k_max (kbar == k_max is admitted; T = 0 gives kbar = 0).  kbar is
+ * computed from exact integer sums with one rounding.  tags / offsets /
+ * n_tokens / trainer_version as for pace_score_pool; kbar device float64
+ * [n_traj] (output, may be NULL); admitted device uint8 [n_traj] (output).
+ * Device-side errors: PACE_ERR_VERSION_ORDER when a tag exceeds j,
+ * PACE_ERR_INVALID_ARG for tags below -1 or bad offsets. */
+PACE_API pace_status pace_stale_k(const int32_t* tags, const int64_t* offsets, int64_t n_traj,
+                                  int64_t n_tokens, int32_t trainer_version, double k_max,
+                                  double* kbar, uint8_t* admitted, void* workspace,
+                                  size_t workspace_bytes, int32_t* status_dev, void* stream);
+
+PACE_API size_t pace_stale_k_workspace_size(int64_t n_traj);
+
+/* Histograms of a per-unit staleness value (K_wait, K_gen, K_eff, s_pre, ...)
+ * for rejected and accepted units, as in the paper's retained-vs-rejected
+ * admission analysis.  n_bins (1..4096) equal-width bins over [lo, hi): the bin
+ * of x is floor((x - lo) / (hi - lo) * n_bins) in fp64, values below lo count
+ * in the first bin and values at or above hi in the last.  hist is device
+ * uint32 [2 * n_bins] (output): [0, n_bins) rejected (flag 0), [n_bins,
+ * 2 n_bins) accepted; with flags NULL every value counts in the first half.
+ * Exact integer counts; NaN values are skipped and reported as
+ * PACE_ERR_NAN_INPUT. */
+PACE_API pace_status pace_staleness_histogram(const double* values, const uint8_t* flags,
+                                              int64_t n, double lo, double hi, int32_t n_bins,
+                                              uint32_t* hist, int32_t* status_dev, void* stream);
+
 /* Prefix Forgetting Score (Eq. 6, Sec. 3.2) with the collection rules of the
  * admission settings.  Each sequence of the batch is an interrupted rollout's
  * prefix (prompt plus the response tokens generated before a weight sync),

@@ -65,6 +65,9 @@ def _load():
                 "oracle_surrogate": [_P, _P, _P, _P, _P, _I64, _P, _F64, _F64, _F64, _I32, _P,
                                      _P, _P],
                 "oracle_prefix_score": [_P, _P, _P, _P, _I64, _I32, _I32, _P],
+                "oracle_stale_k": [_P, _P, _I64, _I32, _F64, _P, _P],
+                "oracle_histogram": [_P, _P, _I64, _F64, _F64, _I32, _P],
+                "oracle_quantile_admit": [_P, _I64, _F64, _I64, _I32, _P, _I64, _P, _P, _P, _P],
             }
             for name, args in sig.items():
                 fn = getattr(lib, name)
@@ -211,3 +214,45 @@ def prefix_score(logprob, behav_lp, seq_offsets, mask=None, min_tokens=32, cap_t
     st = _load().oracle_prefix_score(_ptr(lp), _ptr(bl), _ptr(m), _ptr(so), so.size - 1,
                                      int(min_tokens), int(cap_tokens), _ptr(out))
     return st, out
+
+
+def stale_k(tags, offsets, j, k_max):
+    """Stale-k admission: (status, kbar fp64, admitted uint8)."""
+    tags, offsets = _c(tags, np.int32), _c(offsets, np.int64)
+    n = offsets.size - 1
+    kbar, adm = np.zeros(n, np.float64), np.zeros(n, np.uint8)
+    st = _load().oracle_stale_k(_ptr(tags), _ptr(offsets), n, int(j), float(k_max), _ptr(kbar),
+                                _ptr(adm))
+    return st, kbar, adm
+
+
+def histogram(values, flags, lo, hi, n_bins):
+    """(status, hist uint32 [2, n_bins]): row 0 rejected (flag 0), row 1 accepted."""
+    v = _c(values, np.float64)
+    f = _c(flags, np.uint8)
+    h = np.zeros(2 * n_bins, np.uint32)
+    st = _load().oracle_histogram(_ptr(v), _ptr(f), v.size, float(lo), float(hi), int(n_bins),
+                                  _ptr(h))
+    return st, h.reshape(2, n_bins)
+
+
+class Window:
+    """Ring window of recently observed scores (state of oracle_quantile_admit)."""
+
+    def __init__(self, capacity):
+        self.values = np.zeros(capacity, np.float64)
+        self.count = 0
+        self.head = 0
+
+
+def quantile_admit(scores, r, batch_units, window: Window, min_obs=32):
+    """Sec. 3.1 / Algorithm 1 rule; updates ``window``: (status, decision uint8, kappa)."""
+    sc = _c(scores, np.float64)
+    dec = np.zeros(sc.size, np.uint8)
+    cnt, hd, kap = ctypes.c_int64(window.count), ctypes.c_int64(window.head), ctypes.c_double()
+    st = _load().oracle_quantile_admit(_ptr(sc), sc.size, float(r), int(batch_units),
+                                       int(min_obs), _ptr(window.values), window.values.size,
+                                       ctypes.byref(cnt), ctypes.byref(hd), _ptr(dec),
+                                       ctypes.byref(kap))
+    window.count, window.head = cnt.value, hd.value
+    return st, dec, kap.value

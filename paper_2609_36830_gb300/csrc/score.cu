@@ -284,6 +284,31 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
   }
 }
 
+// Stale-k admission (Sec. 2): kbar = sum (j - v_t) / T = (j T - sum v_t) / T in
+// exact integers, one rounding; admitted when kbar <= k_max.
+__global__ void stale_k_kernel(const int64_t* __restrict__ offsets,
+                               const unsigned long long* __restrict__ sumv,
+                               const unsigned* __restrict__ cnt, const unsigned* __restrict__ maxp1,
+                               int64_t n_traj, int64_t n_tokens, int32_t j, double k_max,
+                               double* __restrict__ kbar, uint8_t* __restrict__ admitted,
+                               int32_t* status) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n_traj) return;
+  const int64_t o0 = offsets[i], o1 = offsets[i + 1];
+  if (o1 < o0 || (i == 0 && o0 != 0) || (i == n_traj - 1 && o1 != n_tokens))
+    report(status, PACE_ERR_INVALID_ARG);
+  const unsigned t_count = cnt[i];
+  const unsigned mp1 = maxp1[i];
+  if (mp1 >= 0x80000000u) report(status, PACE_ERR_INVALID_ARG);
+  if (mp1 != 0u && static_cast<int64_t>(mp1) - 1 > j) report(status, PACE_ERR_VERSION_ORDER);
+  const long long lag_sum = static_cast<long long>(j) * static_cast<long long>(t_count) -
+                            static_cast<long long>(sumv[i]);
+  const double kb =
+      t_count > 0u ? __ddiv_rn(__ll2double_rn(lag_sum), __ull2double_rn(t_count)) : 0.0;
+  if (kbar) kbar[i] = kb;
+  admitted[i] = kb <= k_max ? 1 : 0;
+}
+
 struct ScoreWs {
   unsigned long long* sumv;
   unsigned* cnt;
@@ -299,10 +324,56 @@ ScoreWs carve_score_ws(Carver& cv, int64_t n_traj) {
   return w;
 }
 
+// Zero the accumulators and stream the tags once.
+pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t n_traj,
+                           int64_t n_tokens, const ScoreWs& ws, cudaStream_t st) {
+  PACE_TRY_CUDA(cudaMemsetAsync(ws.sumv, 0, static_cast<size_t>(n_traj) * 16, st));
+  if (n_tokens == 0) return PACE_OK;
+  const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
+  const int warps_per_block = kReduceThreads / 32;
+  int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
+  const int64_t cap = static_cast<int64_t>(sm_count()) * 3;  // one wave at 3 blocks / SM
+  if (blocks > cap) blocks = cap;
+  const ProfileEvents& pe = profile_events(PACE_PROFILE_TAG_REDUCE);
+  if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
+  tag_reduce_kernel<<<static_cast<unsigned>(blocks), kReduceThreads, 0, st>>>(
+      tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1);
+  PACE_TRY(last_launch_status());
+  if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
+  return PACE_OK;
+}
+
 }  // namespace
 }  // namespace pace
 
 using namespace pace;
+
+extern "C" size_t pace_stale_k_workspace_size(int64_t n_traj) {
+  return pace_score_pool_workspace_size(n_traj, 0);
+}
+
+extern "C" pace_status pace_stale_k(const int32_t* tags, const int64_t* offsets, int64_t n_traj,
+                                    int64_t n_tokens, int32_t trainer_version, double k_max,
+                                    double* kbar, uint8_t* admitted, void* workspace,
+                                    size_t workspace_bytes, int32_t* status_dev, void* stream) {
+  if (n_traj < 0 || n_tokens < 0 || n_traj > (int64_t(1) << 31)) return PACE_ERR_INVALID_ARG;
+  if (n_traj > 0 && (!offsets || !admitted)) return PACE_ERR_INVALID_ARG;
+  if (n_tokens > 0 && !tags) return PACE_ERR_INVALID_ARG;
+  if (isnan(k_max)) return PACE_ERR_INVALID_ARG;
+  if (tags && !aligned(tags, 16)) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (n_traj == 0) return n_tokens == 0 ? PACE_OK : PACE_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
+  Carver cv(workspace, workspace_bytes);
+  ScoreWs ws = carve_score_ws(cv, n_traj);
+  if (!cv.fits()) return PACE_ERR_WORKSPACE;
+  cudaStream_t st = as_stream(stream);
+  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, st));
+  const int threads = 256;
+  stale_k_kernel<<<static_cast<unsigned>((n_traj + threads - 1) / threads), threads, 0, st>>>(
+      offsets, ws.sumv, ws.cnt, ws.maxp1, n_traj, n_tokens, trainer_version, k_max, kbar,
+      admitted, status_dev);
+  return last_launch_status();
+}
 
 extern "C" void pace_score_params_default(PaceScoreParams* p) {
   if (!p) return;
@@ -350,20 +421,7 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
 
   cudaStream_t st = as_stream(stream);
-  PACE_TRY_CUDA(cudaMemsetAsync(ws.sumv, 0, static_cast<size_t>(n_traj) * 16, st));
-  if (n_tokens > 0) {
-    const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
-    const int warps_per_block = kReduceThreads / 32;
-    int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
-    const int64_t cap = static_cast<int64_t>(sm_count()) * 3;  // one wave at 3 blocks / SM
-    if (blocks > cap) blocks = cap;
-    const ProfileEvents& pe = profile_events(PACE_PROFILE_TAG_REDUCE);
-    if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
-    tag_reduce_kernel<<<static_cast<unsigned>(blocks), kReduceThreads, 0, st>>>(
-        tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1);
-    PACE_TRY(last_launch_status());
-    if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
-  }
+  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, st));
   FinalizeArgs a;
   a.offsets = offsets;
   a.c_version = c_version;

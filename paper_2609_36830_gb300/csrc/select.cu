@@ -444,6 +444,180 @@ extern "C" pace_status pace_select(const double* unit_score, int64_t n_units, in
 }
 
 // ---------------------------------------------------------------------------
+// Staleness diagnostics: histograms of a per-unit value for rejected and
+// accepted units (the paper's retained-vs-rejected admission analysis).
+// ---------------------------------------------------------------------------
+
+namespace pace {
+namespace {
+
+constexpr int kMaxHistBins = 4096;
+
+__global__ void staleness_hist_kernel(const double* __restrict__ values,
+                                      const uint8_t* __restrict__ flags, int64_t n, double lo,
+                                      double hi, int n_bins, unsigned* __restrict__ hist,
+                                      int32_t* status) {
+  extern __shared__ unsigned h[];  // [2 * n_bins]
+  for (int b = threadIdx.x; b < 2 * n_bins; b += blockDim.x) h[b] = 0;
+  __syncthreads();
+  const double width = __dsub_rn(hi, lo);
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const double x = values[i];
+    if (isnan(x)) {
+      report(status, PACE_ERR_NAN_INPUT);
+      continue;
+    }
+    int b;
+    if (x < lo) b = 0;
+    else if (x >= hi) b = n_bins - 1;
+    else {
+      const double f = floor(__dmul_rn(__ddiv_rn(__dsub_rn(x, lo), width), (double)n_bins));
+      b = f > (double)(n_bins - 1) ? n_bins - 1 : static_cast<int>(f);
+    }
+    atomicAdd(&h[(flags && flags[i] ? n_bins : 0) + b], 1u);
+  }
+  __syncthreads();
+  for (int b = threadIdx.x; b < 2 * n_bins; b += blockDim.x)
+    if (h[b]) atomicAdd(&hist[b], h[b]);
+}
+
+}  // namespace
+}  // namespace pace
+
+extern "C" pace_status pace_staleness_histogram(const double* values, const uint8_t* flags,
+                                                int64_t n, double lo, double hi, int32_t n_bins,
+                                                uint32_t* hist, int32_t* status_dev,
+                                                void* stream) {
+  if (n < 0 || n_bins < 1 || n_bins > kMaxHistBins || !(hi > lo) || !isfinite(lo) ||
+      !isfinite(hi) || !hist || (n > 0 && !values))
+    return PACE_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream);
+  PACE_TRY_CUDA(cudaMemsetAsync(hist, 0, sizeof(uint32_t) * 2 * n_bins, st));
+  if (n == 0) return PACE_OK;
+  staleness_hist_kernel<<<grid_for(n, 256, 4), 256, sizeof(unsigned) * 2 * n_bins, st>>>(
+      values, flags, n, lo, hi, n_bins, hist, status_dev);
+  return last_launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// The literal sliding-window quantile rule (Sec. 3.1, Algorithm 1).
+// ---------------------------------------------------------------------------
+
+namespace pace {
+namespace {
+
+constexpr int kMaxWindowSlots = 4096;
+constexpr int kAdmitThreads = 1024;
+
+// One block: sort the window's recent scores in shared memory (bitonic, +inf
+// padding), take the inverted-CDF (1 - r) quantile, decide the candidates in
+// draw order with block scans, then append the drawn scores to the ring.
+__global__ void __launch_bounds__(kAdmitThreads)
+    quantile_admit_kernel(const double* __restrict__ score, int64_t n_cand, double r,
+                          int64_t batch_units, int32_t min_obs, double* __restrict__ window,
+                          int64_t capacity, long long* __restrict__ state,
+                          uint8_t* __restrict__ decision, double* __restrict__ kappa_out,
+                          int32_t* status) {
+  __shared__ double sw[kMaxWindowSlots];
+  __shared__ long long s_retained, s_drawn;
+  const long long n = state[0], head = state[1];
+  if (n < 0 || n > capacity || head < 0 || head >= capacity) {
+    if (threadIdx.x == 0) report(status, PACE_ERR_INVALID_ARG);
+    return;
+  }
+  double kappa = __longlong_as_double(0x7ff0000000000000ll);  // +inf: no threshold
+  if (n > 0 && n >= min_obs) {
+    int pw = 1;
+    while (pw < n) pw <<= 1;
+    for (int t = threadIdx.x; t < pw; t += blockDim.x)
+      sw[t] = t < n ? window[(head - n + t + capacity) % capacity]
+                    : __longlong_as_double(0x7ff0000000000000ll);
+    __syncthreads();
+    for (int size = 2; size <= pw; size <<= 1) {
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        for (int t = threadIdx.x; t < pw; t += blockDim.x) {
+          const int u = t ^ stride;
+          if (u > t) {
+            const bool up = (t & size) == 0;
+            const double a = sw[t], b = sw[u];
+            if ((a > b) == up) {
+              sw[t] = b;
+              sw[u] = a;
+            }
+          }
+        }
+        __syncthreads();
+      }
+    }
+    long long k = static_cast<long long>(
+        ceil(__dsub_rn(__dmul_rn(__dsub_rn(1.0, r), static_cast<double>(n)), 1e-9)));
+    if (k < 1) k = 1;
+    if (k > n) k = n;
+    kappa = sw[k - 1];
+  }
+  if (threadIdx.x == 0) {
+    s_retained = 0;
+    s_drawn = 0;
+    *kappa_out = kappa;
+  }
+  __syncthreads();
+  for (int64_t c0 = 0; c0 < n_cand; c0 += blockDim.x) {
+    const int64_t i = c0 + threadIdx.x;
+    const double x = i < n_cand ? score[i] : 0.0;
+    if (i < n_cand && isnan(x)) report(status, PACE_ERR_NAN_INPUT);
+    const int keep = (i < n_cand && !(x > kappa)) ? 1 : 0;
+    int tot = 0;
+    const int before = block_exclusive_scan<int>(keep, &tot);
+    const long long ret0 = s_retained;
+    if (i < n_cand) {
+      const bool drawn = batch_units <= 0 || ret0 + before < batch_units;
+      decision[i] = drawn ? (keep ? 1 : 0) : 2;
+    }
+    int last_drawn = -1;  // last candidate of this chunk that was drawn
+    if (i < n_cand && (batch_units <= 0 || ret0 + before < batch_units))
+      last_drawn = threadIdx.x;
+    int chunk_drawn = 0;
+    block_exclusive_scan<int>(last_drawn >= 0 ? 1 : 0, &chunk_drawn);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      s_retained = ret0 + tot;
+      s_drawn += chunk_drawn;
+    }
+    __syncthreads();
+  }
+  // append the drawn scores (in draw order) to the ring; when more were drawn
+  // than the ring holds, only the newest `capacity` of them survive
+  const long long drawn = s_drawn;
+  const long long keep_n = drawn < capacity ? drawn : capacity;
+  for (long long t = drawn - keep_n + threadIdx.x; t < drawn; t += blockDim.x)
+    window[(head + t) % capacity] = score[t];
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    state[1] = (head + drawn) % capacity;
+    state[0] = n + drawn < capacity ? n + drawn : capacity;
+  }
+}
+
+}  // namespace
+}  // namespace pace
+
+extern "C" pace_status pace_quantile_admit(const double* unit_score, int64_t n_cand,
+                                           double r_hat, int64_t batch_units, int32_t min_obs,
+                                           double* window, int64_t capacity,
+                                           int64_t* window_state, uint8_t* decision,
+                                           double* kappa, int32_t* status_dev, void* stream) {
+  if (n_cand < 0 || capacity < 1 || capacity > pace::kMaxWindowSlots || !window ||
+      !window_state || !kappa || (n_cand > 0 && (!unit_score || !decision)))
+    return PACE_ERR_INVALID_ARG;
+  if (!(r_hat >= 0.0 && r_hat <= 1.0)) return PACE_ERR_INVALID_ARG;
+  pace::quantile_admit_kernel<<<1, pace::kAdmitThreads, 0, pace::as_stream(stream)>>>(
+      unit_score, n_cand, r_hat, batch_units, min_obs, window, capacity,
+      reinterpret_cast<long long*>(window_state), decision, kappa, status_dev);
+  return pace::last_launch_status();
+}
+
+// ---------------------------------------------------------------------------
 // Selection without a caller-provided workspace.
 //
 // For callers that may not allocate device memory themselves, the radix path's

@@ -86,6 +86,10 @@ SIGNATURES = {
     "pace_prefix_score": ([_P, _P, _P, _P, _P, _I32, _I32, _F32, _I32, _I32, _P, _P, _P, _SZ,
                            _P, _P], _I32),
     "pace_prefix_score_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
+    "pace_stale_k": ([_P, _P, _I64, _I64, _I32, _F64, _P, _P, _P, _SZ, _P, _P], _I32),
+    "pace_stale_k_workspace_size": ([_I64], _SZ),
+    "pace_staleness_histogram": ([_P, _P, _I64, _F64, _F64, _I32, _P, _P, _P], _I32),
+    "pace_quantile_admit": ([_P, _I64, _F64, _I64, _I32, _P, _I64, _P, _P, _P, _P, _P], _I32),
     "pace_set_profile_events": ([_I32, _P, _P], _I32),
     "pace_kernel_launches": ([], ctypes.c_uint64),
 }
@@ -353,3 +357,57 @@ def prefix_score(batch: PaceBatch, hidden, w_vocab, targets, behav_lp, temperatu
                                  _stream(stream))
     _check(st, "pace_prefix_score")
     return s_pre
+
+
+def stale_k(tags, offsets, trainer_version, k_max, kbar=None, admitted=None, ws=None,
+            status=None, stream=None):
+    """pace_stale_k: (kbar float64, admitted uint8) per trajectory."""
+    dev = offsets.device
+    n = offsets.numel() - 1
+    if kbar is None:
+        kbar = torch.empty(n, dtype=torch.float64, device=dev)
+    if admitted is None:
+        admitted = torch.empty(n, dtype=torch.uint8, device=dev)
+    if ws is None:
+        ws = workspace(lib().pace_stale_k_workspace_size(n), dev)
+    st = lib().pace_stale_k(_ptr(tags), _ptr(_dev(offsets)), n, tags.numel(),
+                            int(trainer_version), float(k_max), _ptr(kbar), _ptr(admitted),
+                            _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    _check(st, "pace_stale_k")
+    return kbar, admitted
+
+
+def staleness_histogram(values, flags, lo, hi, n_bins, hist=None, status=None, stream=None):
+    """pace_staleness_histogram: int32-viewable uint32 counts [2, n_bins] (rejected, accepted)."""
+    if hist is None:
+        hist = torch.empty(2 * n_bins, dtype=torch.int32, device=values.device)
+    st = lib().pace_staleness_histogram(_ptr(_dev(values)), _ptr(flags), values.numel(),
+                                        float(lo), float(hi), int(n_bins), _ptr(hist),
+                                        _ptr(status), _stream(stream))
+    _check(st, "pace_staleness_histogram")
+    return hist.view(2, n_bins)
+
+
+class ScoreWindow:
+    """Device ring window of recent unit scores for quantile_admit (state kept across steps)."""
+
+    def __init__(self, capacity=512, device="cuda"):
+        self.values = torch.zeros(capacity, dtype=torch.float64, device=device)
+        self.state = torch.zeros(2, dtype=torch.int64, device=device)  # count, next slot
+
+
+def quantile_admit(unit_score, r_hat, batch_units, window: ScoreWindow, min_obs=32,
+                   decision=None, kappa=None, status=None, stream=None):
+    """pace_quantile_admit: (decision uint8 [n], kappa float64 [1]); updates ``window``."""
+    n = unit_score.numel()
+    dev = unit_score.device
+    if decision is None:
+        decision = torch.empty(max(n, 1), dtype=torch.uint8, device=dev)
+    if kappa is None:
+        kappa = torch.empty(1, dtype=torch.float64, device=dev)
+    st = lib().pace_quantile_admit(_ptr(_dev(unit_score)), n, float(r_hat), int(batch_units),
+                                   int(min_obs), _ptr(window.values), window.values.numel(),
+                                   _ptr(window.state), _ptr(decision), _ptr(kappa),
+                                   _ptr(status), _stream(stream))
+    _check(st, "pace_quantile_admit")
+    return decision[:n], kappa

@@ -230,3 +230,28 @@ def test_errors():
         oracle.ERR_NAN_INPUT
     assert oracle.score_pool(tags, offsets, c, s_pre, 10, window, group_size=4)[0] == \
         oracle.ERR_INVALID_ARG  # 6 trajectories are not whole groups of 4
+
+
+def test_stale_k_admission_on_hand_pool():
+    h = _hand()
+    tags, offsets, c, _, _ = _pool_arrays(h)
+    kbars = [_frac(t["kbar"]) for t in h["trajectories"]]  # 0, 5/2, 4, 1, 9/2, 5/4
+    for k in (0.0, 1.0, 1.25, 2.5, 4.0, 4.5, 10.0):
+        st, kbar, adm = oracle.stale_k(tags, offsets, 10, k)
+        assert st == oracle.OK
+        for i, kb in enumerate(kbars):
+            assert Fraction(kbar[i]) == kb
+            assert adm[i] == (1 if kb <= Fraction(k) else 0), (k, i)  # kbar == k admitted
+
+
+def test_histogram_hand_counts():
+    vals = np.array([-1.0, 0.0, 0.49, 0.5, 0.99, 1.0, 1.5, 7.0])
+    flags = np.array([0, 1, 1, 0, 1, 0, 1, 1], np.uint8)
+    st, h = oracle.histogram(vals, flags, 0.0, 1.0, 2)
+    assert st == oracle.OK
+    # bins [0, .5) and [.5, 1); below lo -> bin 0, at or above hi -> bin 1
+    assert h[0].tolist() == [1, 2]  # rejected: -1.0 | 0.5, 1.0
+    assert h[1].tolist() == [2, 3]  # accepted: 0.0, 0.49 | 0.99, 1.5, 7.0
+    assert h.sum() == vals.size
+    st, h = oracle.histogram(np.array([np.nan]), None, 0.0, 1.0, 4)
+    assert st == oracle.ERR_NAN_INPUT

@@ -107,3 +107,48 @@ def test_select_matches_brute_force(seed):
 
 def test_select_errors():
     assert oracle.select(np.array([1.0, np.nan]), 1, 1)[0] == oracle.ERR_NAN_INPUT
+
+
+def test_quantile_admit_hand_worked():
+    # window {1..8}, r = 1/4: type-1 quantile at 3/4 -> 6th smallest = 6; reject scores > 6
+    w = oracle.Window(8)
+    st, dec, kappa = oracle.quantile_admit(np.arange(1, 9, dtype=np.float64), 0.0, 0, w,
+                                           min_obs=100)
+    assert st == 0 and kappa == math.inf and (dec == 1).all()  # below min_obs: no threshold
+    assert w.count == 8 and w.head == 0
+    st, dec, kappa = oracle.quantile_admit([7.0, 2.0, 6.0, 9.0, 1.0, 3.0], 0.25, 3, w, min_obs=4)
+    assert st == 0 and kappa == 6.0
+    # draw: 7 rejected, 2 kept, 6 kept (ties at kappa kept), 9 rejected, 1 kept -> 3 kept, stop
+    assert dec.tolist() == [0, 1, 1, 0, 1, 2]
+    # the five drawn scores replaced the five oldest window slots
+    assert w.count == 8 and w.head == 5
+    assert sorted(w.values.tolist()) == sorted([6.0, 7.0, 8.0, 7.0, 2.0, 6.0, 9.0, 1.0])
+
+
+def test_quantile_admit_matches_numpy_inverted_cdf():
+    rng = np.random.default_rng(8)
+    for _ in range(200):
+        n = int(rng.integers(1, 600))
+        vals = np.round(rng.random(n) * 20, 1)
+        # dyadic r: (1 - r) * n is exact in fp64, so numpy's quantile and the
+        # rule agree without the 1e-9 nudge
+        r = float(rng.choice([0.0, 0.125, 0.25, 0.5, 0.75, 0.875, 1.0]))
+        w = oracle.Window(1024)
+        w.values[:n] = vals
+        w.count, w.head = n, n % 1024
+        st, dec, kappa = oracle.quantile_admit(np.zeros(0), r, 0, w, min_obs=1)
+        assert st == 0
+        p = 1.0 - r
+        expect = np.quantile(vals, max(p, 1e-12), method="inverted_cdf")
+        assert kappa == expect, (n, r)
+
+
+def test_quantile_admit_rank_is_the_real_number_rank():
+    # r = 1/3 over 189 values: (1 - r) n is 126 as a real number but 126.00000000000001
+    # in fp64; the rule takes the 126th smallest (reading: the nudge), not the 127th.
+    vals = np.arange(1, 190, dtype=np.float64)
+    w = oracle.Window(256)
+    w.values[:189] = vals
+    w.count, w.head = 189, 189
+    st, _, kappa = oracle.quantile_admit(np.zeros(0), 1 / 3, 0, w, min_obs=1)
+    assert st == 0 and kappa == 126.0
