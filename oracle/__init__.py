@@ -68,6 +68,9 @@ def _load():
                 "oracle_stale_k": [_P, _P, _I64, _I32, _F64, _P, _P],
                 "oracle_histogram": [_P, _P, _I64, _F64, _F64, _I32, _P],
                 "oracle_quantile_admit": [_P, _I64, _F64, _I64, _I32, _P, _I64, _P, _P, _P, _P],
+                "oracle_surrogate_grad": [_P, _P, _P, _P, _P, _I64, _P, _F64, _F64, _F64, _I32,
+                                          _P],
+                "oracle_lmhead_backward": [_P, _P, _P, _P, _I64, _I32, _I32, _F64, _P, _P, _I32],
             }
             for name, args in sig.items():
                 fn = getattr(lib, name)
@@ -256,3 +259,32 @@ def quantile_admit(scores, r, batch_units, window: Window, min_obs=32):
                                        ctypes.byref(kap))
     window.count, window.head = cnt.value, hd.value
     return st, dec, kap.value
+
+
+def surrogate_grad(logprob, behav_lp, seq_offsets, adv, mask=None, seq_accepted=None,
+                   eps_low=0.2, eps_high=0.28, dual_clip=10.0, agg=AGG_TOKEN_MEAN):
+    """dLoss/dlp per row of the clipped surrogate: (status, dlp fp64)."""
+    lp, bl = _c(logprob, np.float64), _c(behav_lp, np.float64)
+    so, a = _c(seq_offsets, np.int64), _c(adv, np.float64)
+    m, sa = _c(mask, np.uint8), _c(seq_accepted, np.uint8)
+    out = np.zeros(lp.size, np.float64)
+    st = _load().oracle_surrogate_grad(_ptr(lp), _ptr(bl), _ptr(m), _ptr(so), _ptr(sa),
+                                       so.size - 1, _ptr(a), float(eps_low), float(eps_high),
+                                       float(dual_clip), int(agg), _ptr(out))
+    return st, out
+
+
+def lmhead_backward(hidden_bits, w_bits, targets, g, temperature=1.0, with_dw=True,
+                    n_threads=None):
+    """(status, dH fp64 [n_rows, H], dW fp64 [V, H] or None) for dLoss/dlp = g."""
+    hb, wb = _c(hidden_bits, np.uint16), _c(w_bits, np.uint16)
+    tg, gg = _c(targets, np.int32), _c(g, np.float64)
+    n, H = hb.shape
+    V = wb.shape[0]
+    dh = np.zeros((n, H), np.float64)
+    dw = np.zeros((V, H), np.float64) if with_dw else None
+    if n_threads is None:
+        n_threads = min(os.cpu_count() or 1, 64)
+    st = _load().oracle_lmhead_backward(_ptr(hb), _ptr(wb), _ptr(tg), _ptr(gg), n, H, V,
+                                        float(temperature), _ptr(dh), _ptr(dw), int(n_threads))
+    return st, dh, dw
