@@ -238,6 +238,50 @@ def _prefix_scoring(steps, warmup, device):
     return res
 
 
+def _lmhead_backward(steps, warmup, device):
+    """pace_surrogate_backward + pace_token_logprob_backward on the math step's accepted rows:
+    3 x 2 H V FLOP per row in the loss (recomputed logits, G W, G^T H)."""
+    import torch
+    from paper_2609_36830_gb300 import pace
+    pool, rows, x, st = _make_step(0, device)
+    st.run()
+    torch.cuda.synchronize()
+    M = st.rows_in_loss()
+    H, V = x.hidden.shape[1], x.w_vocab.shape[0]
+    lse = torch.empty(x.mask.numel(), dtype=torch.float32, device=device)
+    ws_f = pace.workspace(pace.token_logprob_workspace_size(x.mask.numel(), st.n_traj, H, V),
+                          device)
+    pace.token_logprob(st.batch, x.hidden, x.w_vocab, x.targets, 1.0, logprob=st.logprob, lse=lse,
+                       ws=ws_f, status=st.status)
+    del ws_f
+    dlp = pace.surrogate_backward(st.batch, st.logprob, st.loss_args, status=st.status)
+    gh = torch.empty(x.mask.numel(), H, dtype=torch.float32, device=device)
+    gw = torch.empty(V, H, dtype=torch.float32, device=device)
+    ws = pace.workspace(pace.lib().pace_token_logprob_backward_workspace_size(
+        x.mask.numel(), st.n_traj, H, V), device)
+    for _ in range(warmup):
+        pace.token_logprob_backward(st.batch, x.hidden, x.w_vocab, x.targets, lse, dlp,
+                                    grad_hidden=gh, grad_w=gw, ws=ws, status=st.status)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    for b, e in ev:
+        b.record()
+        pace.token_logprob_backward(st.batch, x.hidden, x.w_vocab, x.targets, lse, dlp,
+                                    grad_hidden=gh, grad_w=gw, ws=ws, status=st.status)
+        e.record()
+    torch.cuda.synchronize()
+    assert int(st.status.item()) == 0, pace.status_string(int(st.status.item()))
+    ms = statistics.mean(b.elapsed_time(e) for b, e in ev)
+    flops = 3 * 2.0 * H * V * M
+    res = {"workload": f"{WORKLOAD} step's {M} rows in the loss, H {H}, V {V}",
+           "ms_per_call": ms, "rows_per_s": M / (ms / 1e3),
+           "tflops": flops / (ms / 1e3) / 1e12, "flops_per_call": flops}
+    del gh, gw, ws, x, st
+    torch.cuda.empty_cache()
+    return res
+
+
 def _cpu_baseline(pool, rows, x, step_obj, n_rows_sample):
     """The oracle as it stands on this host's cores: full admission + a row sample."""
     import torch
@@ -447,8 +491,12 @@ def run_gpu(args):
         sweep["hbm_peak_gbs"] = peaks["hbm_gbs"]
 
     prefix = None
+    backward = None
     if not args.no_sweep and rank == 0:
         prefix = _prefix_scoring(max(3, min(K, 5)), 3, device)
+        backward = _lmhead_backward(3, 1, device)
+        peak_s_b = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+        backward["frac_of_sustained"] = backward["tflops"] / peak_s_b
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -484,6 +532,7 @@ def run_gpu(args):
             "clocks": clk.summary(),
             "pool_scoring": sweep,
             "prefix_scoring": prefix,
+            "lmhead_backward": backward,
         }
         print(json.dumps(line), flush=True)
     if ws > 1:

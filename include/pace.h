@@ -390,6 +390,49 @@ PACE_API size_t pace_prefix_score_workspace_size(int64_t n_rows, int64_t n_seq,
                                                  int32_t hidden_size, int32_t vocab_size);
 
 /* ------------------------------------------------------------------------ */
+/* Backward: gradients for the unchanged policy update                       */
+/* ------------------------------------------------------------------------ */
+
+/* Derivative of pace_surrogate_loss's loss with respect to each row's
+ * log-probability (the policy-gradient signal of the clipped objective):
+ *   dL_t/dlp_t = -A rho_t when the unclipped term is the active maximum and the
+ *                dual clip is not active; 0 when the clipped term or the dual
+ *                clip is active or lp - l^mu is clamped; scaled by 1 / sum m
+ *                (TOKEN_MEAN) or 1 / (#sequences * #tokens of the sequence);
+ * dlp device float32 [n_rows] (output; 0 outside the loss).  Arguments as for
+ * pace_surrogate_loss (loss->loss is not written). */
+PACE_API pace_status pace_surrogate_backward(const PaceBatch* batch, const float* logprob,
+                                             const PaceLossArgs* loss, float* dlp,
+                                             void* workspace, size_t workspace_bytes,
+                                             int32_t* status_dev, void* stream);
+
+PACE_API size_t pace_surrogate_backward_workspace_size(int64_t n_rows, int64_t n_seq);
+
+/* Backward of pace_token_logprob through the LM head, without materialising
+ * more than one chunk of logits: with p = softmax(z / tau), z = h W^T and
+ * g_r = dlp[r],
+ *   G_rv = (g_r / tau) (1[v = y_r] - p_rv)
+ *   grad_hidden[r] = sum_v G_rv W_v         device float32 [n_rows][H] (output)
+ *   grad_w[v]      = sum_r G_rv h_r         device float32 [V][H] (output)
+ * over the rows in the loss (rows outside it get 0).  lse is the forward's
+ * output for the same rows (device float32 [n_rows]).  Rows are processed in
+ * chunks of up to 65,536: logits are recomputed on the tensor cores, G is held
+ * in bf16 in the workspace for the chunk, then two tensor-core GEMMs form
+ * G W and G^T H.  Other arguments as for pace_token_logprob. */
+PACE_API pace_status pace_token_logprob_backward(const PaceBatch* batch, const void* hidden,
+                                                 const void* w_vocab, const int32_t* targets,
+                                                 int32_t hidden_size, int32_t vocab_size,
+                                                 float temperature, const float* lse,
+                                                 const float* dlp, float* grad_hidden,
+                                                 float* grad_w, void* workspace,
+                                                 size_t workspace_bytes, int32_t* status_dev,
+                                                 void* stream);
+
+PACE_API size_t pace_token_logprob_backward_workspace_size(int64_t n_rows, int64_t n_seq,
+                                                           int32_t hidden_size,
+                                                           int32_t vocab_size);
+
+/* ------------------------------------------------------------------------ */
 /* Profiling                                                                 */
 /* ------------------------------------------------------------------------ */
 

@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libpace.so")
-SOURCES = ["api.cu", "score.cu", "select.cu", "loss.cu", "lmhead.cu", "prefix.cu"]
+SOURCES = ["api.cu", "score.cu", "select.cu", "loss.cu", "lmhead.cu", "prefix.cu", "backward.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler",
               "-ffp-contract=off", "-Xcompiler", "-fvisibility=hidden",

@@ -1,0 +1,649 @@
+// Backward of the fused LM head and of the clipped surrogate (what the unchanged
+// policy update needs after the log-probs: gradients with respect to the hidden
+// states and the vocabulary matrix), without ever holding the logits of more
+// than one chunk of rows.
+//
+// For the rows in the loss, in chunks of up to kChunkRows compacted rows:
+//   1. gemm_kernel<EPI_G>:    z = H_c W^T recomputed on the tensor cores; the
+//                             epilogue writes G = (g / tau) (onehot(y) - softmax(z / tau))
+//                             in bf16, using the forward's log-sum-exp;
+//   2. gemm_kernel<EPI_ROWS>: dH_c = G W (A = G K-major, B = W read MN-major),
+//                             fp32 rows scattered back to their original row;
+//   3. gemm_kernel<EPI_ACC>:  dW += G^T H_c (A = G and B = H_c, both read
+//                             MN-major), fp32 accumulation in place.
+// The GEMM is one warp-specialised tcgen05 kernel: warp 0 issues TMA into a
+// 4-stage ring (128-byte swizzle), warp 1 issues tcgen05.mma (M 128, N 256,
+// K 16; the instruction descriptor's major bits select K- or MN-major operand
+// layouts), warps 2-5 drain the two TMEM accumulators.  Every wait is bounded.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include <mutex>
+
+#include "pace_internal.cuh"
+#include "pace_loss.cuh"
+
+namespace pace {
+namespace {
+
+constexpr int GBM = 128;
+constexpr int GBN = 256;
+constexpr int GBK = 64;
+constexpr int GSTAGES = 4;
+constexpr int kGemmThreads = 192;
+constexpr uint32_t kGStageA = GBM * GBK * 2;  // 16 KB
+constexpr uint32_t kGStageB = GBN * GBK * 2;  // 32 KB
+constexpr uint32_t kGStageBytes = kGStageA + kGStageB;
+constexpr uint32_t kGTmemCols = 2 * GBN;
+constexpr size_t kGSmemBytes = 1024 + GSTAGES * kGStageBytes + 256;
+constexpr int64_t kChunkRows = 65536;         // rows of G held at once (bf16 M x V)
+constexpr int kGroupM = 38;                   // M tiles per raster group
+
+enum { EPI_G = 0, EPI_ROWS = 1, EPI_ACC = 2 };
+
+struct GemmArgs {
+  int64_t M, N, K;
+  int64_t m_tiles, n_tiles;
+  int raster_n_fast;            // 1: N tile fastest; 0: groups of kGroupM M tiles, M fastest
+  // EPI_G
+  int64_t chunk_row0;           // compact row of the chunk's first row
+  const long long* n_valid;     // rows in the loss (device)
+  const int32_t* rowidx;        // compact -> original row
+  const int32_t* targets;
+  const float* lse;             // forward log-sum-exp per original row
+  const float* dlp;             // dLoss/dlp per original row
+  float scale_log2;             // log2(e) / tau
+  float inv_tau;
+  uint16_t* g_out;              // bf16 [rows of chunk][ldg]
+  int64_t ldg;
+  int32_t V;
+  // EPI_ROWS
+  float* rows_out;              // fp32 [orig rows][ldo]
+  int64_t ldo;
+  // EPI_ACC
+  float* acc_out;               // fp32 [M][ldo]
+  int32_t* status;
+};
+
+__device__ __forceinline__ void tile_of(const GemmArgs& p, int64_t bid, int64_t* m, int64_t* n) {
+  if (p.raster_n_fast) {
+    *m = bid / p.n_tiles;
+    *n = bid % p.n_tiles;
+    return;
+  }
+  const int64_t per_group = static_cast<int64_t>(kGroupM) * p.n_tiles;
+  const int64_t g = bid / per_group;
+  const int64_t r = bid % per_group;
+  const int64_t gm0 = g * kGroupM;
+  const int64_t gm = (p.m_tiles - gm0) < kGroupM ? (p.m_tiles - gm0) : kGroupM;
+  *m = gm0 + r % gm;
+  *n = r / gm;
+}
+
+// 128-byte-swizzled operand tiles.  K-major: rows of 64 K elements (128 B),
+// 8-row groups 1024 B apart; a 16-deep K step is +32 B.  MN-major: 64 MN
+// elements per 128-byte row, one row per k; boxes of 64 (MN) x 64 (K) stacked
+// along MN 8 KB apart (leading byte offset), 8-k groups 1024 B apart (stride
+// byte offset); a 16-deep K step is +2048 B.
+__device__ __forceinline__ uint64_t operand_desc(uint32_t saddr, bool mn_major) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(mn_major ? (8192u >> 4) : 1u) << 16;
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;
+  d |= static_cast<uint64_t>(1u) << 46;
+  d |= static_cast<uint64_t>(2u) << 61;
+  return d;
+}
+
+__host__ __device__ constexpr uint32_t idesc_bf16(bool a_mn, bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) |
+         ((b_mn ? 1u : 0u) << 16) | ((static_cast<uint32_t>(GBN) >> 3) << 17) |
+         ((static_cast<uint32_t>(GBM) >> 4) << 24);
+}
+
+__device__ __forceinline__ uint16_t f32_to_bf16_rn(float x) {
+  uint32_t u = __float_as_uint(x);
+  if ((u & 0x7fffffffu) > 0x7f800000u) return static_cast<uint16_t>((u >> 16) | 0x40u);  // NaN
+  u += 0x7fffu + ((u >> 16) & 1u);
+  return static_cast<uint16_t>(u >> 16);
+}
+
+template <bool A_MN, bool B_MN, int EPI>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
+                GemmArgs p) {
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + GSTAGES * kGStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + GSTAGES;
+  uint64_t* tmem_full = bars + 2 * GSTAGES;
+  uint64_t* tmem_empty = tmem_full + 2;
+  uint64_t* mma_done = tmem_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t n_tiles_total = p.m_tiles * p.n_tiles;
+  const int nkb = static_cast<int>((p.K + GBK - 1) / GBK);
+  if (nkb == 0) return;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < GSTAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tmem_full[b], 1);
+      mbar_init(&tmem_empty[b], 4 * 32);
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kGTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  constexpr uint32_t kIdesc = idesc_bf16(A_MN, B_MN);
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_a);
+      tma_prefetch_desc(&tm_b);
+      uint64_t pol;
+      asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
+      uint32_t it = 0;
+      bool ok = true;
+      for (int64_t t = blockIdx.x; t < n_tiles_total && ok; t += gridDim.x) {
+        int64_t mt, nt;
+        tile_of(p, t, &mt, &nt);
+        const int32_t m0 = static_cast<int32_t>(mt * GBM), n0 = static_cast<int32_t>(nt * GBN);
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const uint32_t s = it % GSTAGES, ph = (it / GSTAGES) & 1u;
+          if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
+            ok = false;
+            break;
+          }
+          unsigned char* sa = smem + s * kGStageBytes;
+          unsigned char* sb = sa + kGStageA;
+          mbar_arrive_expect_tx(&full[s], kGStageBytes);
+          const int32_t k0 = kb * GBK;
+          if (A_MN) {  // box {64 MN, 64 K}: two along M
+            tma_load_2d(sa, &tm_a, &full[s], m0, k0, pol);
+            tma_load_2d(sa + 8192, &tm_a, &full[s], m0 + 64, k0, pol);
+          } else {     // box {64 K, 128 rows}
+            tma_load_2d(sa, &tm_a, &full[s], k0, m0, pol);
+          }
+          if (B_MN) {  // four along N
+#pragma unroll
+            for (int q = 0; q < 4; ++q) tma_load_2d(sb + q * 8192, &tm_b, &full[s], n0 + 64 * q, k0, pol);
+          } else {     // box {64 K, 256 rows}
+            tma_load_2d(sb, &tm_b, &full[s], k0, n0, pol);
+          }
+        }
+      }
+      if (!ok) {
+        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+        *abort_flag = 1;
+      }
+      for (uint32_t s = 0; s < GSTAGES && s < it; ++s) {
+        const uint32_t last = it - 1 - ((it - 1 - s) % GSTAGES);
+        mbar_wait_bounded(&full[s], (last / GSTAGES) & 1u, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      uint32_t it = 0, tc = 0;
+      bool ok = true;
+      for (int64_t t = blockIdx.x; t < n_tiles_total && ok; t += gridDim.x, ++tc) {
+        const uint32_t acc = tc & 1u, acc_ph = (tc >> 1) & 1u;
+        if (!mbar_wait_bounded(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * GBN;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const uint32_t s = it % GSTAGES, ph = (it / GSTAGES) & 1u;
+          if (!mbar_wait_bounded(&full[s], ph, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + s * kGStageBytes);
+          const uint32_t sb = sa + kGStageA;
+#pragma unroll
+          for (int k = 0; k < GBK / 16; ++k) {
+            const uint32_t ka = A_MN ? sa + k * 2048 : sa + k * 32;
+            const uint32_t kbb = B_MN ? sb + k * 2048 : sb + k * 32;
+            tc_mma_f16(d_tmem, operand_desc(ka, A_MN), operand_desc(kbb, B_MN), kIdesc,
+                       (kb > 0 || k > 0) ? 1u : 0u);
+          }
+          tc_commit(&empty[s]);
+        }
+        if (!ok) break;
+        tc_commit(&tmem_full[acc]);
+      }
+      if (!ok) {
+        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+        *abort_flag = 1;
+      }
+      tc_commit(mma_done);
+      mbar_wait_bounded(mma_done, 0, nullptr);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int r_local = quad * 32 + lane;
+    uint32_t tc = 0;
+    for (int64_t t = blockIdx.x; t < n_tiles_total; t += gridDim.x, ++tc) {
+      int64_t mt, nt;
+      tile_of(p, t, &mt, &nt);
+      const uint32_t acc = tc & 1u, acc_ph = (tc >> 1) & 1u;
+      if (!mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag)) {
+        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+        *abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const int64_t row = mt * GBM + r_local;  // row of C
+      const int64_t n0 = nt * GBN;
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * GBN;
+      // per-row context
+      bool row_ok = row < p.M;
+      int32_t y = -1;
+      float gscale = 0.0f, lse2 = 0.0f;
+      int64_t orig = -1;
+      if (EPI == EPI_G || EPI == EPI_ROWS) {
+        const int64_t crow = p.chunk_row0 + row;
+        const bool in_loss = row_ok && crow < static_cast<int64_t>(*p.n_valid);
+        if (in_loss) orig = p.rowidx[crow];
+        if (EPI == EPI_G && in_loss) {
+          y = p.targets[orig];
+          gscale = p.dlp[orig] * p.inv_tau;
+          lse2 = p.lse[orig] * 1.4426950408889634f;
+        }
+        if (EPI == EPI_ROWS) row_ok = in_loss;
+      }
+#pragma unroll 1
+      for (int c = 0; c < GBN; c += 32) {
+        float v[32];
+        tmem_ld_32x32b_x32(tbase + c, v);
+        tmem_wait_ld();
+        const int64_t col0 = n0 + c;
+        if (EPI == EPI_G) {
+          if (row_ok && col0 < p.V) {
+            // G = (g / tau) (onehot - p), zero for rows outside the loss
+            uint32_t packed[16];
+#pragma unroll
+            for (int i = 0; i < 32; i += 2) {
+              float g0 = 0.0f, g1 = 0.0f;
+              if (gscale != 0.0f) {
+                const float p0 = ex2_approx(fmaf(v[i], p.scale_log2, -lse2));
+                const float p1 = ex2_approx(fmaf(v[i + 1], p.scale_log2, -lse2));
+                g0 = col0 + i < p.V ? gscale * ((col0 + i == y ? 1.0f : 0.0f) - p0) : 0.0f;
+                g1 = col0 + i + 1 < p.V ? gscale * ((col0 + i + 1 == y ? 1.0f : 0.0f) - p1) : 0.0f;
+              }
+              packed[i / 2] = static_cast<uint32_t>(f32_to_bf16_rn(g0)) |
+                              (static_cast<uint32_t>(f32_to_bf16_rn(g1)) << 16);
+            }
+            uint16_t* dst = p.g_out + row * p.ldg + col0;
+            if (col0 + 32 <= p.ldg) {
+              uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                d4[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2],
+                                   packed[4 * q + 3]);
+            } else {
+              for (int i = 0; i < 32 && col0 + i < p.ldg; ++i)
+                dst[i] = static_cast<uint16_t>(packed[i / 2] >> (16 * (i & 1)));
+            }
+          }
+        } else if (EPI == EPI_ROWS) {
+          if (row_ok) {
+            float* dst = p.rows_out + orig * p.ldo + col0;
+            if (col0 + 32 <= p.N) {
+              float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+              for (int q = 0; q < 8; ++q)
+                d4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            } else {
+              for (int i = 0; i < 32 && col0 + i < p.N; ++i) dst[i] = v[i];
+            }
+          }
+        } else {
+          if (row_ok) {
+            float* dst = p.acc_out + row * p.ldo + col0;
+            if (col0 + 32 <= p.N) {
+              float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+              for (int q = 0; q < 8; ++q) {
+                float4 o = d4[q];
+                o.x += v[4 * q];
+                o.y += v[4 * q + 1];
+                o.z += v[4 * q + 2];
+                o.w += v[4 * q + 3];
+                d4[q] = o;
+              }
+            } else {
+              for (int i = 0; i < 32 && col0 + i < p.N; ++i) dst[i] += v[i];
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&tmem_empty[acc]);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, kGTmemCols);
+}
+
+// Zero the gathered rows [n_valid, rows_end) of the compact buffer so that
+// rows outside the loss contribute exactly 0 to dW (0 x garbage could be NaN).
+__global__ void zero_tail_rows_kernel(uint4* __restrict__ buf, int64_t row_vecs,
+                                      const long long* __restrict__ n_valid, int64_t rows_end) {
+  const int64_t start = *n_valid;
+  const int64_t total = (rows_end - start) * row_vecs;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    buf[start * row_vecs + i] = make_uint4(0, 0, 0, 0);
+}
+
+// dLoss/dlp per row of the clipped surrogate (oracle: oracle_surrogate_grad).
+__global__ void surrogate_grad_kernel(const int64_t* __restrict__ seq_offsets,
+                                      const uint8_t* __restrict__ seq_accepted,
+                                      const uint8_t* __restrict__ mask,
+                                      const float* __restrict__ logprob,
+                                      const float* __restrict__ behav,
+                                      const float* __restrict__ adv,
+                                      const long long* __restrict__ seq_in,
+                                      const long long* __restrict__ total, int64_t n_seq,
+                                      int64_t n_rows, float eps_low, float eps_high, float dual,
+                                      int agg, const int* __restrict__ n_seq_used,
+                                      float* __restrict__ dlp) {
+  for (int64_t i = blockIdx.x; i < n_seq; i += gridDim.x) {
+    const int64_t r0 = seq_offsets[i], r1 = seq_offsets[i + 1];
+    if (r1 < r0 || r0 < 0 || r1 > n_rows) continue;
+    const bool acc = seq_accepted ? seq_accepted[i] != 0 : true;
+    const float a = adv[i];
+    const double scale = agg == PACE_AGG_TOKEN_MEAN
+                             ? 1.0 / static_cast<double>(*total)
+                             : 1.0 / (static_cast<double>(*n_seq_used) *
+                                      static_cast<double>(seq_in[i]));
+    for (int64_t r = r0 + threadIdx.x; r < r1; r += blockDim.x) {
+      const bool in = acc && (mask ? mask[r] != 0 : true);
+      float g = 0.0f;
+      if (in) {
+        const float d = logprob[r] - behav[r];
+        const float dc = fminf(fmaxf(d, -20.0f), 20.0f);
+        const float rho = expf(dc);
+        const float rc = fminf(fmaxf(rho, 1.0f - eps_low), 1.0f + eps_high);
+        const float p1 = -a * rho, p2 = -a * rc;
+        const float l = fmaxf(p1, p2);
+        if (d > -20.0f && d < 20.0f && p1 >= p2) g = -a * rho;
+        if (a < 0.0f && -dual * a < l) g = 0.0f;
+        g = static_cast<float>(static_cast<double>(g) * scale);
+      }
+      dlp[r] = g;
+    }
+  }
+}
+
+__global__ void count_used_seqs_kernel(const long long* __restrict__ seq_in, int64_t n_seq,
+                                       int* __restrict__ out) {
+  __shared__ int sh[256];
+  int c = 0;
+  for (int64_t i = threadIdx.x; i < n_seq; i += blockDim.x) c += seq_in[i] > 0;
+  sh[threadIdx.x] = c;
+  __syncthreads();
+  for (int o = 128; o > 0; o >>= 1) {
+    if (threadIdx.x < o) sh[threadIdx.x] += sh[threadIdx.x + o];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *out = sh[0];
+}
+
+// ---------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+// bf16 matrix [rows][cols] with row stride ld elements; box {box_inner, box_outer}.
+pace_status encode_2d(CUtensorMap* tm, const void* ptr, int64_t rows, int64_t cols, int64_t ld,
+                      int box_inner, int box_outer) {
+  auto enc = encode_fn();
+  if (!enc) return PACE_ERR_CUDA;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_outer)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? PACE_OK : PACE_ERR_UNSUPPORTED_SHAPE;
+}
+
+template <bool A_MN, bool B_MN, int EPI>
+pace_status launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmArgs a,
+                        cudaStream_t st) {
+  static int done_dev = -1;
+  static std::mutex mu;
+  int dev = 0;
+  PACE_TRY_CUDA(cudaGetDevice(&dev));
+  {
+    std::lock_guard<std::mutex> g(mu);
+    if (done_dev != dev) {
+      PACE_TRY_CUDA(cudaFuncSetAttribute(gemm_kernel<A_MN, B_MN, EPI>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(kGSmemBytes)));
+      done_dev = dev;
+    }
+  }
+  a.m_tiles = (a.M + GBM - 1) / GBM;
+  a.n_tiles = (a.N + GBN - 1) / GBN;
+  const int64_t tiles = a.m_tiles * a.n_tiles;
+  if (tiles == 0) return PACE_OK;
+  int64_t grid = tiles < static_cast<int64_t>(sm_count()) ? tiles : sm_count();
+  gemm_kernel<A_MN, B_MN, EPI><<<static_cast<unsigned>(grid), kGemmThreads, kGSmemBytes, st>>>(
+      ta, tb, a);
+  return last_launch_status();
+}
+
+struct BwWs {
+  LmWs lm;            // compaction + gathered rows (hidden_c)
+  uint16_t* g;        // bf16 [chunk][ldg]
+  int* n_seq_used;
+};
+
+int64_t chunk_rows(int64_t n_rows) {
+  int64_t c = n_rows < kChunkRows ? n_rows : kChunkRows;
+  return (c + GBM - 1) / GBM * GBM;
+}
+
+void carve_bw_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, BwWs* w) {
+  carve_lm_ws(cv, n_rows, n_seq, H, V, true, &w->lm);
+  const int64_t ldg = (static_cast<int64_t>(V) + 7) / 8 * 8;
+  w->g = cv.take<uint16_t>(static_cast<size_t>(chunk_rows(n_rows > 0 ? n_rows : 1)) * ldg);
+  w->n_seq_used = cv.take<int>(1);
+}
+
+}  // namespace
+}  // namespace pace
+
+using namespace pace;
+
+extern "C" size_t pace_surrogate_backward_workspace_size(int64_t n_rows, int64_t n_seq) {
+  Carver cv;
+  CompactWs cw;
+  SurrogateWs sw;
+  carve_compact_ws(cv, n_seq, n_rows, &cw);
+  carve_surrogate_ws(cv, n_seq, &sw);
+  cv.take<int>(1);
+  return cv.used;
+}
+
+extern "C" pace_status pace_surrogate_backward(const PaceBatch* batch, const float* logprob,
+                                               const PaceLossArgs* loss, float* dlp,
+                                               void* workspace, size_t workspace_bytes,
+                                               int32_t* status_dev, void* stream) {
+  PACE_TRY(check_batch(batch));
+  PACE_TRY(check_loss_args(batch, loss));
+  if (batch->n_rows > 0 && (!logprob || !dlp)) return PACE_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
+  Carver cv(workspace, workspace_bytes);
+  CompactWs cw;
+  SurrogateWs sw;
+  carve_compact_ws(cv, batch->n_seq, batch->n_rows, &cw);
+  carve_surrogate_ws(cv, batch->n_seq, &sw);
+  int* n_used = cv.take<int>(1);
+  if (!cv.fits()) return PACE_ERR_WORKSPACE;
+  cudaStream_t st = as_stream(stream);
+  if (batch->n_rows > 0)
+    PACE_TRY_CUDA(cudaMemsetAsync(dlp, 0, static_cast<size_t>(batch->n_rows) * 4, st));
+  if (batch->n_seq == 0) return PACE_OK;
+  float* adv = loss->adv ? loss->adv : sw.adv;
+  PACE_TRY(launch_group_adv(loss->reward, batch->seq_accepted, batch->n_seq,
+                                   loss->group_size, loss->params.adv_eps,
+                                   loss->params.std_unbiased, adv, st));
+  PACE_TRY(run_compaction(batch, cw, status_dev, st));  // rows in the loss per sequence
+  count_used_seqs_kernel<<<1, 256, 0, st>>>(cw.seq_in, batch->n_seq, n_used);
+  PACE_TRY(last_launch_status());
+  int64_t grid = batch->n_seq;
+  const int64_t cap = static_cast<int64_t>(sm_count()) * 8;
+  if (grid > cap) grid = cap;
+  surrogate_grad_kernel<<<static_cast<unsigned>(grid), 256, 0, st>>>(
+      batch->seq_offsets, batch->seq_accepted, batch->mask, logprob, loss->behav_lp, adv,
+      cw.seq_in, cw.total, batch->n_seq, batch->n_rows, loss->params.eps_low,
+      loss->params.eps_high, loss->params.dual_clip, loss->params.agg, n_used, dlp);
+  return last_launch_status();
+}
+
+extern "C" size_t pace_token_logprob_backward_workspace_size(int64_t n_rows, int64_t n_seq,
+                                                             int32_t hidden_size,
+                                                             int32_t vocab_size) {
+  if (n_rows < 0 || n_seq < 0 || hidden_size <= 0 || vocab_size <= 0) return 0;
+  Carver cv;
+  BwWs w;
+  carve_bw_ws(cv, n_rows, n_seq, hidden_size, vocab_size, &w);
+  return cv.used;
+}
+
+extern "C" pace_status pace_token_logprob_backward(
+    const PaceBatch* batch, const void* hidden, const void* w_vocab, const int32_t* targets,
+    int32_t hidden_size, int32_t vocab_size, float temperature, const float* lse,
+    const float* dlp, float* grad_hidden, float* grad_w, void* workspace,
+    size_t workspace_bytes, int32_t* status_dev, void* stream) {
+  const int H = hidden_size, V = vocab_size;
+  PACE_TRY(check_lm_args(batch, hidden, w_vocab, targets, H, V, temperature, dlp));
+  if (batch->n_rows > 0 && (!lse || !grad_hidden || !grad_w)) return PACE_ERR_INVALID_ARG;
+  if (!aligned(grad_hidden, 16) || !aligned(grad_w, 16)) return PACE_ERR_UNSUPPORTED_SHAPE;
+  if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
+  Carver cv(workspace, workspace_bytes);
+  BwWs ws;
+  carve_bw_ws(cv, batch->n_rows, batch->n_seq, H, V, &ws);
+  if (!cv.fits()) return PACE_ERR_WORKSPACE;
+  cudaStream_t st = as_stream(stream);
+  const int64_t n_rows = batch->n_rows;
+  PACE_TRY_CUDA(cudaMemsetAsync(grad_w, 0, static_cast<size_t>(V) * H * 4, st));
+  if (n_rows == 0) return PACE_OK;
+  PACE_TRY_CUDA(cudaMemsetAsync(grad_hidden, 0, static_cast<size_t>(n_rows) * H * 4, st));
+  // the rows in the loss, gathered densely (always compacted here)
+  PACE_TRY(run_compaction(batch, ws.lm.cw, status_dev, st));
+  PACE_TRY(run_gather(hidden, H, n_rows, ws.lm.cw, ws.lm.hidden_c, st));
+  const int64_t rows_cap = n_rows > 128 ? n_rows : 128;
+  const int64_t row_vecs = static_cast<int64_t>(H) * 2 / 16;
+  zero_tail_rows_kernel<<<static_cast<unsigned>(sm_count() * 4), 256, 0, st>>>(
+      static_cast<uint4*>(ws.lm.hidden_c), row_vecs, ws.lm.cw.total, rows_cap);
+  PACE_TRY(last_launch_status());
+  const int64_t chunk = chunk_rows(n_rows);
+  const int64_t ldg = (static_cast<int64_t>(V) + 7) / 8 * 8;
+  for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
+    const int64_t rows_c = (n_rows - c0) < chunk ? (n_rows - c0) : chunk;
+    const int64_t rows_c_pad = (rows_c + GBM - 1) / GBM * GBM;
+    const void* hc = static_cast<const uint16_t*>(ws.lm.hidden_c) + c0 * H;
+    // rows of the gathered buffer from c0 on (the padded tail of a chunk past the
+    // buffer is read as zeros by TMA)
+    const int64_t hc_rows = (rows_cap - c0) < rows_c_pad ? (rows_cap - c0) : rows_c_pad;
+    // 1. G = (g / tau) (onehot - softmax) for the chunk's rows (bf16)
+    {
+      CUtensorMap ta, tb;
+      PACE_TRY(encode_2d(&ta, hc, hc_rows, H, H, 64, GBM));
+      PACE_TRY(encode_2d(&tb, w_vocab, V, H, H, 64, GBN));
+      GemmArgs a = {};
+      a.M = rows_c_pad;
+      a.N = V;
+      a.K = H;
+      a.raster_n_fast = 0;
+      a.chunk_row0 = c0;
+      a.n_valid = ws.lm.cw.total;
+      a.rowidx = ws.lm.cw.rowidx;
+      a.targets = targets;
+      a.lse = lse;
+      a.dlp = dlp;
+      a.scale_log2 = 1.4426950408889634f / temperature;
+      a.inv_tau = 1.0f / temperature;
+      a.g_out = ws.g;
+      a.ldg = ldg;
+      a.V = V;
+      a.status = status_dev;
+      PACE_TRY((launch_gemm<false, false, EPI_G>(ta, tb, a, st)));
+    }
+    // 2. dH rows = G W   (W read MN-major: [K = V][N = H])
+    {
+      CUtensorMap ta, tb;
+      PACE_TRY(encode_2d(&ta, ws.g, rows_c_pad, V, ldg, 64, GBM));
+      PACE_TRY(encode_2d(&tb, w_vocab, V, H, H, 64, 64));
+      GemmArgs a = {};
+      a.M = rows_c_pad;
+      a.N = H;
+      a.K = V;
+      a.raster_n_fast = 1;
+      a.chunk_row0 = c0;
+      a.n_valid = ws.lm.cw.total;
+      a.rowidx = ws.lm.cw.rowidx;
+      a.rows_out = grad_hidden;
+      a.ldo = H;
+      a.status = status_dev;
+      PACE_TRY((launch_gemm<false, true, EPI_ROWS>(ta, tb, a, st)));
+    }
+    // 3. dW += G^T H_c   (G read MN-major: [K = rows][M = V]; H_c MN-major: [K = rows][N = H])
+    {
+      CUtensorMap ta, tb;
+      PACE_TRY(encode_2d(&ta, ws.g, rows_c_pad, V, ldg, 64, 64));
+      PACE_TRY(encode_2d(&tb, hc, hc_rows, H, H, 64, 64));
+      GemmArgs a = {};
+      a.M = V;
+      a.N = H;
+      a.K = rows_c_pad;
+      a.raster_n_fast = 1;
+      a.acc_out = grad_w;
+      a.ldo = H;
+      a.status = status_dev;
+      PACE_TRY((launch_gemm<true, true, EPI_ACC>(ta, tb, a, st)));
+    }
+  }
+  return PACE_OK;
+}

@@ -90,6 +90,11 @@ SIGNATURES = {
     "pace_stale_k_workspace_size": ([_I64], _SZ),
     "pace_staleness_histogram": ([_P, _P, _I64, _F64, _F64, _I32, _P, _P, _P], _I32),
     "pace_quantile_admit": ([_P, _I64, _F64, _I64, _I32, _P, _I64, _P, _P, _P, _P, _P], _I32),
+    "pace_surrogate_backward": ([_P, _P, _P, _P, _P, _SZ, _P, _P], _I32),
+    "pace_surrogate_backward_workspace_size": ([_I64, _I64], _SZ),
+    "pace_token_logprob_backward": ([_P, _P, _P, _P, _I32, _I32, _F32, _P, _P, _P, _P, _P, _SZ,
+                                     _P, _P], _I32),
+    "pace_token_logprob_backward_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
     "pace_set_profile_events": ([_I32, _P, _P], _I32),
     "pace_kernel_launches": ([], ctypes.c_uint64),
 }
@@ -411,3 +416,42 @@ def quantile_admit(unit_score, r_hat, batch_units, window: ScoreWindow, min_obs=
                                    _ptr(status), _stream(stream))
     _check(st, "pace_quantile_admit")
     return decision[:n], kappa
+
+
+def surrogate_backward(batch: PaceBatch, logprob, loss: PaceLossArgs, dlp=None, ws=None,
+                       status=None, stream=None):
+    """pace_surrogate_backward: float32 dLoss/dlp per row."""
+    dev = logprob.device
+    if dlp is None:
+        dlp = torch.empty(batch.n_rows, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(lib().pace_surrogate_backward_workspace_size(batch.n_rows, batch.n_seq),
+                       dev)
+    st = lib().pace_surrogate_backward(ctypes.byref(batch), _ptr(_dev(logprob)),
+                                       ctypes.byref(loss), _ptr(dlp), _ptr(ws), ws.numel(),
+                                       _ptr(status), _stream(stream))
+    _check(st, "pace_surrogate_backward")
+    return dlp
+
+
+def token_logprob_backward(batch: PaceBatch, hidden, w_vocab, targets, lse, dlp,
+                           temperature=1.0, grad_hidden=None, grad_w=None, ws=None, status=None,
+                           stream=None):
+    """pace_token_logprob_backward: (grad_hidden fp32 [n_rows, H], grad_w fp32 [V, H])."""
+    n_rows, H = hidden.shape
+    V = w_vocab.shape[0]
+    dev = hidden.device
+    if grad_hidden is None:
+        grad_hidden = torch.empty(n_rows, H, dtype=torch.float32, device=dev)
+    if grad_w is None:
+        grad_w = torch.empty(V, H, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(lib().pace_token_logprob_backward_workspace_size(n_rows, batch.n_seq, H,
+                                                                        V), dev)
+    st = lib().pace_token_logprob_backward(ctypes.byref(batch), _ptr(_dev(hidden)),
+                                           _ptr(_dev(w_vocab)), _ptr(_dev(targets)), int(H),
+                                           int(V), float(temperature), _ptr(_dev(lse)),
+                                           _ptr(_dev(dlp)), _ptr(grad_hidden), _ptr(grad_w),
+                                           _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    _check(st, "pace_token_logprob_backward")
+    return grad_hidden, grad_w
