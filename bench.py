@@ -571,6 +571,39 @@ def run_case(args):
         tf = 2.0 * rows * H * V / (ms / 1e3) / 1e12
         print(json.dumps({"case": "lmhead", "rows": rows, "H": H, "V": V, "kernel_ms": ms,
                           "tflops": tf, "frac_burst": tf / peaks["bf16_tflops"]}), flush=True)
+    elif args.case == "lmhead_bwd":
+        spec = workloads.SPECS[WORKLOAD]
+        H, V, rows = spec.hidden, spec.vocab, args.case_rows
+        hidden = workloads.bf16_normal_device((rows, H), 1.0, 101, device)
+        w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), 102, device)
+        gen = torch.Generator(device=device)
+        gen.manual_seed(103)
+        targets = torch.randint(0, V, (rows,), generator=gen, device=device, dtype=torch.int32)
+        dlp = torch.randn(rows, generator=gen, device=device) * 1e-6
+        b = pace.make_batch(torch.tensor([0, rows], dtype=torch.int64, device=device), rows)
+        lp = torch.empty(rows, dtype=torch.float32, device=device)
+        lse = torch.empty(rows, dtype=torch.float32, device=device)
+        status = pace.new_status(device)
+        pace.token_logprob(b, hidden, w, targets, 1.0, logprob=lp, lse=lse, status=status)
+        gh = torch.empty(rows, H, dtype=torch.float32, device=device)
+        gw = torch.empty(V, H, dtype=torch.float32, device=device)
+        ws = pace.workspace(pace.lib().pace_token_logprob_backward_workspace_size(rows, 1, H, V),
+                            device)
+        for i in range(args.warmup + args.steps):
+            if i == args.warmup:
+                torch.cuda.synchronize()
+                t0 = torch.cuda.Event(enable_timing=True)
+                t1 = torch.cuda.Event(enable_timing=True)
+                t0.record()
+            pace.token_logprob_backward(b, hidden, w, targets, lse, dlp, grad_hidden=gh,
+                                        grad_w=gw, ws=ws, status=status)
+        t1.record()
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0
+        ms = t0.elapsed_time(t1) / args.steps
+        tf = 3 * 2.0 * rows * H * V / (ms / 1e3) / 1e12
+        print(json.dumps({"case": "lmhead_bwd", "rows": rows, "H": H, "V": V, "ms": ms,
+                          "tflops": tf}), flush=True)
     else:
         pool = workloads.make_pool("sweep", n_traj=args.case_traj, device=device)
         n = pool.n_traj
@@ -603,7 +636,7 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=64)
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", choices=["lmhead", "tagreduce"], default=None,
+    ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce"], default=None,
                     help="time one kernel on a small case (profiler captures)")
     ap.add_argument("--case-rows", type=int, default=4864)
     ap.add_argument("--case-traj", type=int, default=16384)

@@ -68,18 +68,24 @@ struct GemmArgs {
   int32_t* status;
 };
 
-__device__ __forceinline__ void tile_of(const GemmArgs& p, int64_t bid, int64_t* m, int64_t* n) {
+// Work items are (pair of M tiles, N tile); the two CTAs of a cluster take the
+// two M tiles of a pair and share every B tile, each loading half of it and
+// multicasting it to both.
+__device__ __forceinline__ void item_of(const GemmArgs& p, int64_t item, int64_t* mp,
+                                        int64_t* n) {
+  const int64_t pairs = (p.m_tiles + 1) / 2;
   if (p.raster_n_fast) {
-    *m = bid / p.n_tiles;
-    *n = bid % p.n_tiles;
+    *mp = item / p.n_tiles;
+    *n = item % p.n_tiles;
     return;
   }
-  const int64_t per_group = static_cast<int64_t>(kGroupM) * p.n_tiles;
-  const int64_t g = bid / per_group;
-  const int64_t r = bid % per_group;
-  const int64_t gm0 = g * kGroupM;
-  const int64_t gm = (p.m_tiles - gm0) < kGroupM ? (p.m_tiles - gm0) : kGroupM;
-  *m = gm0 + r % gm;
+  const int64_t gp = kGroupM / 2;  // pairs per raster group
+  const int64_t per_group = gp * p.n_tiles;
+  const int64_t g = item / per_group;
+  const int64_t r = item % per_group;
+  const int64_t g0 = g * gp;
+  const int64_t gm = (pairs - g0) < gp ? (pairs - g0) : gp;
+  *mp = g0 + r % gm;
   *n = r / gm;
 }
 
@@ -112,7 +118,7 @@ __device__ __forceinline__ uint16_t f32_to_bf16_rn(float x) {
 }
 
 template <bool A_MN, bool B_MN, int EPI>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                 GemmArgs p) {
   extern __shared__ unsigned char smem_raw[];
@@ -128,14 +134,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t n_tiles_total = p.m_tiles * p.n_tiles;
+  const uint32_t crank = cluster_ctarank();
+  const int64_t n_items = (p.m_tiles + 1) / 2 * p.n_tiles;
+  const int64_t cid = blockIdx.x / 2, n_clusters = gridDim.x / 2;
   const int nkb = static_cast<int>((p.K + GBK - 1) / GBK);
-  if (nkb == 0) return;
+  if (nkb == 0) return;  // uniform over the grid
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < GSTAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], 2);  // both CTAs' MMAs (each stage holds the peer's half of B)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tmem_full[b], 1);
@@ -150,10 +158,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tmem_relinquish();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   constexpr uint32_t kIdesc = idesc_bf16(A_MN, B_MN);
+  constexpr uint16_t kPair = 0x3;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -163,10 +172,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
       uint32_t it = 0;
       bool ok = true;
-      for (int64_t t = blockIdx.x; t < n_tiles_total && ok; t += gridDim.x) {
-        int64_t mt, nt;
-        tile_of(p, t, &mt, &nt);
-        const int32_t m0 = static_cast<int32_t>(mt * GBM), n0 = static_cast<int32_t>(nt * GBN);
+      for (int64_t t = cid; t < n_items && ok; t += n_clusters) {
+        int64_t mp, nt;
+        item_of(p, t, &mp, &nt);
+        const int32_t m0 = static_cast<int32_t>((2 * mp + crank) * GBM);
+        const int32_t n0 = static_cast<int32_t>(nt * GBN);
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const uint32_t s = it % GSTAGES, ph = (it / GSTAGES) & 1u;
           if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
@@ -183,11 +193,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           } else {     // box {64 K, 128 rows}
             tma_load_2d(sa, &tm_a, &full[s], k0, m0, pol);
           }
-          if (B_MN) {  // four along N
+          // this CTA's half of B, multicast into both CTAs of the pair
+          if (B_MN) {  // four {64 N, 64 K} boxes along N; this CTA loads two
 #pragma unroll
-            for (int q = 0; q < 4; ++q) tma_load_2d(sb + q * 8192, &tm_b, &full[s], n0 + 64 * q, k0, pol);
-          } else {     // box {64 K, 256 rows}
-            tma_load_2d(sb, &tm_b, &full[s], k0, n0, pol);
+            for (int q = 2 * static_cast<int>(crank); q < 2 * static_cast<int>(crank) + 2; ++q)
+              tma_load_2d_multicast(sb + q * 8192, &tm_b, &full[s], n0 + 64 * q, k0, kPair, pol);
+          } else {     // {64 K, 128 rows}, one half of the 256 rows
+            tma_load_2d_multicast(sb + crank * (kGStageB / 2), &tm_b, &full[s], k0,
+                                  n0 + static_cast<int32_t>(crank) * (GBN / 2), kPair, pol);
           }
         }
       }
@@ -204,7 +217,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (lane == 0) {
       uint32_t it = 0, tc = 0;
       bool ok = true;
-      for (int64_t t = blockIdx.x; t < n_tiles_total && ok; t += gridDim.x, ++tc) {
+      for (int64_t t = cid; t < n_items && ok; t += n_clusters, ++tc) {
         const uint32_t acc = tc & 1u, acc_ph = (tc >> 1) & 1u;
         if (!mbar_wait_bounded(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
           ok = false;
@@ -228,7 +241,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             tc_mma_f16(d_tmem, operand_desc(ka, A_MN), operand_desc(kbb, B_MN), kIdesc,
                        (kb > 0 || k > 0) ? 1u : 0u);
           }
-          tc_commit(&empty[s]);
+          tc_commit_multicast(&empty[s], kPair);
         }
         if (!ok) break;
         tc_commit(&tmem_full[acc]);
@@ -244,9 +257,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int quad = warp & 3;
     const int r_local = quad * 32 + lane;
     uint32_t tc = 0;
-    for (int64_t t = blockIdx.x; t < n_tiles_total; t += gridDim.x, ++tc) {
-      int64_t mt, nt;
-      tile_of(p, t, &mt, &nt);
+    for (int64_t t = cid; t < n_items; t += n_clusters, ++tc) {
+      int64_t mp, nt;
+      item_of(p, t, &mp, &nt);
+      const int64_t mt = 2 * mp + crank;
       const uint32_t acc = tc & 1u, acc_ph = (tc >> 1) & 1u;
       if (!mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag)) {
         if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
@@ -346,6 +360,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // the peer may still multicast into this CTA until it is done too
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem_base, kGTmemCols);
 }
@@ -464,9 +479,10 @@ pace_status launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmArgs a
   }
   a.m_tiles = (a.M + GBM - 1) / GBM;
   a.n_tiles = (a.N + GBN - 1) / GBN;
-  const int64_t tiles = a.m_tiles * a.n_tiles;
-  if (tiles == 0) return PACE_OK;
-  int64_t grid = tiles < static_cast<int64_t>(sm_count()) ? tiles : sm_count();
+  const int64_t items = (a.m_tiles + 1) / 2 * a.n_tiles;
+  if (items == 0) return PACE_OK;
+  const int64_t max_clusters = sm_count() / 2;
+  const int64_t grid = 2 * (items < max_clusters ? items : max_clusters);
   gemm_kernel<A_MN, B_MN, EPI><<<static_cast<unsigned>(grid), kGemmThreads, kGSmemBytes, st>>>(
       ta, tb, a);
   return last_launch_status();
@@ -591,7 +607,7 @@ extern "C" pace_status pace_token_logprob_backward(
     {
       CUtensorMap ta, tb;
       PACE_TRY(encode_2d(&ta, hc, hc_rows, H, H, 64, GBM));
-      PACE_TRY(encode_2d(&tb, w_vocab, V, H, H, 64, GBN));
+      PACE_TRY(encode_2d(&tb, w_vocab, V, H, H, 64, GBN / 2));
       GemmArgs a = {};
       a.M = rows_c_pad;
       a.N = V;
