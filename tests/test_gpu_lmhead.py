@@ -177,3 +177,32 @@ def test_full_size_heads_sampled_rows(name):
     assert st == 0
     err = np.abs(lp[sample] - olp)
     assert err.max() <= TOL, err.max()
+
+
+@pytest.mark.parametrize("case", ["no_rows", "all_masked", "none_accepted", "one_row"])
+def test_degenerate_batches(case):
+    H, V = 128, 640
+    rng = np.random.default_rng(13)
+    rows = {"no_rows": 0, "all_masked": 300, "none_accepted": 300, "one_row": 1}[case]
+    hb = workloads.bf16_normal_host((max(rows, 1), H), 1.0, 5)[:rows]
+    wb = workloads.bf16_normal_host((V, H), 0.1, 6)
+    y = rng.integers(0, V, size=rows).astype(np.int32)
+    so = np.array([0, rows // 2, rows], np.int64)
+    mask = np.zeros(rows, np.uint8) if case == "all_masked" else np.ones(rows, np.uint8)
+    acc = np.zeros(2, np.uint8) if case == "none_accepted" else np.ones(2, np.uint8)
+    hidden = bf16_dev(hb) if rows else torch.empty(0, H, dtype=torch.bfloat16, device=DEV)
+    b = pace.make_batch(to_dev(so), rows, seq_accepted=to_dev(acc), mask=to_dev(mask))
+    loss = torch.full((1,), 5.0, dtype=torch.float64, device=DEV)
+    la = pace.make_loss_args(to_dev(np.zeros(max(rows, 1), np.float32)),
+                             to_dev(np.ones(2, np.float32)), 2, pace.loss_params(), loss)
+    status = pace.new_status(DEV)
+    lp = pace.token_logprob(b, hidden, bf16_dev(wb), to_dev(y), 1.0, loss=la, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    lp = as_np(lp)
+    if case == "one_row":
+        st, olp, _ = oracle.token_logprob(hb, wb, y)
+        assert abs(lp[0] - olp[0]) <= TOL
+    else:
+        assert (lp == 0).all()
+        assert float(loss.item()) == 0.0
