@@ -449,6 +449,16 @@ typedef enum {
  * the caller.  Returns PACE_ERR_INVALID_ARG for an unknown kernel. */
 PACE_API pace_status pace_set_profile_events(int32_t kernel, void* begin, void* end);
 
+/* Not part of the method: exercises the failure path every tensor-core
+ * kernel relies on.  One GPU thread waits, with the same bounded wait the
+ * kernels use, on an mbarrier that nothing ever completes; after limit_ns
+ * (1 .. 2e9) it gives up, writes PACE_ERR_TIMEOUT to *status_dev (device, the
+ * usual first-error-wins word) and the kernel returns normally, leaving the
+ * context usable.  Returns PACE_ERR_INVALID_ARG for a NULL status or a limit
+ * outside that range. */
+PACE_API pace_status pace_wait_timeout_selftest(uint64_t limit_ns, int32_t* status_dev,
+                                                void* stream);
+
 /* Not part of the method: the number of CUDA kernels this library has
  * launched from the calling host thread since it was loaded (memsets and
  * copies are not kernels and are not counted). */

@@ -25,6 +25,7 @@
 
 #include "pace_internal.cuh"
 #include "pace_loss.cuh"
+#include "pace_tma.cuh"
 
 namespace pace {
 namespace {
@@ -432,35 +433,6 @@ __global__ void count_used_seqs_kernel(const long long* __restrict__ seq_in, int
 
 // ---------------------------------------------------------------- host side
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* f = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-  });
-  return fn;
-}
-
-// bf16 matrix [rows][cols] with row stride ld elements; box {box_inner, box_outer}.
-pace_status encode_2d(CUtensorMap* tm, const void* ptr, int64_t rows, int64_t cols, int64_t ld,
-                      int box_inner, int box_outer) {
-  auto enc = encode_fn();
-  if (!enc) return PACE_ERR_CUDA;
-  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_outer)};
-  cuuint32_t estr[2] = {1, 1};
-  CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
-                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS ? PACE_OK : PACE_ERR_UNSUPPORTED_SHAPE;
-}
-
 template <bool A_MN, bool B_MN, int EPI>
 pace_status launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmArgs a,
                         cudaStream_t st) {
@@ -606,8 +578,8 @@ extern "C" pace_status pace_token_logprob_backward(
     // 1. G = (g / tau) (onehot - softmax) for the chunk's rows (bf16)
     {
       CUtensorMap ta, tb;
-      PACE_TRY(encode_2d(&ta, hc, hc_rows, H, H, 64, GBM));
-      PACE_TRY(encode_2d(&tb, w_vocab, V, H, H, 64, GBN / 2));
+      PACE_TRY(encode_bf16_2d(&ta, hc, hc_rows, H, H, 64, GBM));
+      PACE_TRY(encode_bf16_2d(&tb, w_vocab, V, H, H, 64, GBN / 2));
       GemmArgs a = {};
       a.M = rows_c_pad;
       a.N = V;
@@ -630,8 +602,8 @@ extern "C" pace_status pace_token_logprob_backward(
     // 2. dH rows = G W   (W read MN-major: [K = V][N = H])
     {
       CUtensorMap ta, tb;
-      PACE_TRY(encode_2d(&ta, ws.g, rows_c_pad, V, ldg, 64, GBM));
-      PACE_TRY(encode_2d(&tb, w_vocab, V, H, H, 64, 64));
+      PACE_TRY(encode_bf16_2d(&ta, ws.g, rows_c_pad, V, ldg, 64, GBM));
+      PACE_TRY(encode_bf16_2d(&tb, w_vocab, V, H, H, 64, 64));
       GemmArgs a = {};
       a.M = rows_c_pad;
       a.N = H;
@@ -648,8 +620,8 @@ extern "C" pace_status pace_token_logprob_backward(
     // 3. dW += G^T H_c   (G read MN-major: [K = rows][M = V]; H_c MN-major: [K = rows][N = H])
     {
       CUtensorMap ta, tb;
-      PACE_TRY(encode_2d(&ta, ws.g, rows_c_pad, V, ldg, 64, 64));
-      PACE_TRY(encode_2d(&tb, hc, hc_rows, H, H, 64, 64));
+      PACE_TRY(encode_bf16_2d(&ta, ws.g, rows_c_pad, V, ldg, 64, 64));
+      PACE_TRY(encode_bf16_2d(&tb, hc, hc_rows, H, H, 64, 64));
       GemmArgs a = {};
       a.M = V;
       a.N = H;

@@ -36,6 +36,7 @@
 
 #include "pace_internal.cuh"
 #include "pace_loss.cuh"
+#include "pace_tma.cuh"
 
 namespace pace {
 namespace {
@@ -344,35 +345,6 @@ __global__ void lse_merge_kernel(int64_t rows_cap, const long long* __restrict__
 
 // ---------------------------------------------------------------- host side
 
-PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* f = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-  });
-  return fn;
-}
-
-// 2-D bf16 tensor [rows][H] (row-major), boxes of box_rows x 64 with the
-// 128-byte swizzle the UMMA descriptors expect.
-pace_status encode_bf16_2d(CUtensorMap* tm, const void* ptr, int64_t rows, int H, int box_rows) {
-  auto enc = get_encode_fn();
-  if (!enc) return PACE_ERR_CUDA;
-  cuuint64_t dims[2] = {static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(H) * 2};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
-  cuuint32_t estr[2] = {1, 1};
-  CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
-                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS ? PACE_OK : PACE_ERR_UNSUPPORTED_SHAPE;
-}
-
 int choose_splits(int n_vtiles) {
   int s = 4;
   if (s > n_vtiles) s = n_vtiles;
@@ -479,8 +451,8 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   const int S = choose_splits(n_vtiles);
   const int tps = (n_vtiles + S - 1) / S;
   CUtensorMap tm_a, tm_b;
-  PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, BM));
-  PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, BN / CLUSTER));
+  PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, H, BK, BM));
+  PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, H, BK, BN / CLUSTER));
   LmLaunchInfo li;
   PACE_TRY(lm_launch_info(&li));
   LmArgs a;

@@ -7,6 +7,7 @@
 #include <math.h>
 #include <stdint.h>
 
+#include "pace_block.cuh"
 #include "pace_internal.cuh"
 #include "pace_loss.cuh"
 
@@ -64,19 +65,6 @@ pace_status launch_group_adv(const float* reward, const uint8_t* accepted, int64
 
 constexpr int kSurThreads = 256;
 
-// Fixed-shape block tree sum (blockDim.x == kSurThreads); deterministic.
-__device__ double block_sum_fixed(double v, double* sh) {
-  sh[threadIdx.x] = v;
-  __syncthreads();
-  for (int o = kSurThreads / 2; o > 0; o >>= 1) {
-    if (threadIdx.x < o) sh[threadIdx.x] = __dadd_rn(sh[threadIdx.x], sh[threadIdx.x + o]);
-    __syncthreads();
-  }
-  const double r = sh[0];
-  __syncthreads();
-  return r;
-}
-
 __device__ __forceinline__ float clipped_term(float lp, float behav, float a, float eps_low,
                                               float eps_high, float dual, float* rho_out) {
   float d = lp - behav;
@@ -122,8 +110,8 @@ __global__ void __launch_bounds__(kSurThreads)
       }
       if (ratio) ratio[r] = in ? rho : 0.0f;
     }
-    const double ts = block_sum_fixed(tot, sh);
-    const double tc = block_sum_fixed(cnt, sh);
+    const double ts = block_sum_fixed<kSurThreads>(tot, sh);
+    const double tc = block_sum_fixed<kSurThreads>(cnt, sh);
     if (threadIdx.x == 0) {
       seq_sum[i] = ts;
       seq_cnt[i] = tc;
@@ -147,8 +135,8 @@ __global__ void __launch_bounds__(kSurThreads)
       b = __dadd_rn(b, 1.0);
     }
   }
-  const double ta = block_sum_fixed(a, sh);
-  const double tb = block_sum_fixed(b, sh);
+  const double ta = block_sum_fixed<kSurThreads>(a, sh);
+  const double tb = block_sum_fixed<kSurThreads>(b, sh);
   if (threadIdx.x == 0) *loss = tb > 0.0 ? __ddiv_rn(ta, tb) : 0.0;
 }
 

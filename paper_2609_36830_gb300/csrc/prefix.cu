@@ -7,6 +7,7 @@
 #include <math.h>
 #include <stdint.h>
 
+#include "pace_block.cuh"
 #include "pace_internal.cuh"
 #include "pace_loss.cuh"
 
@@ -54,19 +55,6 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
-// Fixed-shape block tree sum in fp64 (deterministic).
-__device__ double block_sum(double v, double* sh) {
-  sh[threadIdx.x] = v;
-  __syncthreads();
-  for (int o = kThreads / 2; o > 0; o >>= 1) {
-    if (threadIdx.x < o) sh[threadIdx.x] = __dadd_rn(sh[threadIdx.x], sh[threadIdx.x + o]);
-    __syncthreads();
-  }
-  const double r = sh[0];
-  __syncthreads();
-  return r;
-}
-
 __global__ void __launch_bounds__(kThreads)
     prefix_reduce_kernel(const int64_t* __restrict__ seq_offsets,
                          const uint8_t* __restrict__ mask_c, const long long* __restrict__ n_elig,
@@ -83,7 +71,7 @@ __global__ void __launch_bounds__(kThreads)
       for (int64_t r = r0 + threadIdx.x; r < r1; r += kThreads)
         if (mask_c[r])
           acc = __dadd_rn(acc, fabs(static_cast<double>(logprob[r]) - static_cast<double>(behav[r])));
-    const double tot = block_sum(acc, sh);
+    const double tot = block_sum_fixed<kThreads>(acc, sh);
     if (threadIdx.x == 0) {
       const long long m = ne < cap ? ne : cap;
       s_pre[i] = ne >= min_tokens ? static_cast<float>(__ddiv_rn(tot, static_cast<double>(m)))

@@ -17,6 +17,7 @@
 
 #include <mutex>
 
+#include "pace_block.cuh"
 #include "pace_internal.cuh"
 
 namespace pace {
@@ -47,37 +48,6 @@ struct SelectState {
   int done;
   int pad;
 };
-
-// Block-wide exclusive scan of one value per thread (blockDim.x a multiple of
-// 32, <= 1024).  Returns the exclusive prefix; *total gets the block sum.
-template <typename T>
-__device__ T block_exclusive_scan(T v, T* total) {
-  __shared__ T warp_sums[32];
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  T x = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const T y = __shfl_up_sync(0xffffffffu, x, o);
-    if (lane >= o) x += y;
-  }
-  if (lane == 31) warp_sums[wid] = x;
-  __syncthreads();
-  const int nw = blockDim.x >> 5;
-  if (wid == 0) {
-    T w = lane < nw ? warp_sums[lane] : T(0);
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const T y = __shfl_up_sync(0xffffffffu, w, o);
-      if (lane >= o) w += y;
-    }
-    if (lane < nw) warp_sums[lane] = w;  // inclusive
-  }
-  __syncthreads();
-  const T before = wid > 0 ? warp_sums[wid - 1] : T(0);
-  if (total) *total = warp_sums[nw - 1];
-  __syncthreads();
-  return before + x - v;
-}
 
 __device__ __forceinline__ void write_unit(int64_t u, bool rejected, int64_t rej_pos,
                                            int64_t acc_pos, int G, int32_t* accepted_ids,

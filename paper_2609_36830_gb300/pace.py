@@ -97,6 +97,7 @@ SIGNATURES = {
     "pace_token_logprob_backward_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
     "pace_set_profile_events": ([_I32, _P, _P], _I32),
     "pace_kernel_launches": ([], ctypes.c_uint64),
+    "pace_wait_timeout_selftest": ([ctypes.c_uint64, _P, _P], _I32),
 }
 
 
