@@ -31,6 +31,15 @@ __device__ __forceinline__ int4 ld_stream_v4(const int32_t* p) {
   return v;
 }
 
+constexpr int64_t kPrefetchAhead = 4;
+
+// Bulk prefetch of a 16-byte-aligned range into L2 (no data returned).
+__device__ __forceinline__ void l2_prefetch_bulk(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)),
+               "r"(bytes)
+               : "memory");
+}
+
 struct LaneAcc {
   long long sum;   // sum of policy tags seen by this lane for the current trajectory
   unsigned cnt;    // number of policy tokens
@@ -95,7 +104,7 @@ __device__ __forceinline__ bool acc_batch_fast(LaneAcc& a, const int4 (&v)[kTile
 // any length mix are balanced across warps.  The walk never leaves
 // [0, n_traj) and loads only tags[0, n_tokens), whatever the offsets hold;
 // inconsistent offsets are reported by the finalize kernel.
-__global__ void __launch_bounds__(kReduceThreads, 3)
+__global__ void __launch_bounds__(kReduceThreads, 2)
     tag_reduce_kernel(const int32_t* __restrict__ tags, const int64_t* __restrict__ offsets,
                       int64_t n_traj, int64_t n_tokens, unsigned long long* __restrict__ sumv,
                       unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1) {
@@ -119,10 +128,12 @@ __global__ void __launch_bounds__(kReduceThreads, 3)
   int64_t cur_end = offsets[cur + 1];
   LaneAcc acc{0, 0u, 0u};
 
-  for (int64_t b = b_begin; b < b_end; ++b) {
+  auto load_batch = [&](int4 (&v)[kTilesPerBatch], int64_t b) {
     const int64_t bt0 = b * kBatchTokens;
-    const int64_t bt1 = (bt0 + kBatchTokens < n_tokens) ? bt0 + kBatchTokens : n_tokens;
-    int4 v[kTilesPerBatch];
+    // ask L2 for a batch further ahead (no registers held while it is in flight)
+    const int64_t pf = b + kPrefetchAhead;
+    if (lane == 0 && pf < b_end && (pf + 1) * kBatchTokens <= n_tokens)
+      l2_prefetch_bulk(tags + pf * kBatchTokens, static_cast<uint32_t>(kBatchTokens * 4));
     if (bt0 + kBatchTokens <= n_tokens) {
 #pragma unroll
       for (int u = 0; u < kTilesPerBatch; ++u)
@@ -137,6 +148,13 @@ __global__ void __launch_bounds__(kReduceThreads, 3)
         v[u].w = (t + 3 < n_tokens) ? tags[t + 3] : -1;
       }
     }
+  };
+
+  // Adds batch b to the running trajectory sums; false when the offsets end
+  // before the tokens do (inconsistent offsets: stop).
+  auto process = [&](const int4 (&v)[kTilesPerBatch], int64_t b) -> bool {
+    const int64_t bt0 = b * kBatchTokens;
+    const int64_t bt1 = (bt0 + kBatchTokens < n_tokens) ? bt0 + kBatchTokens : n_tokens;
     int64_t pos = bt0;
     while (true) {
       const int64_t seg_hi = cur_end < bt1 ? cur_end : bt1;
@@ -163,16 +181,29 @@ __global__ void __launch_bounds__(kReduceThreads, 3)
           acc_elem(acc, v[u].w, t + 3 >= lo_r && t + 3 < hi_r);
         }
       }
-      if (cur_end > bt1) break;  // trajectory continues into the next batch
+      if (cur_end > bt1) return true;  // trajectory continues into the next batch
       flush(acc, cur, sumv, cnt, maxp1);
       if (seg_hi > pos) pos = seg_hi;
       ++cur;
-      if (cur >= n_traj) return;  // tokens past the last trajectory: offsets are bad
+      if (cur >= n_traj) return false;  // tokens past the last trajectory: offsets are bad
       cur_end = offsets[cur + 1];
       // the next trajectory starts at the batch edge: continue in the next batch;
       // otherwise loop (more of this batch, or empty trajectories to step over)
-      if (pos >= bt1 && cur_end > bt1) break;
+      if (pos >= bt1 && cur_end > bt1) return true;
     }
+  };
+
+  // two register sets: the next batch's loads are in flight while one is added up
+  int4 va[kTilesPerBatch], vb[kTilesPerBatch];
+  int64_t b = b_begin;
+  load_batch(va, b);
+  while (true) {
+    if (b + 1 < b_end) load_batch(vb, b + 1);
+    if (!process(va, b)) return;
+    if (++b >= b_end) break;
+    if (b + 1 < b_end) load_batch(va, b + 1);
+    if (!process(vb, b)) return;
+    if (++b >= b_end) break;
   }
   if (cur < n_traj) flush(acc, cur, sumv, cnt, maxp1);
 }
@@ -332,7 +363,7 @@ pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t 
   const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
   const int warps_per_block = kReduceThreads / 32;
   int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
-  const int64_t cap = static_cast<int64_t>(sm_count()) * 3;  // one wave at 3 blocks / SM
+  const int64_t cap = static_cast<int64_t>(sm_count()) * 2;  // one wave at 2 blocks / SM
   if (blocks > cap) blocks = cap;
   const ProfileEvents& pe = profile_events(PACE_PROFILE_TAG_REDUCE);
   if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
