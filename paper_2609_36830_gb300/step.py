@@ -44,6 +44,12 @@ class StepInputs:
 
 
 class PaceStep:
+    """Buffers and calls of one trainer step; call ``run`` once per step.
+
+    The pool in ``x`` may be refreshed in place between steps (new tags, versions,
+    rows); ``n_target``, ``beta`` and ``r_max`` follow the paper's Eqs. 3-4 and the
+    admission settings."""
+
     def __init__(self, x: StepInputs, score_params=None, loss_params=None, beta=0.0,
                  r_max=0.9, temperature=1.0, device="cuda"):
         self.x = x
@@ -84,7 +90,9 @@ class PaceStep:
         self.k_units = None
 
     def run(self, stream=None):
-        """Queue one step; returns (k_units, r_hat).  Nothing is synchronised."""
+        """Queue one step; returns (k_units, r_hat).  Nothing is synchronised.
+
+        r_hat (Eq. 4) is carried into the next call's budget as r-hat_{j-1}."""
         x = self.x
         pace.score_pool(x.tags, x.offsets, x.c_version, x.s_pre, x.trainer_version, x.window,
                         self.sp, out=self.score_out, ws=self.ws_score, status=self.status,
@@ -98,6 +106,7 @@ class PaceStep:
                            loss=self.loss_args, logprob=self.logprob, ws=self.ws_lm,
                            status=self.status, stream=stream)
         self.k_units = k
+        self.r_hat = r_hat
         return k, r_hat
 
     def rows_in_loss(self) -> int:

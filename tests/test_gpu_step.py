@@ -59,3 +59,59 @@ def test_math7b_step(n_traj):
     assert float(st.loss.item()) == float(loss2.item())
     assert math.isfinite(float(st.loss.item()))
     assert st.rows_in_loss() == int(in_loss.sum())
+
+
+
+def test_ema_budget_carried_across_steps():
+    """Eq. 4 across steps: r-hat_j = beta r-hat_{j-1} + (1 - beta) r_j.  The step
+    driver carries r-hat from one call to the next while the pool occupancy changes;
+    the oracle runs the same recurrence and the rejected groups must match."""
+    beta, n_target = 0.5, 24
+    o_rhat, r_hat_prev = 0.0, 0.0
+    for i, n_traj in enumerate([96, 64, 48, 80, 96, 24]):
+        pool = workloads.make_pool("tiny", seed=900 + i, n_traj=n_traj)
+        rw = workloads.make_rows(pool)
+        H, V = pool.spec.hidden, pool.spec.vocab
+        hidden = workloads.bf16_normal_device((rw.n_rows, H), 1.0, 40 + i)
+        w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), 41)
+        behav = workloads.behaviour_logprob(rw, pool.trainer_version,
+                                            workloads.uniform_center(V), i)
+        x = step.build_inputs(pool, rw, hidden, w, behav)
+        x.n_target = n_target
+        st = step.PaceStep(x, beta=beta)
+        st.r_hat = r_hat_prev  # a new pool shape needs new buffers; the state carries over
+        k, r_hat = st.run()
+        torch.cuda.synchronize()
+        assert int(st.status.item()) == 0
+        U = n_traj // pool.group_size
+        _, _, o_rhat, ok = oracle.budget(n_traj, n_target, beta, 0.9, o_rhat, U)
+        assert (k, r_hat) == (ok, o_rhat), i
+        assert st.r_hat == r_hat
+        _, _, _, _, _, ous = oracle.score_pool(pool.tags, pool.meta["offsets_host"],
+                                               pool.c_version, pool.s_pre,
+                                               pool.trainer_version, pool.window,
+                                               group_size=pool.group_size)
+        _, _, _, oflag = oracle.select(ous, pool.group_size, ok)
+        np.testing.assert_array_equal(as_np(st.sel_out["flags"]), oflag)
+        r_hat_prev = r_hat
+    assert o_rhat > 0.0  # the carried state reached the last, under-target step
+
+
+def test_repeated_run_advances_ema():
+    """Calling run() twice on one pool applies Eq. 4 twice."""
+    pool = workloads.make_pool("tiny", seed=77, n_traj=96)
+    rw = workloads.make_rows(pool)
+    H, V = pool.spec.hidden, pool.spec.vocab
+    hidden = workloads.bf16_normal_device((rw.n_rows, H), 1.0, 78)
+    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), 79)
+    behav = workloads.behaviour_logprob(rw, pool.trainer_version, workloads.uniform_center(V), 1)
+    x = step.build_inputs(pool, rw, hidden, w, behav)
+    st = step.PaceStep(x, beta=0.75)
+    U = 96 // pool.group_size
+    o = 0.0
+    for _ in range(3):
+        k, r_hat = st.run()
+        _, _, o, ok = oracle.budget(96, x.n_target, 0.75, 0.9, o, U)
+        assert (k, r_hat) == (ok, o)
+    torch.cuda.synchronize()
+    assert int(st.status.item()) == 0
