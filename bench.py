@@ -6,9 +6,10 @@ log-probs, GRPO advantages and clipped surrogate of the accepted rows
 (pace_token_logprob).  The workload is the 7B-shaped single-turn math pool
 (512 trajectories = 64 prompts x 8, 256 masked prompt rows + lognormal
 responses, hidden 3584, vocab 152064, capacity 384): the metric is accepted
-tokens per second (rows in the loss / step time).  A second line item times
-pool scoring + selection alone on the 1M-trajectory sweep pool against HBM
-bandwidth.
+tokens per second (rows in the loss / step time).  Further line items time
+pool scoring + selection alone on the sweep pools (1k, 16k, 128k and 1M
+trajectories) against HBM bandwidth, prefix rescoring (Eq. 6) and the LM-head
+backward.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
@@ -41,6 +42,7 @@ WORKLOAD = "math7b"
 LMHEAD_DRAM_BYTES_PER_ROW = 1.135e9 / 4864
 TAG_REDUCE_DRAM_BYTES_PER_TAG = 223.226e6 / 54929421
 SWEEP_N = 1048576
+SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)
 METRIC = "accepted tokens/sec (logprob+loss) and % bf16 tensor peak; pool scoring traj/s + HBM GB/s"
 UNIT = "tokens/s"
 
@@ -126,11 +128,12 @@ def _make_step(seed_offset, device):
     return pool, rows, x, step.PaceStep(x, loss_params=lp_params, device=device)
 
 
-def _sweep_scoring(steps, warmup, device):
-    """pace_score_pool + pace_select on the 1M-trajectory pool; tag-reduction roofline."""
+def _sweep_scoring(steps, warmup, device, n_traj=SWEEP_N):
+    """pace_score_pool + pace_select on one sweep pool; tag-reduction roofline.  L2 is
+    flushed before every timed call (the small pools fit in it)."""
     import torch
     from paper_2609_36830_gb300 import pace, workloads
-    pool = workloads.make_pool("sweep", n_traj=SWEEP_N, device=device)
+    pool = workloads.make_pool("sweep", n_traj=n_traj, device=device)
     n = pool.n_traj
     tok = int(pool.meta["offsets_host"][-1])
     c = torch.from_numpy(pool.c_version).to(device)
@@ -306,10 +309,30 @@ def _cpu_baseline(pool, rows, x, step_obj, n_rows_sample):
                                      rows.targets[sample], n_threads=cores)
     t_lp = time.perf_counter() - t0
     t_step = t_adm + t_lp * (M / n_rows_sample)
+    # the same oracle on one core, on a 16x smaller row sample
+    n1 = max(n_rows_sample // 16, 1)
+    t0 = time.perf_counter()
+    oracle.token_logprob(hb[:n1].view(np.uint16), wb.view(np.uint16),
+                         rows.targets[sample[:n1]], n_threads=1)
+    t_lp1 = time.perf_counter() - t0
     return {"value": M / t_step, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "cpu": _cpu_model(),
             "sample": f"full admission of the {pool.n_traj}-trajectory pool ({t_adm:.3f} s) + "
                       f"fp64 log-probs of {n_rows_sample} of the {M} rows in the loss "
-                      f"({t_lp:.1f} s), extrapolated to all rows"}
+                      f"({t_lp:.1f} s), extrapolated to all rows",
+            "single_core": {"value": M / (t_adm + t_lp1 * (M / n1)), "unit": UNIT, "cores": 1,
+                            "sample": f"fp64 log-probs of {n1} rows on one thread ({t_lp1:.1f} s)"}}
+
+
+def _cpu_model():
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return None
 
 
 def run_reference(args):
@@ -332,7 +355,7 @@ def run_reference(args):
     else:
         wb = workloads.bf16_normal_host((V, H), 1.0 / math.sqrt(H), pool.seed + 12)
     cores = os.cpu_count() or 1
-    rows_per_step = 16
+    rows_per_step = 64
     times = []
     M = None
     for i in range(args.warmup + args.steps):
@@ -486,9 +509,18 @@ def run_gpu(args):
     if not args.no_sweep and rank == 0:
         del x, st
         torch.cuda.empty_cache()
-        sweep = _sweep_scoring(max(3, min(K, 5)), 3, device)
-        sweep["tag_reduce_frac_of_hbm"] = sweep["tag_reduce_gbs"] / peaks["hbm_gbs"]
-        sweep["hbm_peak_gbs"] = peaks["hbm_gbs"]
+        sizes = []
+        for n_sw in SWEEP_SIZES:
+            r_sw = _sweep_scoring(max(3, min(K, 5)) if n_sw == SWEEP_N else 10, 3, device, n_sw)
+            r_sw["tag_reduce_frac_of_hbm"] = r_sw["tag_reduce_gbs"] / peaks["hbm_gbs"]
+            r_sw["hbm_peak_gbs"] = peaks["hbm_gbs"]
+            if n_sw == SWEEP_N:
+                sweep = r_sw
+            else:
+                sizes.append({k: r_sw[k] for k in ("workload", "traj_per_s", "ms_per_call",
+                                                   "tag_reduce_ms", "tag_reduce_gbs",
+                                                   "tag_reduce_frac_of_hbm")})
+        sweep["smaller_pools"] = sizes
 
     prefix = None
     backward = None
@@ -634,7 +666,7 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--cpu-rows", type=int, default=64)
+    ap.add_argument("--cpu-rows", type=int, default=512)
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce"], default=None,

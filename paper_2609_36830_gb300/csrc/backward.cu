@@ -6,7 +6,10 @@
 // For the rows in the loss, in chunks of up to kChunkRows compacted rows:
 //   1. gemm_kernel<EPI_G>:    z = H_c W^T recomputed on the tensor cores; the
 //                             epilogue writes G = (g / tau) (onehot(y) - softmax(z / tau))
-//                             in bf16, using the forward's log-sum-exp;
+//                             in bf16, using the forward's log-sum-exp, in 64-column
+//                             blocks: G[v / 64][row][v % 64], so that both later
+//                             GEMMs read it in long contiguous runs (a K step of
+//                             dH is one 16 KB run, a K step of dW 8 KB);
 //   2. gemm_kernel<EPI_ROWS>: dH_c = G W (A = G K-major, B = W read MN-major),
 //                             fp32 rows scattered back to their original row;
 //   3. gemm_kernel<EPI_ACC>:  dW += G^T H_c (A = G and B = H_c, both read
@@ -44,11 +47,14 @@ constexpr int64_t kChunkRows = 65536;         // rows of G held at once (bf16 M 
 constexpr int kGroupM = 38;                   // M tiles per raster group
 
 enum { EPI_G = 0, EPI_ROWS = 1, EPI_ACC = 2 };
+enum { TRIM_NONE = 0, TRIM_M = 1, TRIM_K = 2 };
 
 struct GemmArgs {
   int64_t M, N, K;
   int64_t m_tiles, n_tiles;
   int raster_n_fast;            // 1: N tile fastest; 0: groups of kGroupM M tiles, M fastest
+  int trim;                     // TRIM_M / TRIM_K: that extent is cut, on the device, to the
+                                // chunk's rows in the loss rounded up to GBM (TRIM_NONE: as given)
   // EPI_G
   int64_t chunk_row0;           // compact row of the chunk's first row
   const long long* n_valid;     // rows in the loss (device)
@@ -58,8 +64,11 @@ struct GemmArgs {
   const float* dlp;             // dLoss/dlp per original row
   float scale_log2;             // log2(e) / tau
   float inv_tau;
-  uint16_t* g_out;              // bf16 [rows of chunk][ldg]
-  int64_t ldg;
+  uint16_t* g_out;              // bf16 G in 64-column blocks: [g_cols / 64][g_pitch][64]
+  int64_t g_cols;               // V rounded up to 64 (columns >= V hold zeros)
+  int64_t g_pitch;              // rows per 64-column block
+  // A operand from the blocked G (a_pitch > 0: rows per 64-column block); 0: plain matrix
+  int64_t a_pitch;
   int32_t V;
   // EPI_ROWS
   float* rows_out;              // fp32 [orig rows][ldo]
@@ -72,9 +81,9 @@ struct GemmArgs {
 // Work items are (pair of M tiles, N tile); the two CTAs of a cluster take the
 // two M tiles of a pair and share every B tile, each loading half of it and
 // multicasting it to both.
-__device__ __forceinline__ void item_of(const GemmArgs& p, int64_t item, int64_t* mp,
-                                        int64_t* n) {
-  const int64_t pairs = (p.m_tiles + 1) / 2;
+__device__ __forceinline__ void item_of(const GemmArgs& p, int64_t m_tiles, int64_t item,
+                                        int64_t* mp, int64_t* n) {
+  const int64_t pairs = (m_tiles + 1) / 2;
   if (p.raster_n_fast) {
     *mp = item / p.n_tiles;
     *n = item % p.n_tiles;
@@ -136,10 +145,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t crank = cluster_ctarank();
-  const int64_t n_items = (p.m_tiles + 1) / 2 * p.n_tiles;
+  // The host sizes a chunk by its row capacity; the rows of it that are in the
+  // loss are known only on the device (the compaction's count).  Tiles past
+  // them hold zero rows: M (G, dH) or K (dW) is cut to the count rounded up to
+  // GBM, the same value in every CTA, so every early exit below is uniform.
+  int64_t M = p.M, K = p.K, m_tiles = p.m_tiles;
+  if (p.trim != TRIM_NONE) {
+    int64_t v = static_cast<int64_t>(*p.n_valid) - p.chunk_row0;
+    const int64_t cap = p.trim == TRIM_M ? p.M : p.K;
+    v = v < 0 ? 0 : (v > cap ? cap : v);
+    v = (v + GBM - 1) / GBM * GBM;
+    if (v > cap) v = cap;
+    if (p.trim == TRIM_M) {
+      M = v;
+      m_tiles = (v + GBM - 1) / GBM;
+    } else {
+      K = v;
+    }
+  }
+  const int64_t n_items = (m_tiles + 1) / 2 * p.n_tiles;
   const int64_t cid = blockIdx.x / 2, n_clusters = gridDim.x / 2;
-  const int nkb = static_cast<int>((p.K + GBK - 1) / GBK);
-  if (nkb == 0) return;  // uniform over the grid
+  const int nkb = static_cast<int>((K + GBK - 1) / GBK);
+  if (nkb == 0 || n_items == 0) return;  // uniform over the grid
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < GSTAGES; ++s) {
@@ -175,7 +202,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       bool ok = true;
       for (int64_t t = cid; t < n_items && ok; t += n_clusters) {
         int64_t mp, nt;
-        item_of(p, t, &mp, &nt);
+        item_of(p, m_tiles, t, &mp, &nt);
         const int32_t m0 = static_cast<int32_t>((2 * mp + crank) * GBM);
         const int32_t n0 = static_cast<int32_t>(nt * GBN);
         for (int kb = 0; kb < nkb; ++kb, ++it) {
@@ -188,7 +215,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           unsigned char* sb = sa + kGStageA;
           mbar_arrive_expect_tx(&full[s], kGStageBytes);
           const int32_t k0 = kb * GBK;
-          if (A_MN) {  // box {64 MN, 64 K}: two along M
+          if (p.a_pitch > 0) {  // blocked G: one 64-wide block is the inner dimension
+            const int64_t ap = p.a_pitch;
+            if (A_MN) {  // M = vocabulary: blocks m0 / 64 and m0 / 64 + 1, rows k0..k0+63
+              const int64_t b0 = m0 / 64;
+              tma_load_2d(sa, &tm_a, &full[s], 0, static_cast<int32_t>(b0 * ap + k0), pol);
+              tma_load_2d(sa + 8192, &tm_a, &full[s], 0,
+                          static_cast<int32_t>((b0 + 1) * ap + k0), pol);
+            } else {     // K = vocabulary: block kb, rows m0..m0+127
+              tma_load_2d(sa, &tm_a, &full[s], 0, static_cast<int32_t>(kb * ap + m0), pol);
+            }
+          } else if (A_MN) {  // box {64 MN, 64 K}: two along M
             tma_load_2d(sa, &tm_a, &full[s], m0, k0, pol);
             tma_load_2d(sa + 8192, &tm_a, &full[s], m0 + 64, k0, pol);
           } else {     // box {64 K, 128 rows}
@@ -260,7 +297,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     uint32_t tc = 0;
     for (int64_t t = cid; t < n_items; t += n_clusters, ++tc) {
       int64_t mp, nt;
-      item_of(p, t, &mp, &nt);
+      item_of(p, m_tiles, t, &mp, &nt);
       const int64_t mt = 2 * mp + crank;
       const uint32_t acc = tc & 1u, acc_ph = (tc >> 1) & 1u;
       if (!mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag)) {
@@ -273,7 +310,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       const int64_t n0 = nt * GBN;
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * GBN;
       // per-row context
-      bool row_ok = row < p.M;
+      bool row_ok = row < M;
       int32_t y = -1;
       float gscale = 0.0f, lse2 = 0.0f;
       int64_t orig = -1;
@@ -295,7 +332,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         tmem_wait_ld();
         const int64_t col0 = n0 + c;
         if (EPI == EPI_G) {
-          if (row_ok && col0 < p.V) {
+          if (row_ok && col0 < p.g_cols) {
             // G = (g / tau) (onehot - p), zero for rows outside the loss
             uint32_t packed[16];
 #pragma unroll
@@ -310,17 +347,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
               packed[i / 2] = static_cast<uint32_t>(f32_to_bf16_rn(g0)) |
                               (static_cast<uint32_t>(f32_to_bf16_rn(g1)) << 16);
             }
-            uint16_t* dst = p.g_out + row * p.ldg + col0;
-            if (col0 + 32 <= p.ldg) {
-              uint4* d4 = reinterpret_cast<uint4*>(dst);
+            // col0 is a multiple of 32, so the 32 columns lie in one 64-column block
+            uint4* d4 = reinterpret_cast<uint4*>(
+                p.g_out + ((col0 >> 6) * p.g_pitch + row) * 64 + (col0 & 63));
 #pragma unroll
-              for (int q = 0; q < 4; ++q)
-                d4[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2],
-                                   packed[4 * q + 3]);
-            } else {
-              for (int i = 0; i < 32 && col0 + i < p.ldg; ++i)
-                dst[i] = static_cast<uint16_t>(packed[i / 2] >> (16 * (i & 1)));
-            }
+            for (int q = 0; q < 4; ++q)
+              d4[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2],
+                                 packed[4 * q + 3]);
           }
         } else if (EPI == EPI_ROWS) {
           if (row_ok) {
@@ -366,12 +399,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   if (warp == 1) tmem_dealloc(tmem_base, kGTmemCols);
 }
 
-// Zero the gathered rows [n_valid, rows_end) of the compact buffer so that
-// rows outside the loss contribute exactly 0 to dW (0 x garbage could be NaN).
+// Zero the gathered rows from n_valid up to the next multiple of GBM (at most
+// rows_end) of the compact buffer: dW reads whole GBM-row tiles of them, and the
+// rows outside the loss must contribute exactly 0 (0 x garbage could be NaN).
 __global__ void zero_tail_rows_kernel(uint4* __restrict__ buf, int64_t row_vecs,
                                       const long long* __restrict__ n_valid, int64_t rows_end) {
   const int64_t start = *n_valid;
-  const int64_t total = (rows_end - start) * row_vecs;
+  int64_t end = (start + GBM - 1) / GBM * GBM;
+  if (end > rows_end) end = rows_end;
+  const int64_t total = (end - start) * row_vecs;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x)
     buf[start * row_vecs + i] = make_uint4(0, 0, 0, 0);
@@ -462,7 +498,7 @@ pace_status launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmArgs a
 
 struct BwWs {
   LmWs lm;            // compaction + gathered rows (hidden_c)
-  uint16_t* g;        // bf16 [chunk][ldg]
+  uint16_t* g;        // bf16 G of one chunk, 64-column blocks [ceil(V / 64)][chunk][64]
   int* n_seq_used;
 };
 
@@ -473,8 +509,8 @@ int64_t chunk_rows(int64_t n_rows) {
 
 void carve_bw_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, BwWs* w) {
   carve_lm_ws(cv, n_rows, n_seq, H, V, true, &w->lm);
-  const int64_t ldg = (static_cast<int64_t>(V) + 7) / 8 * 8;
-  w->g = cv.take<uint16_t>(static_cast<size_t>(chunk_rows(n_rows > 0 ? n_rows : 1)) * ldg);
+  const int64_t g_cols = (static_cast<int64_t>(V) + 63) / 64 * 64;
+  w->g = cv.take<uint16_t>(static_cast<size_t>(chunk_rows(n_rows > 0 ? n_rows : 1)) * g_cols);
   w->n_seq_used = cv.take<int>(1);
 }
 
@@ -567,7 +603,10 @@ extern "C" pace_status pace_token_logprob_backward(
       static_cast<uint4*>(ws.lm.hidden_c), row_vecs, ws.lm.cw.total, rows_cap);
   PACE_TRY(last_launch_status());
   const int64_t chunk = chunk_rows(n_rows);
-  const int64_t ldg = (static_cast<int64_t>(V) + 7) / 8 * 8;
+  const int64_t g_cols = (static_cast<int64_t>(V) + 63) / 64 * 64;
+  const int64_t g_blocks = g_cols / 64;
+  // TMA row coordinates of the blocked G are 32-bit
+  if (g_blocks * chunk > static_cast<int64_t>(INT32_MAX)) return PACE_ERR_UNSUPPORTED_SHAPE;
   for (int64_t c0 = 0; c0 < n_rows; c0 += chunk) {
     const int64_t rows_c = (n_rows - c0) < chunk ? (n_rows - c0) : chunk;
     const int64_t rows_c_pad = (rows_c + GBM - 1) / GBM * GBM;
@@ -585,6 +624,7 @@ extern "C" pace_status pace_token_logprob_backward(
       a.N = V;
       a.K = H;
       a.raster_n_fast = 0;
+      a.trim = TRIM_M;
       a.chunk_row0 = c0;
       a.n_valid = ws.lm.cw.total;
       a.rowidx = ws.lm.cw.rowidx;
@@ -594,7 +634,8 @@ extern "C" pace_status pace_token_logprob_backward(
       a.scale_log2 = 1.4426950408889634f / temperature;
       a.inv_tau = 1.0f / temperature;
       a.g_out = ws.g;
-      a.ldg = ldg;
+      a.g_cols = g_cols;
+      a.g_pitch = rows_c_pad;
       a.V = V;
       a.status = status_dev;
       PACE_TRY((launch_gemm<false, false, EPI_G>(ta, tb, a, st)));
@@ -602,13 +643,15 @@ extern "C" pace_status pace_token_logprob_backward(
     // 2. dH rows = G W   (W read MN-major: [K = V][N = H])
     {
       CUtensorMap ta, tb;
-      PACE_TRY(encode_bf16_2d(&ta, ws.g, rows_c_pad, V, ldg, 64, GBM));
+      PACE_TRY(encode_bf16_2d(&ta, ws.g, g_blocks * rows_c_pad, 64, 64, 64, GBM));
       PACE_TRY(encode_bf16_2d(&tb, w_vocab, V, H, H, 64, 64));
       GemmArgs a = {};
       a.M = rows_c_pad;
       a.N = H;
       a.K = V;
+      a.a_pitch = rows_c_pad;
       a.raster_n_fast = 1;
+      a.trim = TRIM_M;
       a.chunk_row0 = c0;
       a.n_valid = ws.lm.cw.total;
       a.rowidx = ws.lm.cw.rowidx;
@@ -620,13 +663,17 @@ extern "C" pace_status pace_token_logprob_backward(
     // 3. dW += G^T H_c   (G read MN-major: [K = rows][M = V]; H_c MN-major: [K = rows][N = H])
     {
       CUtensorMap ta, tb;
-      PACE_TRY(encode_bf16_2d(&ta, ws.g, rows_c_pad, V, ldg, 64, 64));
+      PACE_TRY(encode_bf16_2d(&ta, ws.g, g_blocks * rows_c_pad, 64, 64, 64, 64));
       PACE_TRY(encode_bf16_2d(&tb, hc, hc_rows, H, H, 64, 64));
       GemmArgs a = {};
       a.M = V;
       a.N = H;
       a.K = rows_c_pad;
+      a.a_pitch = rows_c_pad;
       a.raster_n_fast = 1;
+      a.trim = TRIM_K;
+      a.chunk_row0 = c0;
+      a.n_valid = ws.lm.cw.total;
       a.acc_out = grad_w;
       a.ldo = H;
       a.status = status_dev;

@@ -118,3 +118,31 @@ def test_full_size_backward_sampled_rows_and_identity():
     col_sum = dw.double().sum(dim=0)
     assert float(col_sum.norm()) <= 1e-2 * float(dw.double().norm())
     assert torch.isfinite(dw).all()
+
+
+@pytest.mark.parametrize("rows,frac", [(135000, 0.3), (135000, 0.98)])
+def test_lmhead_backward_multi_chunk_trimmed(rows, frac):
+    """More rows than one 65,536-row chunk, with the rows in the loss ending inside
+    the first (frac 0.3: later chunks hold none) or inside the last chunk (0.98):
+    the GEMMs cut their extent to the device-side count and dW must still be whole."""
+    H, V = 64, 256
+    rng = np.random.default_rng(int(frac * 100))
+    hb = workloads.bf16_normal_host((rows, H), 1.0, 5)
+    wb = workloads.bf16_normal_host((V, H), 2.0 / math.sqrt(H), 6)
+    y = rng.integers(0, V, size=rows).astype(np.int32)
+    mask = (rng.random(rows) < frac).astype(np.uint8)
+    g = (rng.standard_normal(rows) * mask).astype(np.float32)
+    so = to_dev(np.array([0, rows], np.int64))
+    b = pace.make_batch(so, rows, mask=to_dev(mask))
+    hidden, w = bf16_dev(hb), bf16_dev(wb)
+    lse = torch.empty(rows, dtype=torch.float32, device=DEV)
+    status = pace.new_status(DEV)
+    pace.token_logprob(b, hidden, w, to_dev(y), 1.0, lse=lse, status=status)
+    dh, dw = pace.token_logprob_backward(b, hidden, w, to_dev(y), lse, to_dev(g), status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    st, odh, odw = oracle.lmhead_backward(hb, wb, y, g.astype(np.float64))
+    assert st == 0
+    assert _rel(as_np(dh), odh) <= REL, _rel(as_np(dh), odh)
+    assert _rel(as_np(dw), odw) <= REL, _rel(as_np(dw), odw)
+    assert (as_np(dh)[mask == 0] == 0).all()
