@@ -117,12 +117,33 @@ __global__ void __launch_bounds__(kReduceThreads, 2)
   if (b_begin >= b_end) return;
   const int64_t t_begin = b_begin * kBatchTokens;
 
-  // trajectory holding token t_begin: largest i < n_traj with offsets[i] <= t_begin
+  // Start the stream before the search below: the warp's first batches are
+  // requested into L2 while the offsets are searched (lanes 0..kPrefetchAhead-1,
+  // one batch each; the pipeline then keeps kPrefetchAhead batches ahead).
+  if (lane < kPrefetchAhead) {
+    const int64_t pf = b_begin + lane;
+    if (pf < b_end && (pf + 1) * kBatchTokens <= n_tokens)
+      l2_prefetch_bulk(tags + pf * kBatchTokens, static_cast<uint32_t>(kBatchTokens * 4));
+  }
+
+  // trajectory holding token t_begin: the largest i in [1, n_traj) with
+  // offsets[i] <= t_begin, else 0.  A 32-way search: the lanes probe 32 points of
+  // [lo, hi) at once and a ballot keeps the sub-range after the last probe that
+  // is <= t_begin (4 rounds for a million trajectories instead of 20 dependent
+  // loads).  Whatever the offsets hold, lo stays in [0, n_traj).
   int64_t lo = 0, hi = n_traj;
   while (hi - lo > 1) {
-    const int64_t mid = lo + (hi - lo) / 2;
-    if (offsets[mid] <= t_begin) lo = mid;
-    else hi = mid;
+    const int64_t span = hi - lo;
+    const int64_t q = lo + 1 + ((span - 1) * lane) / 32;  // in [lo + 1, hi - 1], nondecreasing
+    const unsigned bal = __ballot_sync(0xffffffffu, offsets[q] <= t_begin);
+    if (bal == 0u) {
+      hi = lo + 1;
+    } else {
+      const int j = 31 - __clz(bal);
+      const int64_t qj = lo + 1 + ((span - 1) * j) / 32;
+      hi = j < 31 ? lo + 1 + ((span - 1) * (j + 1)) / 32 : hi;
+      lo = qj;
+    }
   }
   int64_t cur = lo;
   int64_t cur_end = offsets[cur + 1];
