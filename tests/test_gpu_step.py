@@ -1,9 +1,11 @@
 """One whole PACE step (score -> budget/select -> fused log-prob + loss) at
-the 7B-shaped single-turn workload, in exactly the launch configuration
-bench.py times: the selection must match the oracle id for id, sampled
-log-probs within 5e-3, and the fused loss must equal the standalone
-surrogate on the same log-probs (whose parity with the oracle is pinned in
-test_gpu_loss.py at these sizes)."""
+the full-size workloads (7B single-turn at occupancies 1.0 / 1.33 / 2.0 of
+capacity, multi-turn with tool segments at 1.0 / 2.5, the MoE head), in
+exactly the launch configuration bench.py times: the selection must match the
+oracle id for id, sampled log-probs within 5e-3, and the fused loss must equal
+the standalone surrogate on the same log-probs (whose parity with the oracle
+is pinned in test_gpu_loss.py at these sizes).  Then the occupancy EMA
+(Eq. 4) carried across steps."""
 import math
 
 import numpy as np
@@ -17,9 +19,10 @@ from paper_2609_36830_gb300 import pace, step, workloads
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("n_traj", [512, 768])
-def test_math7b_step(n_traj):
-    pool = workloads.make_pool("math7b", n_traj=n_traj)
+@pytest.mark.parametrize("name,n_traj", [("math7b", 384), ("math7b", 512), ("math7b", 768),
+                                         ("multiturn", 256), ("multiturn", 480), ("moe", 1024)])
+def test_full_size_step(name, n_traj):
+    pool = workloads.make_pool(name, n_traj=n_traj)
     rw = workloads.make_rows(pool)
     H, V = pool.spec.hidden, pool.spec.vocab
     hidden = workloads.bf16_normal_device((rw.n_rows, H), 1.0, pool.seed + 11)
@@ -59,7 +62,6 @@ def test_math7b_step(n_traj):
     assert float(st.loss.item()) == float(loss2.item())
     assert math.isfinite(float(st.loss.item()))
     assert st.rows_in_loss() == int(in_loss.sum())
-
 
 
 def test_ema_budget_carried_across_steps():
