@@ -38,9 +38,9 @@ WORKLOAD = "math7b"
 # DRAM bytes per unit from the committed ncu captures of the current kernels
 # (profiles/lmhead_lse_kernel_one_wave.md: 1.135 GB for one full round of 4864 rows, W read
 # once per round, so traffic grows with the rows processed; profiles/tag_reduce_kernel_sweep16k.md:
-# 223.1 MB for 54.93 M tags).  Set to None when a kernel changes until it is captured again.
+# 223.4 MB for 54.93 M tags).  Set to None when a kernel changes until it is captured again.
 LMHEAD_DRAM_BYTES_PER_ROW = 1.135e9 / 4864
-TAG_REDUCE_DRAM_BYTES_PER_TAG = 223.106e6 / 54929421
+TAG_REDUCE_DRAM_BYTES_PER_TAG = 223.412e6 / 54929421
 SWEEP_N = 1048576
 SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)
 METRIC = "accepted tokens/sec (logprob+loss) and % bf16 tensor peak; pool scoring traj/s + HBM GB/s"

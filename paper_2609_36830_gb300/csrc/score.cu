@@ -78,25 +78,47 @@ __device__ __forceinline__ void flush(LaneAcc& a, int64_t traj, unsigned long lo
   a.maxp1 = 0;
 }
 
+// The stream is integer-ALU heavy (a few operations per 4-byte tag), so the
+// common cases avoid per-element work: a tag is a policy tag below 2^26 exactly
+// when none of its bits 26..31 is set, so one OR over a group of tags decides
+// whether the whole group is (no tool tag -1, nothing negative or huge), and
+// then up to 32 of them fit a 32-bit sum; 3-input max (DPX) halves the max tree.
+__device__ __forceinline__ bool small_policy(int bits_or) {
+  return (static_cast<unsigned>(bits_or) >> 26) == 0u;
+}
+
 // Sum, count and max of a batch that lies inside one trajectory and holds only
-// policy tags below 2^26: then 32 tags fit a 32-bit sum.  Returns false (and
-// leaves acc untouched) when the batch needs the general per-element path.
+// policy tags below 2^26.  Returns false (and leaves acc untouched) when the
+// batch needs the per-group path.
 __device__ __forceinline__ bool acc_batch_fast(LaneAcc& a, const int4 (&v)[kTilesPerBatch]) {
-  int mx = v[0].x, mn = v[0].x;
+  int o = 0, mx = 0, s = 0;
 #pragma unroll
   for (int u = 0; u < kTilesPerBatch; ++u) {
-    mx = max(max(mx, v[u].x), max(v[u].y, max(v[u].z, v[u].w)));
-    mn = min(min(mn, v[u].x), min(v[u].y, min(v[u].z, v[u].w)));
+    o |= (v[u].x | v[u].y) | (v[u].z | v[u].w);
+    mx = __vimax3_s32(__vimax3_s32(mx, v[u].x, v[u].y), v[u].z, v[u].w);
+    s += (v[u].x + v[u].y) + (v[u].z + v[u].w);
   }
-  if (mn < 0 || mx >= (1 << 26)) return false;
-  int s = 0;
-#pragma unroll
-  for (int u = 0; u < kTilesPerBatch; ++u) s += (v[u].x + v[u].y) + (v[u].z + v[u].w);
+  if (!small_policy(o)) return false;
   a.sum += s;
   a.cnt += 4 * kTilesPerBatch;
   const unsigned mp1 = static_cast<unsigned>(mx) + 1u;
   a.maxp1 = mp1 > a.maxp1 ? mp1 : a.maxp1;
   return true;
+}
+
+// The four tags of one lane's int4, all inside the current trajectory.
+__device__ __forceinline__ void acc_group(LaneAcc& a, const int4& q) {
+  if (small_policy((q.x | q.y) | (q.z | q.w))) {
+    a.sum += (q.x + q.y) + (q.z + q.w);
+    a.cnt += 4u;
+    const unsigned mp1 = static_cast<unsigned>(__vimax3_s32(q.x, q.y, max(q.z, q.w))) + 1u;
+    a.maxp1 = mp1 > a.maxp1 ? mp1 : a.maxp1;
+  } else {
+    acc_elem(a, q.x, true);
+    acc_elem(a, q.y, true);
+    acc_elem(a, q.z, true);
+    acc_elem(a, q.w, true);
+  }
 }
 
 // Each warp owns a contiguous range of 1024-token batches of the flattened
@@ -183,23 +205,26 @@ __global__ void __launch_bounds__(kReduceThreads, 2)
         // whole batch inside one trajectory: no position tests
         if (!acc_batch_fast(acc, v)) {
 #pragma unroll
-          for (int u = 0; u < kTilesPerBatch; ++u) {
-            acc_elem(acc, v[u].x, true);
-            acc_elem(acc, v[u].y, true);
-            acc_elem(acc, v[u].z, true);
-            acc_elem(acc, v[u].w, true);
-          }
+          for (int u = 0; u < kTilesPerBatch; ++u) acc_group(acc, v[u]);
         }
       } else if (seg_hi > pos) {
-        // batch-relative bounds fit 32 bits
+        // batch-relative bounds fit 32 bits; they are the same in every lane, so
+        // whole 128-token tiles outside [lo_r, hi_r) are skipped and tiles inside
+        // it need no position tests
         const int lo_r = static_cast<int>(pos - bt0), hi_r = static_cast<int>(seg_hi - bt0);
 #pragma unroll
         for (int u = 0; u < kTilesPerBatch; ++u) {
-          const int t = u * kTileTokens + lane * 4;
-          acc_elem(acc, v[u].x, t + 0 >= lo_r && t + 0 < hi_r);
-          acc_elem(acc, v[u].y, t + 1 >= lo_r && t + 1 < hi_r);
-          acc_elem(acc, v[u].z, t + 2 >= lo_r && t + 2 < hi_r);
-          acc_elem(acc, v[u].w, t + 3 >= lo_r && t + 3 < hi_r);
+          const int t0 = u * kTileTokens;
+          if (t0 + kTileTokens <= lo_r || t0 >= hi_r) continue;
+          if (t0 >= lo_r && t0 + kTileTokens <= hi_r) {
+            acc_group(acc, v[u]);
+          } else {
+            const int t = t0 + lane * 4;
+            acc_elem(acc, v[u].x, t + 0 >= lo_r && t + 0 < hi_r);
+            acc_elem(acc, v[u].y, t + 1 >= lo_r && t + 1 < hi_r);
+            acc_elem(acc, v[u].z, t + 2 >= lo_r && t + 2 < hi_r);
+            acc_elem(acc, v[u].w, t + 3 >= lo_r && t + 3 < hi_r);
+          }
         }
       }
       if (cur_end > bt1) return true;  // trajectory continues into the next batch

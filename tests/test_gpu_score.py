@@ -103,9 +103,12 @@ def _mk(lens, rng, j=50, tool=0.0):
 
 
 @pytest.mark.parametrize("case", ["empty_traj", "ragged", "one_long", "tiny_many", "all_tool",
-                                  "single"])
+                                  "single", "huge_versions", "mixed_versions"])
 def test_edge_cases(case):
-    rng = np.random.default_rng(hash(case) % 1000)
+    """Pool shapes and tag ranges that take every path of the tag reduction: empty
+    trajectories, boundaries at and off batch edges, tool tags, and versions at and
+    above 2^26 (no 32-bit partial sums), alone and mixed with small ones."""
+    rng = np.random.default_rng(sum(map(ord, case)))
     if case == "empty_traj":
         lens = [0, 5, 0, 0, 130, 0, 1, 0]
     elif case == "ragged":
@@ -117,13 +120,24 @@ def test_edge_cases(case):
         lens = list(rng.integers(0, 4, size=40000))
     elif case == "all_tool":
         lens = [10, 20, 30, 40]
+    elif case in ("huge_versions", "mixed_versions"):
+        lens = list(rng.integers(1, 5000, size=64))
     else:
         lens = [1]
     lens = list(lens)
     while len(lens) % 4:
         lens.append(int(rng.integers(0, 9)))
     tool = 1.0 if case == "all_tool" else 0.2
-    tags, offsets, c, s_pre, j, window = _mk(lens, rng, tool=tool)
+    j = 2_000_000_000 if case in ("huge_versions", "mixed_versions") else 50
+    tags, offsets, c, s_pre, j, window = _mk(lens, rng, j=j, tool=tool)
+    if case == "huge_versions":  # every policy tag at or above 2^26
+        pol = tags >= 0
+        c = np.maximum(c, (1 << 26) + 1000).astype(np.int32)
+        tags[pol] = np.minimum(tags[pol] + (1 << 26), np.repeat(c, lens)[pol]).astype(np.int32)
+    elif case == "mixed_versions":  # alternate trajectories small (< 2^26) and large
+        small = np.repeat(np.arange(len(lens)) % 2 == 0, lens)
+        tags[small & (tags >= 0)] %= 1 << 20
+        c = np.where(np.arange(len(lens)) % 2 == 0, np.minimum(c, 1 << 20), c).astype(np.int32)
     for G in (1, 4):
         g = gpu_score(tags, offsets, c, s_pre, j, window, group_size=G, min_obs=10)
         o = oracle_score(tags, offsets, c, s_pre, j, window, group_size=G, min_obs=10)
