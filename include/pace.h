@@ -124,7 +124,9 @@ PACE_API pace_status pace_score_pool(const int32_t* tags, const int64_t* offsets
                             void* workspace, size_t workspace_bytes, int32_t* status_dev,
                             void* stream);
 
-/* Workspace bytes pace_score_pool needs for a pool of n_traj trajectories. */
+/* Workspace bytes pace_score_pool needs for a pool of n_traj trajectories and
+ * a window of window_len values (the per-trajectory accumulators, the sorted
+ * window and the table of F over every possible ECDF count). */
 PACE_API size_t pace_score_pool_workspace_size(int64_t n_traj, int64_t window_len);
 
 /* ------------------------------------------------------------------------ */

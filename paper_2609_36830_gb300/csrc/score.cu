@@ -5,10 +5,13 @@
 //                       bound): per trajectory the count T of policy tokens,
 //                       the exact integer sum of their tags and the largest
 //                       tag (+1, for the Lemma 1 premise check).
+//   window_prep_kernel  one block: sorts the prefix-score window W and
+//                       tabulates F = phi(count / |W|) (Eqs. 9-10) for every
+//                       possible count 0..|W| (F depends on s only through the count).
 //   score_finalize_kernel  one thread per trajectory: K_gen, K_wait, the ECDF
-//                       percentile q against the window (Eq. 9), F = phi(q)
-//                       (Eq. 10), the mode's score (Eqs. 7-8), and the mean of
-//                       each group of G in fixed left-to-right order.
+//                       count of s against the sorted window (binary search),
+//                       F from the table, the mode's score (Eqs. 7-8), and the
+//                       mean of each group of G in fixed left-to-right order.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -258,7 +261,8 @@ struct FinalizeArgs {
   const int64_t* offsets;
   const int32_t* c_version;
   const float* s_pre;
-  const float* window;
+  const float* window_sorted;   // ascending, window_len values
+  const double* f_table;        // F for counts 0..window_len
   const unsigned long long* sumv;
   const unsigned* cnt;
   const unsigned* maxp1;
@@ -291,6 +295,45 @@ __device__ __forceinline__ double sharpen(double q, int gamma) {
   return __ddiv_rn(a, __dadd_rn(a, b));
 }
 
+// Sorts the window ascending (bitonic, in shared memory, padded to a power of
+// two with +inf, which sorts last and is never read back) and tabulates
+// F[c] = phi_gamma(c / n) for c = 0..n.  NaN in the window is a data error.
+__global__ void __launch_bounds__(1024) window_prep_kernel(const float* __restrict__ window, int n,
+                                                           int gamma, float* __restrict__ sorted,
+                                                           double* __restrict__ f_table,
+                                                           int32_t* status) {
+  __shared__ float sw[kMaxWindow];
+  int np2 = 1;
+  while (np2 < n) np2 <<= 1;
+  for (int k = threadIdx.x; k < np2; k += blockDim.x) {
+    float w = k < n ? window[k] : __int_as_float(0x7f800000);
+    if (isnan(w)) {
+      report(status, PACE_ERR_NAN_INPUT);
+      w = __int_as_float(0x7f800000);
+    }
+    sw[k] = w;
+  }
+  for (int size = 2; size <= np2; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      __syncthreads();
+      for (int k = threadIdx.x; k < np2; k += blockDim.x) {
+        const int partner = k ^ stride;
+        if (partner > k) {
+          const float a = sw[k], b = sw[partner];
+          if ((a > b) == ((k & size) == 0)) {
+            sw[k] = b;
+            sw[partner] = a;
+          }
+        }
+      }
+    }
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < n; k += blockDim.x) sorted[k] = sw[k];
+  for (int c = threadIdx.x; c <= n; c += blockDim.x)
+    f_table[c] = sharpen(__ddiv_rn(static_cast<double>(c), static_cast<double>(n)), gamma);
+}
+
 __global__ void score_finalize_kernel(FinalizeArgs p) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int wpad = (p.window_len + 3) & ~3;
@@ -298,11 +341,7 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
   double* sscore = reinterpret_cast<double*>(smem_raw + align_up(wpad * sizeof(float), 16));
 
   if (p.window_ready) {
-    for (int k = threadIdx.x; k < wpad; k += blockDim.x) {
-      const float w = k < p.window_len ? p.window[k] : __int_as_float(0x7fc00000);  // NaN pad
-      swin[k] = w;
-      if (k < p.window_len && isnan(w)) report(p.status, PACE_ERR_NAN_INPUT);
-    }
+    for (int k = threadIdx.x; k < p.window_len; k += blockDim.x) swin[k] = p.window_sorted[k];
   }
   __syncthreads();
 
@@ -333,14 +372,15 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
       if (isnan(s)) {
         f = p.f_missing;
       } else {
-        int count = 0;
-        const float4* w4 = reinterpret_cast<const float4*>(swin);
-        for (int k = 0; k < wpad / 4; ++k) {
-          const float4 w = w4[k];
-          count += (w.x <= s) + (w.y <= s) + (w.z <= s) + (w.w <= s);
+        // count of window values <= s: the first index of the sorted window
+        // holding a value > s
+        int lo = 0, hi = p.window_len;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (swin[mid] <= s) lo = mid + 1;
+          else hi = mid;
         }
-        const double q = __ddiv_rn(static_cast<double>(count), static_cast<double>(p.window_len));
-        f = sharpen(q, p.gamma);
+        f = p.f_table[lo];
       }
     }
     double sc;
@@ -391,6 +431,18 @@ struct ScoreWs {
   unsigned* cnt;
   unsigned* maxp1;
 };
+
+struct WindowWs {
+  float* sorted;    // [window_len]
+  double* f_table;  // [window_len + 1]
+};
+
+WindowWs carve_window_ws(Carver& cv, int64_t window_len) {
+  WindowWs w;
+  w.sorted = cv.take<float>(static_cast<size_t>(window_len > 0 ? window_len : 1));
+  w.f_table = cv.take<double>(static_cast<size_t>(window_len + 1));
+  return w;
+}
 
 ScoreWs carve_score_ws(Carver& cv, int64_t n_traj) {
   ScoreWs w;
@@ -462,10 +514,10 @@ extern "C" void pace_score_params_default(PaceScoreParams* p) {
 }
 
 extern "C" size_t pace_score_pool_workspace_size(int64_t n_traj, int64_t window_len) {
-  (void)window_len;
-  if (n_traj < 0) return 0;
+  if (n_traj < 0 || window_len < 0) return 0;
   Carver cv;
   carve_score_ws(cv, n_traj);
+  carve_window_ws(cv, window_len);
   return cv.used;
 }
 
@@ -495,15 +547,23 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
   Carver cv(workspace, workspace_bytes);
   ScoreWs ws = carve_score_ws(cv, n_traj);
+  WindowWs wws = carve_window_ws(cv, window_len);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
 
   cudaStream_t st = as_stream(stream);
   PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, st));
+  const bool window_ready = window_len > 0 && window_len >= params->min_obs;
+  if (window_ready) {
+    window_prep_kernel<<<1, 1024, 0, st>>>(window, static_cast<int>(window_len), params->gamma,
+                                          wws.sorted, wws.f_table, status_dev);
+    PACE_TRY(last_launch_status());
+  }
   FinalizeArgs a;
   a.offsets = offsets;
   a.c_version = c_version;
   a.s_pre = s_pre;
-  a.window = window;
+  a.window_sorted = wws.sorted;
+  a.f_table = wws.f_table;
   a.sumv = ws.sumv;
   a.cnt = ws.cnt;
   a.maxp1 = ws.maxp1;
@@ -511,7 +571,7 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   a.n_tokens = n_tokens;
   a.j = trainer_version;
   a.window_len = static_cast<int32_t>(window_len);
-  a.window_ready = (window_len > 0 && window_len >= params->min_obs) ? 1 : 0;
+  a.window_ready = window_ready ? 1 : 0;
   a.mode = params->mode;
   a.gamma = params->gamma;
   a.group_size = G;

@@ -157,6 +157,33 @@ def test_window_below_min_obs_and_no_window():
     _check(g, o, "no window")
 
 
+@pytest.mark.parametrize("wlen", [1, 7, 32, 512, 513, 1000, 4096])
+@pytest.mark.parametrize("gamma", [1, 2, 4, 7])
+def test_window_shapes_and_ties(wlen, gamma):
+    """The ECDF count of Eq. 9 against windows of every size up to the 4096
+    maximum, heavy ties, +0 and -0, +inf, and s exactly on window values; F of
+    Eq. 10 for several gamma.  Bits must match the oracle."""
+    rng = np.random.default_rng(wlen * 10 + gamma)
+    window = (np.round(rng.random(wlen) * 8) / 8).astype(np.float32)  # ties
+    window[rng.random(wlen) < 0.05] = -0.0
+    window[rng.random(wlen) < 0.02] = np.inf
+    lens = list(rng.integers(1, 40, size=256))
+    tags, offsets, c, s_pre, j, _ = _mk(lens, rng)
+    pick = rng.random(len(lens))
+    s_pre = np.where(pick < 0.4, rng.choice(window, size=len(lens)),  # exactly on window values
+                     np.where(pick < 0.5, np.float32(0.0),
+                              np.where(pick < 0.55, np.float32(np.inf),
+                                       np.where(pick < 0.6, np.nan,
+                                                rng.random(len(lens)) * 1.2 - 0.1)))).astype(
+        np.float32)
+    for mode in ("eff", "gen"):
+        g = gpu_score(tags, offsets, c, s_pre, j, window, mode=mode, gamma=gamma, min_obs=1,
+                      group_size=4)
+        o = oracle_score(tags, offsets, c, s_pre, j, window, mode=mode, gamma=gamma, min_obs=1,
+                         group_size=4)
+        _check(g, o, f"w{wlen}/g{gamma}/{mode}")
+
+
 def test_empty_pool():
     out = gpu_score(np.zeros(0, np.int32), np.zeros(1, np.int64), np.zeros(0, np.int32),
                     np.zeros(0, np.float32), 5, np.ones(4, np.float32), group_size=1)
