@@ -201,8 +201,79 @@ def _sweep_scoring(steps, warmup, device, n_traj=SWEEP_N):
                                   if TAG_REDUCE_DRAM_BYTES_PER_TAG else None),
            "ms_per_call": s_ms, "tag_reduce_ms": k_ms,
            "tag_reduce_gbs": k_bytes / (k_ms / 1e3) / 1e9, "tag_reduce_bytes": k_bytes}
+    if n_traj == SWEEP_N:
+        res["admission_variants"] = _admission_variants(pool, tok, out, sel, status, flush,
+                                                        steps, warmup, device)
     del pool, flush
     torch.cuda.empty_cache()
+    return res
+
+
+def _timed(fn, steps, warmup, flush=None):
+    """Mean CUDA-event time (ms) of fn() over `steps` calls after `warmup`, L2 flushed
+    before each timed call when a flush is given."""
+    import torch
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(steps)]
+    for b, e in evs:
+        if flush is not None:
+            flush()
+        b.record()
+        fn()
+        e.record()
+    torch.cuda.synchronize()
+    return statistics.mean(b.elapsed_time(e) for b, e in evs)
+
+
+def _admission_variants(pool, tok, out, sel, status, flush, steps, warmup, device):
+    """The two alternative admission rules and the diagnostics on the 1M sweep pool:
+    Stale-k (tag stream + one pass over trajectories, HBM), the retained-vs-rejected
+    staleness histogram (one pass over 1M values), and the literal sliding-window
+    quantile rule (one block: sort a 512-score window, decide candidates in draw
+    order; latency-bound by design) for one step's 64 prompt groups and for 16,384."""
+    import torch
+    from paper_2609_36830_gb300 import pace
+    n = pool.n_traj
+    L = pace.lib()
+    kbar = torch.empty(n, dtype=torch.float64, device=device)
+    adm = torch.empty(n, dtype=torch.uint8, device=device)
+    ws = pace.workspace(L.pace_stale_k_workspace_size(n), device)
+    k_ms = _timed(lambda: pace.stale_k(pool.tags, pool.offsets, pool.trainer_version, 8.0,
+                                       kbar=kbar, admitted=adm, ws=ws, status=status),
+                  steps, warmup, flush)
+    k_bytes = 4 * tok + 8 * (n + 1) + 16 * n + 9 * n
+    hist = torch.empty(2 * 64, dtype=torch.int32, device=device)
+    h_ms = _timed(lambda: pace.staleness_histogram(out["kgen"], sel["flags"], 0.0, 32.0, 64,
+                                                   hist=hist, status=status),
+                  steps, warmup, flush)
+    h_bytes = 9 * n
+    res = {"stale_k": {"workload": f"{n} trajectories, {tok} tags, k = 8",
+                       "ms_per_call": k_ms, "traj_per_s": n / (k_ms / 1e3),
+                       "gbs": k_bytes / (k_ms / 1e3) / 1e9},
+           "staleness_histogram": {"workload": f"K_gen of {n} trajectories, 64 bins, "
+                                               "retained / rejected",
+                                   "ms_per_call": h_ms, "values_per_s": n / (h_ms / 1e3),
+                                   "gbs": h_bytes / (h_ms / 1e3) / 1e9}}
+    qa = {}
+    for n_cand in (64, 16384):
+        cand = out["unit_score"][:n_cand].contiguous()
+        win = pace.ScoreWindow(512, device)
+        dec = torch.empty(n_cand, dtype=torch.uint8, device=device)
+        kap = torch.empty(1, dtype=torch.float64, device=device)
+        pace.quantile_admit(out["unit_score"][-512:].contiguous(), 0.0, 512, win, min_obs=32,
+                            decision=torch.empty(512, dtype=torch.uint8, device=device),
+                            kappa=kap, status=status)  # fill the window
+        q_ms = _timed(lambda: pace.quantile_admit(cand, 0.25, n_cand * 3 // 4, win, min_obs=32,
+                                                  decision=dec, kappa=kap, status=status),
+                      steps, warmup)
+        qa[str(n_cand)] = {"ms_per_call": q_ms, "units_per_s": n_cand / (q_ms / 1e3)}
+    res["quantile_admit"] = {"workload": "window of 512 unit scores, r = 0.25, draw until 3/4 "
+                                         "of the candidates are retained", "candidates": qa}
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0, pace.status_string(int(status.item()))
     return res
 
 

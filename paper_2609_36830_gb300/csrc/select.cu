@@ -49,6 +49,21 @@ struct SelectState {
   int pad;
 };
 
+// Start state of the radix select (nothing fixed yet, k units left to reject) and
+// a cleared histogram.  A kernel rather than a host copy, so the call stays valid
+// inside a captured CUDA graph (a captured copy would re-read host memory that
+// no longer holds the values at replay).
+__global__ void select_init_kernel(SelectState* state, long long k, unsigned* hist) {
+  if (threadIdx.x == 0) {
+    state->prefix = 0ull;
+    state->mask = 0ull;
+    state->k_rem = k;
+    state->done = 0;
+    state->pad = 0;
+  }
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = 0u;
+}
+
 __device__ __forceinline__ void write_unit(int64_t u, bool rejected, int64_t rej_pos,
                                            int64_t acc_pos, int G, int32_t* accepted_ids,
                                            int32_t* rejected_ids, uint8_t* flags) {
@@ -370,9 +385,8 @@ extern "C" pace_status pace_select_k(const double* unit_score, int64_t n_units, 
   Carver cv(workspace, workspace_bytes);
   SelectWs ws = carve_select_ws(cv, n_units);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
-  SelectState init{0ull, 0ull, static_cast<long long>(k), 0, 0};
-  PACE_TRY_CUDA(cudaMemcpyAsync(ws.state, &init, sizeof(init), cudaMemcpyHostToDevice, st));
-  PACE_TRY_CUDA(cudaMemsetAsync(ws.hist, 0, kHistBins * sizeof(unsigned), st));
+  select_init_kernel<<<1, 256, 0, st>>>(ws.state, static_cast<long long>(k), ws.hist);
+  PACE_TRY(last_launch_status());
   const int hist_grid = grid_for(n_units, 256, 2);
   for (int pass = 0; pass < kPasses; ++pass) {
     radix_hist_kernel<<<hist_grid, 256, 0, st>>>(unit_score, n_units, pass, ws.state, ws.hist,
