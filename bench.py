@@ -21,6 +21,7 @@ sample of the same workload (rank 0 only).
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import math
 import os
@@ -492,7 +493,7 @@ def _workload_name():
 def run_gpu(args):
     import torch
     import torch.distributed as dist
-    from paper_2609_36830_gb300 import pace
+    from paper_2609_36830_gb300 import pace, step
     ws, rank, local = _dist()
     if ws > 1:
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
@@ -542,9 +543,10 @@ def run_gpu(args):
 
     # End to end through the same C ABI with host buffers: every step's inputs are
     # copied from pinned host memory and its log-probs and loss copied back.  The
-    # copy of step i+1's inputs (on a copy stream, into a device staging set)
-    # overlaps step i's compute; a device-to-device move then hands them to the
-    # step, as a trainer that prefetches its next batch would do.
+    # copy of step i+1's inputs (on a copy stream) overlaps step i's compute.  The
+    # step alternates between two device input sets, each with its own step
+    # driver, as a trainer that prefetches its next batch would do: the copy
+    # into a set waits only for the step that last read it.
     names = ("tags", "offsets", "c_version", "s_pre", "window", "row_offsets", "mask",
              "targets", "behav_lp", "reward", "hidden", "w_vocab")
     host = {}
@@ -553,7 +555,9 @@ def run_gpu(args):
         h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
         h.copy_(t)
         host[name] = h
-    stage = {name: torch.empty_like(getattr(x, name)) for name in names}
+    x2 = dataclasses.replace(x, **{name: torch.empty_like(getattr(x, name)) for name in names})
+    st2 = step.PaceStep(x2, loss_params=st.lp_params, device=device)
+    sets = [(x, st), (x2, st2)]
     h2d = sum(h.numel() * h.element_size() for h in host.values())
     lp_host = torch.empty(x.mask.numel(), dtype=torch.float32, pin_memory=True)
     loss_host = torch.empty(1, dtype=torch.float64, pin_memory=True)
@@ -562,14 +566,15 @@ def run_gpu(args):
     copy_stream = torch.cuda.Stream(device=device)
     comp = torch.cuda.current_stream(device)
     staged = [torch.cuda.Event() for _ in range(e_steps)]
-    consumed = [torch.cuda.Event() for _ in range(e_steps)]
+    done = [torch.cuda.Event() for _ in range(e_steps)]
 
     def h2d_copy(i):
+        xi = sets[i % 2][0]
         with torch.cuda.stream(copy_stream):
-            if i > 0:
-                copy_stream.wait_event(consumed[i - 1])  # staging set free again
+            if i >= 2:
+                copy_stream.wait_event(done[i - 2])  # the last step that read this set
             for name in names:
-                stage[name].copy_(host[name], non_blocking=True)
+                getattr(xi, name).copy_(host[name], non_blocking=True)
             staged[i].record(copy_stream)
 
     torch.cuda.synchronize()
@@ -578,20 +583,20 @@ def run_gpu(args):
     e_b.record()
     h2d_copy(0)
     for i in range(e_steps):
+        sti = sets[i % 2][1]
         comp.wait_event(staged[i])
-        for name in names:
-            getattr(x, name).copy_(stage[name])
-        consumed[i].record(comp)
         if i + 1 < e_steps:
             h2d_copy(i + 1)
-        st.run()
-        lp_host.copy_(st.logprob, non_blocking=True)
-        loss_host.copy_(st.loss, non_blocking=True)
+        sti.run()
+        done[i].record(comp)
+        lp_host.copy_(sti.logprob, non_blocking=True)
+        loss_host.copy_(sti.loss, non_blocking=True)
     e_e.record()
     torch.cuda.synchronize()
+    assert int(st2.status.item()) == 0, pace.status_string(int(st2.status.item()))
     e_ms = e_b.elapsed_time(e_e) / e_steps
     _, e_ms = replicas.job_totals(M, e_ms, device)
-    del host, stage
+    del host, x2, st2, sets
 
     sweep = None
     if not args.no_sweep and rank == 0:

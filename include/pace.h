@@ -187,7 +187,7 @@ PACE_API size_t pace_select_workspace_size(int64_t n_units);
  * a plugin running inside a host framework whose memory pool owns all device
  * memory, or a latency-critical loop where an allocation could synchronise
  * the device.  Such a caller still passes its inputs and outputs; the scratch
- * the radix path needs comes from a fixed array of 32 KB inside the library,
+ * the radix path needs comes from a fixed array of 128 KB inside the library,
  * which every GPU that loads the library keeps until the process exits.
  *   - n_units must be at most 2^20 (1,048,576); larger pools get
  *     PACE_ERR_UNSUPPORTED_SHAPE and nothing is launched.

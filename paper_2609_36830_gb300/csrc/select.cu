@@ -26,7 +26,7 @@ namespace {
 constexpr int kSmallMax = 512;
 constexpr int kSmallThreads = 512;
 constexpr int kHistBins = 2048;
-constexpr int kTile = 2048;  // units per compaction block
+constexpr int kTile = 256;  // units per compaction block (enough blocks to fill the GPU at 16k units)
 constexpr int kTileThreads = 256;
 constexpr int kPerThread = kTile / kTileThreads;
 constexpr int kPasses = 6;
@@ -49,19 +49,59 @@ struct SelectState {
   int pad;
 };
 
-// Start state of the radix select (nothing fixed yet, k units left to reject) and
-// a cleared histogram.  A kernel rather than a host copy, so the call stays valid
-// inside a captured CUDA graph (a captured copy would re-read host memory that
-// no longer holds the values at replay).
-__global__ void select_init_kernel(SelectState* state, long long k, unsigned* hist) {
+// Start state of the radix select (nothing fixed yet, k units left to reject) in
+// state slot 0 and a cleared first histogram.  A kernel rather than a host copy,
+// so the call stays valid inside a captured CUDA graph (a captured copy would
+// re-read host memory that no longer holds the values at replay).
+__global__ void select_init_kernel(SelectState* states, long long k, unsigned* hist0) {
   if (threadIdx.x == 0) {
-    state->prefix = 0ull;
-    state->mask = 0ull;
-    state->k_rem = k;
-    state->done = 0;
-    state->pad = 0;
+    states[0].prefix = 0ull;
+    states[0].mask = 0ull;
+    states[0].k_rem = k;
+    states[0].done = 0;
+    states[0].pad = 0;
   }
-  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist[b] = 0u;
+  for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) hist0[b] = 0u;
+}
+
+// The radix step of one pass, computed identically by every block that needs
+// it: in the histogram of the keys matching st's prefix, find the digit holding
+// the k_rem-th largest of them, and narrow st to it.  Thread t (of 256) owns the
+// eight digits below nbins - 8t, so an exclusive scan in thread order counts the
+// keys with larger digits.  Every thread of the block must call it; st is the
+// same in every thread before and after.
+__device__ void block_pick(const unsigned* __restrict__ hist, int pass, SelectState& st) {
+  __shared__ int s_digit;
+  __shared__ long long s_left;
+  const int shift = c_shift[pass];
+  const int nbins = 1 << c_width[pass];
+  const int top = nbins - 1 - 8 * static_cast<int>(threadIdx.x);
+  long long h[8];
+  long long mine = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    h[i] = top - i >= 0 ? hist[top - i] : 0;
+    mine += h[i];
+  }
+  if (threadIdx.x == 0) s_digit = -1;
+  long long run = block_exclusive_scan<long long>(mine, nullptr);  // has a barrier after s_digit
+  const long long k_rem = st.k_rem;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    if (top - i >= 0 && run < k_rem && k_rem <= run + h[i]) {  // exactly one thread and digit
+      s_digit = top - i;
+      s_left = k_rem - run;
+    }
+    run += h[i];
+  }
+  __syncthreads();
+  const int digit = s_digit;
+  if (digit >= 0) {
+    st.prefix |= static_cast<unsigned long long>(digit) << shift;
+    st.mask |= static_cast<unsigned long long>(nbins - 1) << shift;
+    st.k_rem = s_left;
+  }
+  __syncthreads();  // s_digit and s_left may be rewritten by the next call
 }
 
 __device__ __forceinline__ void write_unit(int64_t u, bool rejected, int64_t rej_pos,
@@ -107,13 +147,29 @@ __global__ void __launch_bounds__(kSmallThreads)
     write_unit(u, rejected, rej_before, u - rej_before, G, accepted_ids, rejected_ids, flags);
 }
 
-__global__ void radix_hist_kernel(const double* __restrict__ score, int64_t n_units, int pass,
-                                  const SelectState* __restrict__ state,
-                                  unsigned* __restrict__ hist, int32_t* status) {
+// Pass `pass` of the MSB-first radix select (256 threads per block).  The state
+// it filters with is the previous pass's result, which every block derives
+// from the previous histogram (block 0 stores it for the next pass), so the
+// passes need no separate pick launches.  Histograms rotate through three
+// buffers: pass p adds into hist[p % 3], reads hist[(p - 1) % 3] and clears
+// hist[(p + 1) % 3] (last read by pass p - 1) for pass p + 1.  State slots
+// alternate: pass p reads slot (p - 1) & 1 and writes slot p & 1.
+__global__ void __launch_bounds__(256)
+    radix_pass_kernel(const double* __restrict__ score, int64_t n_units, int pass,
+                      SelectState* states, unsigned* hist3, int32_t* status) {
   __shared__ unsigned h[kHistBins];
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) h[b] = 0;
+  SelectState st = states[pass == 0 ? 0 : (pass - 1) & 1];
+  if (pass > 0) {
+    block_pick(hist3 + ((pass - 1) % 3) * kHistBins, pass - 1, st);
+    if (blockIdx.x == 0 && threadIdx.x == 0) states[pass & 1] = st;
+  }
+  unsigned* clear = hist3 + ((pass + 1) % 3) * kHistBins;
+  for (int64_t b = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < kHistBins;
+       b += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    clear[b] = 0u;
   __syncthreads();
-  const unsigned long long prefix = state->prefix, mask = state->mask;
+  const unsigned long long prefix = st.prefix, mask = st.mask;
   const int shift = c_shift[pass];
   const unsigned dmask = (1u << c_width[pass]) - 1u;
   for (int64_t u = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; u < n_units;
@@ -124,50 +180,21 @@ __global__ void radix_hist_kernel(const double* __restrict__ score, int64_t n_un
     if ((key & mask) == prefix) atomicAdd(&h[(key >> shift) & dmask], 1u);
   }
   __syncthreads();
+  unsigned* out = hist3 + (pass % 3) * kHistBins;
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x)
-    if (h[b]) atomicAdd(&hist[b], h[b]);
+    if (h[b]) atomicAdd(&out[b], h[b]);
 }
 
-// One block of 1024 threads: find the digit holding the k_rem-th largest key
-// among those matching the prefix, narrow the prefix, clear the histogram.
-// Thread t owns digits nbins-1-2t and nbins-2-2t, so an exclusive scan in
-// thread order counts the matching keys with larger digits.
-__global__ void __launch_bounds__(1024) radix_pick_kernel(int pass, SelectState* state,
-                                                          unsigned* hist) {
-  __shared__ long long s_krem;
-  const int shift = c_shift[pass];
-  const int nbins = 1 << c_width[pass];
-  const int d1 = nbins - 1 - 2 * static_cast<int>(threadIdx.x);
-  const int d2 = d1 - 1;
-  const long long h1 = d1 >= 0 ? hist[d1] : 0;
-  const long long h2 = d2 >= 0 ? hist[d2] : 0;
-  if (threadIdx.x == 0) s_krem = state->k_rem;
-  __syncthreads();
-  const long long k_rem = s_krem;
-  const long long above = block_exclusive_scan<long long>(h1 + h2, nullptr);
-  int digit = -1;
-  long long left = 0;
-  if (d1 >= 0 && above < k_rem && k_rem <= above + h1) {
-    digit = d1;
-    left = k_rem - above;
-  } else if (d2 >= 0 && above + h1 < k_rem && k_rem <= above + h1 + h2) {
-    digit = d2;
-    left = k_rem - above - h1;
-  }
-  if (digit >= 0) {  // exactly one thread
-    state->prefix |= static_cast<unsigned long long>(digit) << shift;
-    state->mask |= static_cast<unsigned long long>(nbins - 1) << shift;
-    state->k_rem = left;
-  }
-  if (d1 >= 0) hist[d1] = 0;
-  if (d2 >= 0) hist[d2] = 0;
-}
-
-// Phase 1: per tile, units equal to the pivot and above it.
+// Phase 1: per tile, units equal to the pivot and above it.  The pivot is the
+// last pass's result, derived here from its histogram (block 0 stores it in
+// state slot kPasses & 1 for the later phases).
 __global__ void __launch_bounds__(kTileThreads)
-    count_tile_kernel(const double* __restrict__ score, int64_t n_units,
-                      const SelectState* __restrict__ state, int* eq_cnt, int* gt_cnt) {
-  const unsigned long long pivot = state->prefix;
+    count_tile_kernel(const double* __restrict__ score, int64_t n_units, SelectState* states,
+                      const unsigned* hist3, int* eq_cnt, int* gt_cnt) {
+  SelectState st = states[(kPasses - 1) & 1];
+  block_pick(hist3 + ((kPasses - 1) % 3) * kHistBins, kPasses - 1, st);
+  if (blockIdx.x == 0 && threadIdx.x == 0) states[kPasses & 1] = st;
+  const unsigned long long pivot = st.prefix;
   int eq = 0, gt = 0;
   const int64_t base = static_cast<int64_t>(blockIdx.x) * kTile + threadIdx.x * kPerThread;
   for (int i = 0; i < kPerThread; ++i) {
@@ -279,8 +306,8 @@ __global__ void nan_check_kernel(const double* __restrict__ score, int64_t n, in
 }
 
 struct SelectWs {
-  SelectState* state;
-  unsigned* hist;
+  SelectState* states;  // two slots, alternating between passes
+  unsigned* hist;       // three rotating histograms of kHistBins
   int* eq_cnt;
   int* gt_cnt;
   long long* eq_before;
@@ -290,8 +317,8 @@ struct SelectWs {
 SelectWs carve_select_ws(Carver& cv, int64_t n_units) {
   const int64_t n_tiles = (n_units + kTile - 1) / kTile;
   SelectWs w;
-  w.state = cv.take<SelectState>(1);
-  w.hist = cv.take<unsigned>(kHistBins);
+  w.states = cv.take<SelectState>(2);
+  w.hist = cv.take<unsigned>(3 * kHistBins);
   w.eq_cnt = cv.take<int>(n_tiles);
   w.gt_cnt = cv.take<int>(n_tiles);
   w.eq_before = cv.take<long long>(n_tiles);
@@ -385,25 +412,24 @@ extern "C" pace_status pace_select_k(const double* unit_score, int64_t n_units, 
   Carver cv(workspace, workspace_bytes);
   SelectWs ws = carve_select_ws(cv, n_units);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
-  select_init_kernel<<<1, 256, 0, st>>>(ws.state, static_cast<long long>(k), ws.hist);
+  select_init_kernel<<<1, 256, 0, st>>>(ws.states, static_cast<long long>(k), ws.hist);
   PACE_TRY(last_launch_status());
   const int hist_grid = grid_for(n_units, 256, 2);
   for (int pass = 0; pass < kPasses; ++pass) {
-    radix_hist_kernel<<<hist_grid, 256, 0, st>>>(unit_score, n_units, pass, ws.state, ws.hist,
+    radix_pass_kernel<<<hist_grid, 256, 0, st>>>(unit_score, n_units, pass, ws.states, ws.hist,
                                                  status_dev);
-    PACE_TRY(last_launch_status());
-    radix_pick_kernel<<<1, 1024, 0, st>>>(pass, ws.state, ws.hist);
     PACE_TRY(last_launch_status());
   }
   const int64_t n_tiles = (n_units + kTile - 1) / kTile;
+  const SelectState* final_state = ws.states + (kPasses & 1);
   count_tile_kernel<<<static_cast<unsigned>(n_tiles), kTileThreads, 0, st>>>(
-      unit_score, n_units, ws.state, ws.eq_cnt, ws.gt_cnt);
+      unit_score, n_units, ws.states, ws.hist, ws.eq_cnt, ws.gt_cnt);
   PACE_TRY(last_launch_status());
-  scan_tiles_kernel<<<1, 1024, 0, st>>>(static_cast<int>(n_tiles), ws.state, ws.eq_cnt,
+  scan_tiles_kernel<<<1, 1024, 0, st>>>(static_cast<int>(n_tiles), final_state, ws.eq_cnt,
                                         ws.gt_cnt, ws.eq_before, ws.rej_before);
   PACE_TRY(last_launch_status());
   write_tile_kernel<<<static_cast<unsigned>(n_tiles), kTileThreads, 0, st>>>(
-      unit_score, n_units, G, ws.state, ws.eq_before, ws.rej_before, accepted_ids, rejected_ids,
+      unit_score, n_units, G, final_state, ws.eq_before, ws.rej_before, accepted_ids, rejected_ids,
       traj_accepted);
   return last_launch_status();
 }
@@ -606,14 +632,14 @@ extern "C" pace_status pace_quantile_admit(const double* unit_score, int64_t n_c
 //
 // For callers that may not allocate device memory themselves, the radix path's
 // scratch lives in this file-scope array instead of a workspace.  Every GPU
-// that loads the library holds it (32 KB) until the process exits; every call
+// that loads the library holds it (128 KB) until the process exits; every call
 // on a device shares it, so calls that overlap on that device race.
 // ---------------------------------------------------------------------------
 
 namespace {
 
 constexpr int64_t kNoAllocMaxUnits = int64_t(1) << 20;
-constexpr size_t kNoAllocScratchBytes = 32768;
+constexpr size_t kNoAllocScratchBytes = 131072;
 
 }  // namespace
 

@@ -1,6 +1,6 @@
 """pace_select_k_noalloc: the selection entry point for callers that cannot
 allocate device memory (for example a plugin inside a framework whose memory
-pool owns all device memory).  Its scratch is a fixed 32 KB array inside the
+pool owns all device memory).  Its scratch is a fixed 128 KB array inside the
 library, so it must give exactly the ids of pace_select_k, which uses a
 caller-provided workspace, and keep doing so on back-to-back calls that reuse
 the shared array.  This file is collected last on purpose."""
