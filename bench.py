@@ -673,6 +673,42 @@ def run_case(args):
     peaks, _ = _peaks()
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(args.steps)]
+    if args.case == "step_tiny":
+        # the smallest workload (64 trajectories, H 256, V 2048): a step is a few
+        # tens of microseconds of kernels, so launch latency matters; time it
+        # eagerly and as one CUDA-graph replay
+        from paper_2609_36830_gb300 import step
+        pool = workloads.make_pool("tiny")
+        rows = workloads.make_rows(pool)
+        H, V = pool.spec.hidden, pool.spec.vocab
+        hidden = workloads.bf16_normal_device((rows.n_rows, H), 1.0, pool.seed + 11, device)
+        w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), pool.seed + 12, device)
+        behav = workloads.behaviour_logprob(rows, pool.trainer_version,
+                                            workloads.uniform_center(V), pool.seed)
+        x = step.build_inputs(pool, rows, hidden, w, behav, device=device)
+        st = step.PaceStep(x, loss_params=pace.loss_params(eps_low=0.2, eps_high=0.2),
+                           device=device)
+        M = None
+        res = {}
+        for mode in ("eager", "graph"):
+            fn = st.run if mode == "eager" else st.capture().replay
+            for _ in range(max(args.warmup, 3)):
+                fn()
+            torch.cuda.synchronize()
+            b, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            n_rep = max(args.steps, 100)
+            b.record()
+            for _ in range(n_rep):
+                fn()
+            e.record()
+            torch.cuda.synchronize()
+            res[mode] = b.elapsed_time(e) / n_rep * 1e3
+            M = st.rows_in_loss()
+        assert int(st.status.item()) == 0
+        print(json.dumps({"case": "step_tiny", "rows_in_loss": M, "us_per_step": res,
+                          "tokens_per_s": {k: M / (v / 1e6) for k, v in res.items()}}),
+              flush=True)
+        return
     if args.case == "lmhead":
         spec = workloads.SPECS[args.case_workload]
         H, V, rows = spec.hidden, spec.vocab, args.case_rows
@@ -764,7 +800,8 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=512)
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce"], default=None,
+    ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce", "step_tiny"],
+                    default=None,
                     help="time one kernel on a small case (profiler captures)")
     ap.add_argument("--case-rows", type=int, default=4864)
     ap.add_argument("--case-workload", default=WORKLOAD, choices=["math7b", "multiturn", "moe"])

@@ -109,6 +109,25 @@ class PaceStep:
         self.r_hat = r_hat
         return k, r_hat
 
+    def capture(self):
+        """One step recorded as a CUDA graph (torch.cuda.CUDAGraph) for replay on a
+        pool of fixed shape whose inputs are refreshed in place: every call of the
+        step is stream-ordered with no host synchronisation, so a replay re-runs the
+        whole step with one launch.  The budget k is host arithmetic and is frozen
+        at capture, so capture needs beta = 0 (with beta > 0 the occupancy EMA of
+        Eq. 4 would move k from step to step)."""
+        if self.beta != 0.0:
+            raise ValueError("capture needs beta = 0: the budget is frozen into the graph")
+        side = torch.cuda.Stream(device=self.dev)
+        side.wait_stream(torch.cuda.current_stream(self.dev))
+        with torch.cuda.stream(side):
+            self.run()  # one-time launch set-up outside the capture
+        torch.cuda.current_stream(self.dev).wait_stream(side)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.run()
+        return g
+
     def rows_in_loss(self) -> int:
         """Rows the step's LM head processed (host count, synchronising)."""
         flags = self.sel_out["flags"].to(torch.int64)

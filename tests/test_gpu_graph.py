@@ -83,7 +83,7 @@ def test_tiny_step_replay():
     torch.cuda.synchronize()
     lp_ref, loss_ref = st.logprob.clone(), st.loss.clone()
     flags_ref = st.sel_out["flags"].clone()
-    g = _capture(st.run)
+    g = st.capture()
     st.logprob.fill_(0)
     st.loss.fill_(0)
     st.sel_out["flags"].fill_(0)
@@ -94,3 +94,15 @@ def test_tiny_step_replay():
     assert torch.equal(st.logprob, lp_ref)
     assert float(st.loss.item()) == float(loss_ref.item())
     assert np.isfinite(float(st.loss.item()))
+
+
+def test_capture_refuses_a_moving_budget():
+    pool = workloads.make_pool("tiny")
+    rw = workloads.make_rows(pool)
+    H, V = pool.spec.hidden, pool.spec.vocab
+    hidden = workloads.bf16_normal_device((rw.n_rows, H), 1.0, 1)
+    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), 2)
+    behav = workloads.behaviour_logprob(rw, pool.trainer_version, workloads.uniform_center(V), 3)
+    st = step.PaceStep(step.build_inputs(pool, rw, hidden, w, behav), beta=0.5)
+    with pytest.raises(ValueError):
+        st.capture()
