@@ -5,13 +5,16 @@
 //                       bound): per trajectory the count T of policy tokens,
 //                       the exact integer sum of their tags and the largest
 //                       tag (+1, for the Lemma 1 premise check).
-//   window_prep_kernel  one block: sorts the prefix-score window W and
-//                       tabulates F = phi(count / |W|) (Eqs. 9-10) for every
-//                       possible count 0..|W| (F depends on s only through the count).
+//   window_prep_kernel  (pools of 32k trajectories and more) one block: sorts
+//                       the prefix-score window W and tabulates F = phi(count / |W|)
+//                       (Eqs. 9-10) for every possible count 0..|W| (F depends on
+//                       s only through the count).
 //   score_finalize_kernel  one thread per trajectory: K_gen, K_wait, the ECDF
-//                       count of s against the sorted window (binary search),
-//                       F from the table, the mode's score (Eqs. 7-8), and the
-//                       mean of each group of G in fixed left-to-right order.
+//                       count of s against the window (binary search in the
+//                       sorted window, or a direct count on small pools), F
+//                       (from the table, or computed), the mode's score
+//                       (Eqs. 7-8), and the mean of each group of G in fixed
+//                       left-to-right order.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -25,6 +28,7 @@ constexpr int kTileTokens = 128;     // one int4 per lane
 constexpr int kTilesPerBatch = 8;    // 1024 tokens (4 KB) per warp batch in flight
 constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
 constexpr int kMaxWindow = 4096;
+constexpr int64_t kTableMinTraj = 32768;  // pools from this size sort W and tabulate F
 
 __device__ __forceinline__ int4 ld_stream_v4(const int32_t* p) {
   int4 v;
@@ -261,8 +265,9 @@ struct FinalizeArgs {
   const int64_t* offsets;
   const int32_t* c_version;
   const float* s_pre;
-  const float* window_sorted;   // ascending, window_len values
-  const double* f_table;        // F for counts 0..window_len
+  const float* window;           // W as given (used when window_sorted is null)
+  const float* window_sorted;   // ascending, window_len values, or null
+  const double* f_table;        // F for counts 0..window_len (with window_sorted)
   const unsigned long long* sumv;
   const unsigned* cnt;
   const unsigned* maxp1;
@@ -340,8 +345,17 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
   float* swin = reinterpret_cast<float*>(smem_raw);
   double* sscore = reinterpret_cast<double*>(smem_raw + align_up(wpad * sizeof(float), 16));
 
+  const bool sorted = p.window_sorted != nullptr;
   if (p.window_ready) {
-    for (int k = threadIdx.x; k < p.window_len; k += blockDim.x) swin[k] = p.window_sorted[k];
+    if (sorted) {
+      for (int k = threadIdx.x; k < p.window_len; k += blockDim.x) swin[k] = p.window_sorted[k];
+    } else {  // raw window, NaN-padded to a multiple of 4 (NaN never counts as <= s)
+      for (int k = threadIdx.x; k < wpad; k += blockDim.x) {
+        const float w = k < p.window_len ? p.window[k] : __int_as_float(0x7fc00000);
+        swin[k] = w;
+        if (k < p.window_len && isnan(w)) report(p.status, PACE_ERR_NAN_INPUT);
+      }
+    }
   }
   __syncthreads();
 
@@ -372,15 +386,26 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
       if (isnan(s)) {
         f = p.f_missing;
       } else {
-        // count of window values <= s: the first index of the sorted window
-        // holding a value > s
-        int lo = 0, hi = p.window_len;
-        while (lo < hi) {
-          const int mid = (lo + hi) >> 1;
-          if (swin[mid] <= s) lo = mid + 1;
-          else hi = mid;
+        if (sorted) {
+          // count of window values <= s: the first index of the sorted window
+          // holding a value > s
+          int lo = 0, hi = p.window_len;
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (swin[mid] <= s) lo = mid + 1;
+            else hi = mid;
+          }
+          f = p.f_table[lo];
+        } else {  // small pools: count directly, F from the count
+          int count = 0;
+          const float4* w4 = reinterpret_cast<const float4*>(swin);
+          for (int k = 0; k < wpad / 4; ++k) {
+            const float4 w = w4[k];
+            count += (w.x <= s) + (w.y <= s) + (w.z <= s) + (w.w <= s);
+          }
+          f = sharpen(__ddiv_rn(static_cast<double>(count), static_cast<double>(p.window_len)),
+                      p.gamma);
         }
-        f = p.f_table[lo];
       }
     }
     double sc;
@@ -553,7 +578,10 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   cudaStream_t st = as_stream(stream);
   PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, st));
   const bool window_ready = window_len > 0 && window_len >= params->min_obs;
-  if (window_ready) {
+  // Sorting W and tabulating F is one extra launch that pays off only on large
+  // pools; smaller ones count against the raw window (the same bits either way).
+  const bool use_table = window_ready && n_traj >= kTableMinTraj;
+  if (use_table) {
     window_prep_kernel<<<1, 1024, 0, st>>>(window, static_cast<int>(window_len), params->gamma,
                                           wws.sorted, wws.f_table, status_dev);
     PACE_TRY(last_launch_status());
@@ -562,8 +590,9 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   a.offsets = offsets;
   a.c_version = c_version;
   a.s_pre = s_pre;
-  a.window_sorted = wws.sorted;
-  a.f_table = wws.f_table;
+  a.window = window;
+  a.window_sorted = use_table ? wws.sorted : nullptr;
+  a.f_table = use_table ? wws.f_table : nullptr;
   a.sumv = ws.sumv;
   a.cnt = ws.cnt;
   a.maxp1 = ws.maxp1;

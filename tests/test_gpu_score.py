@@ -88,6 +88,21 @@ def test_sweep_128k_full_and_1m_sampled():
     np.testing.assert_array_equal(g["score"], g["kwait"] + g["weight"] * g["kgen"])
 
 
+def _mk_fast(lens, rng, j=50):
+    """_mk without tool tags, vectorised for large pools: tags of trajectory i
+    uniform in [0, c_i], sorted within the trajectory."""
+    lens = np.asarray(lens, np.int64)
+    offsets = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    n = lens.size
+    c = rng.integers(0, j + 1, size=n).astype(np.int32)
+    owner = np.repeat(np.arange(n), lens)
+    tags = np.floor(rng.random(owner.size) * (c[owner].astype(np.float64) + 1)).astype(np.int32)
+    tags = tags[np.lexsort((tags, owner))]
+    s_pre = np.where(rng.random(n) < 0.5, rng.random(n), np.nan).astype(np.float32)
+    window = rng.random(100).astype(np.float32)
+    return tags, offsets, c, s_pre, j, window
+
+
 def _mk(lens, rng, j=50, tool=0.0):
     offsets = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
     n = len(lens)
@@ -157,18 +172,20 @@ def test_window_below_min_obs_and_no_window():
     _check(g, o, "no window")
 
 
+@pytest.mark.parametrize("n_traj", [256, 32768])  # direct count / sorted window + F table
 @pytest.mark.parametrize("wlen", [1, 7, 32, 512, 513, 1000, 4096])
 @pytest.mark.parametrize("gamma", [1, 2, 4, 7])
-def test_window_shapes_and_ties(wlen, gamma):
+def test_window_shapes_and_ties(n_traj, wlen, gamma):
     """The ECDF count of Eq. 9 against windows of every size up to the 4096
     maximum, heavy ties, +0 and -0, +inf, and s exactly on window values; F of
-    Eq. 10 for several gamma.  Bits must match the oracle."""
+    Eq. 10 for several gamma; on a small pool (counted directly) and a large one
+    (sorted window and a table of F).  Bits must match the oracle."""
     rng = np.random.default_rng(wlen * 10 + gamma)
     window = (np.round(rng.random(wlen) * 8) / 8).astype(np.float32)  # ties
     window[rng.random(wlen) < 0.05] = -0.0
     window[rng.random(wlen) < 0.02] = np.inf
-    lens = list(rng.integers(1, 40, size=256))
-    tags, offsets, c, s_pre, j, _ = _mk(lens, rng)
+    lens = rng.integers(1, 40, size=n_traj)
+    tags, offsets, c, s_pre, j, _ = _mk_fast(lens, rng)
     pick = rng.random(len(lens))
     s_pre = np.where(pick < 0.4, rng.choice(window, size=len(lens)),  # exactly on window values
                      np.where(pick < 0.5, np.float32(0.0),
