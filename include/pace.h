@@ -418,12 +418,12 @@ PACE_API size_t pace_surrogate_backward_workspace_size(int64_t n_rows, int64_t n
  *   grad_w[v]      = sum_r G_rv h_r         device float32 [V][H] (output)
  * over the rows in the loss (rows outside it get 0).  lse is the forward's
  * output for the same rows (device float32 [n_rows]).  Rows are processed in
- * chunks of up to 65,536: logits are recomputed on the tensor cores, G is held
+ * chunks of up to 32,768: logits are recomputed on the tensor cores, G is held
  * in bf16 in the workspace for the chunk (in 64-column blocks), then two
  * tensor-core GEMMs form G W and G^T H.  Chunks past the rows in the loss (a
  * count known only on the device) cost no tensor-core work.  Returns
  * PACE_ERR_UNSUPPORTED_SHAPE when ceil(V / 64) x the chunk's rows exceeds
- * 2^31 - 1 (V above about 2.1M at full chunks).  Other arguments and errors as
+ * 2^31 - 1 (V above about 4.2M at full chunks).  Other arguments and errors as
  * for pace_token_logprob. */
 PACE_API pace_status pace_token_logprob_backward(const PaceBatch* batch, const void* hidden,
                                                  const void* w_vocab, const int32_t* targets,

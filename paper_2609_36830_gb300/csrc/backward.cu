@@ -43,7 +43,7 @@ constexpr uint32_t kGStageB = GBN * GBK * 2;  // 32 KB
 constexpr uint32_t kGStageBytes = kGStageA + kGStageB;
 constexpr uint32_t kGTmemCols = 2 * GBN;
 constexpr size_t kGSmemBytes = 1024 + GSTAGES * kGStageBytes + 256;
-constexpr int64_t kChunkRows = 65536;         // rows of G held at once (bf16 M x V)
+constexpr int64_t kChunkRows = 32768;         // rows of G held at once (bf16 M x V)
 constexpr int kGroupM = 38;                   // M tiles per raster group
 
 enum { EPI_G = 0, EPI_ROWS = 1, EPI_ACC = 2 };

@@ -122,7 +122,7 @@ def test_full_size_backward_sampled_rows_and_identity():
 
 @pytest.mark.parametrize("rows,frac", [(135000, 0.3), (135000, 0.98)])
 def test_lmhead_backward_multi_chunk_trimmed(rows, frac):
-    """More rows than one 65,536-row chunk, with the rows in the loss ending inside
+    """More rows than four 32,768-row chunks, with the rows in the loss ending inside
     the first (frac 0.3: later chunks hold none) or inside the last chunk (0.98):
     the GEMMs cut their extent to the device-side count and dW must still be whole."""
     H, V = 64, 256
