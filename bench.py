@@ -36,11 +36,12 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOAD = "math7b"
-# DRAM bytes per unit from the committed ncu captures of the current kernels
-# (profiles/lmhead_lse_kernel_one_wave.md: 1.135 GB for one full round of 4864 rows, W read
-# once per round, so traffic grows with the rows processed; profiles/tag_reduce_kernel_sweep16k.md:
+# DRAM bytes per unit from the committed ncu captures of the current kernels, by the LM head's
+# vocabulary split count (profiles/lmhead_lse_kernel_one_wave.md: 4 splits, 1.130 GB for one
+# full round of 4864 rows, W read once per round, so traffic grows with the rows processed;
+# 2 splits, 18.87 GB for four rounds of 9728 rows; profiles/tag_reduce_kernel_sweep16k.md:
 # 223.4 MB for 54.93 M tags).  Set to None when a kernel changes until it is captured again.
-LMHEAD_DRAM_BYTES_PER_ROW = 1.135e9 / 4864
+LMHEAD_DRAM_BYTES_PER_ROW = {4: 1.12978e9 / 4864, 2: 18.8672e9 / 38912}
 TAG_REDUCE_DRAM_BYTES_PER_TAG = 223.412e6 / 54929421
 SWEEP_N = 1048576
 SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)
@@ -503,6 +504,8 @@ def run_gpu(args):
 
     pool, rows, x, st = _make_step(rank, device)
     H, V = x.hidden.shape[1], x.w_vocab.shape[0]
+    # the LM head's vocabulary split count, measured on this GPU (untimed)
+    splits, split_ms = st.tune_lmhead_splits()
     k_units = None
     for _ in range(args.warmup):
         k_units, _ = st.run()
@@ -638,7 +641,10 @@ def run_gpu(args):
                        "rows_in_loss_per_step": M, "rows_total": int(rows.n_rows),
                        "k_units_rejected": k_units,
                        "parallelism": f"{ws} independent pool replica(s), no collective",
-                       "l2": "inputs larger than L2 (hidden states 10.7 GB per step)"},
+                       "l2": "inputs larger than L2 (hidden states 10.7 GB per step)",
+                       "lmhead_splits": {"chosen": splits,
+                                         "tuning_ms_per_step": {str(k): v
+                                                                for k, v in split_ms.items()}}},
             "roofline": {"bound": "tensor", "kernel": "lmhead_lse_kernel", "achieved": achieved,
                          "peak": peak_s, "unit": "TFLOP/s", "frac": achieved / peak_s,
                          "peak_source": f"{peak_src} bf16_tflops_sustained",
@@ -646,8 +652,9 @@ def run_gpu(args):
                          "frac_of_nominal_2250": achieved / 2250.0,
                          "kernel_ms": lm_ms, "kernel_ms_each": lm_each,
                          "flops_per_launch": flops,
-                         "traffic": (LMHEAD_DRAM_BYTES_PER_ROW * M
-                                     if LMHEAD_DRAM_BYTES_PER_ROW else None),
+                         "traffic": (LMHEAD_DRAM_BYTES_PER_ROW[splits] * M
+                                     if LMHEAD_DRAM_BYTES_PER_ROW
+                                     and splits in LMHEAD_DRAM_BYTES_PER_ROW else None),
                          "traffic_note": "dram read+write bytes per launch, scaled by rows from "
                                          "the one-round ncu capture"},
             "cpu_baseline": cpu,
@@ -721,6 +728,7 @@ def run_case(args):
         lp = torch.empty(rows, dtype=torch.float32, device=device)
         ws = pace.workspace(pace.token_logprob_workspace_size(rows, 1, H, V), device)
         status = pace.new_status(device)
+        pace.set_lmhead_splits(args.case_splits)
         for i in range(args.warmup + args.steps):
             if i >= args.warmup:
                 pace.set_profile_events(pace.PROFILE_LMHEAD, *evs[i - args.warmup])
@@ -806,6 +814,8 @@ def main():
     ap.add_argument("--case-rows", type=int, default=4864)
     ap.add_argument("--case-workload", default=WORKLOAD, choices=["math7b", "multiturn", "moe"])
     ap.add_argument("--case-traj", type=int, default=16384)
+    ap.add_argument("--case-splits", type=int, default=0,
+                    help="LM-head vocabulary splits for --case lmhead (0 = automatic)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

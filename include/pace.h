@@ -447,6 +447,21 @@ typedef enum {
   PACE_PROFILE_TAG_REDUCE = 1  /* the tag-stream reduction of pace_score_pool */
 } pace_profile_kernel;
 
+/* Not part of the method: a tuning control for the fused LM head
+ * (pace_token_logprob, pace_prefix_score).  Its work items are (pair of
+ * 128-row blocks, vocabulary split); how many contiguous splits the
+ * vocabulary is cut into changes neither results beyond rounding order nor
+ * FLOPs, but it changes how many vocabulary streams are in flight at once and
+ * so the power, and on GB300 the power-capped clock, of a long launch, in a
+ * way that differs from GPU to GPU (2 or 4 splits, either may be 2-10 %
+ * faster).  From now on, in this process, batches with enough rows to give
+ * every resident cluster at least four items use `splits` (clamped to the
+ * number of 256-column vocabulary tiles); smaller batches and splits = 0 use
+ * the automatic choice (the first of 4, 2, 3, 6, 8 that keeps rounds of items
+ * at least 90 % full; 4 reads the vocabulary from HBM about once per round).
+ * Returns PACE_ERR_INVALID_ARG unless 0 <= splits <= 8. */
+PACE_API pace_status pace_set_lmhead_splits(int32_t splits);
+
 /* Not part of the method: a measurement aid.  From now on, on the calling
  * host thread, record the CUDA event `begin` (a cudaEvent_t) on the call's
  * stream immediately before each launch of the given kernel and `end`

@@ -32,6 +32,11 @@ uint64_t& launch_counter() {
   return n;
 }
 
+std::atomic<int>& lmhead_split_pref() {
+  static std::atomic<int> s{0};
+  return s;
+}
+
 namespace {
 
 // cuTensorMapEncodeTiled from the driver, looked up through the runtime so the
@@ -106,6 +111,12 @@ extern "C" pace_status pace_set_profile_events(int32_t kernel, void* begin, void
 }
 
 extern "C" uint64_t pace_kernel_launches(void) { return pace::launch_counter(); }
+
+extern "C" pace_status pace_set_lmhead_splits(int32_t splits) {
+  if (splits < 0 || splits > 8) return PACE_ERR_INVALID_ARG;
+  pace::lmhead_split_pref().store(splits);
+  return PACE_OK;
+}
 
 extern "C" const char* pace_status_string(pace_status status) {
   switch (status) {

@@ -19,6 +19,7 @@
 // A CTA covers 128 rows and one of S contiguous vocabulary splits; it writes
 // one (max, sum) pair per row and split.  Consecutive CTAs share a row block,
 // so the hidden tile they re-read stays in L2 while the vocabulary streams.
+// S is chosen on the device from the rows actually present (pick_splits).
 //
 // lse_merge_kernel: per row, merges the S partial pairs into the log-sum-exp
 //   and writes lp = z_y / tau - lse.
@@ -55,16 +56,55 @@ constexpr uint32_t kTmemCols = 2 * BN;          // two fp32 accumulators of 256 
 constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
 constexpr uint16_t kPairMask = 0x3;
 constexpr size_t kSmemBytes = 1024 /* alignment slack */ + STAGES * kStageBytes + 256;
+constexpr int kMaxSplits = 8;
+
+// Number of vocabulary splits S for row_pairs row pairs on n_clusters persistent
+// clusters.  With S = 4 the 19 clusters sweeping one split stay close enough
+// for L2 to serve each vocabulary tile to all of them: the vocabulary is read
+// from HBM about once per round of items.  With S = 2 the 38 clusters of a
+// split drift apart over its 545 MB and it is read ~4 times per round (18.9 GB
+// of DRAM reads for four 9,728-row rounds of the 7B head), yet on some GPUs the
+// power-capped clock still comes out 2-10 % higher, on others as much lower;
+// S = 1 is far slower.  Small batches need more splits to give
+// every cluster an item.  So: the first of 4, 2, 3, 6, 8 whose rounds of items
+// are at least 90 % full, else whichever fills its rounds best (the earlier on
+// ties); a preferred count (pace_set_lmhead_splits, from a measurement on this
+// GPU) replaces the choice when it still gives every cluster at least four
+// items.  Evaluated identically on the device by the LM head and the merge,
+// from the device-side row count.
+__host__ __device__ inline int pick_splits(int64_t row_pairs, int64_t n_clusters, int n_vtiles,
+                                           int pref) {
+  if (pref > 0) {
+    const int sp = pref < n_vtiles ? pref : (n_vtiles > 0 ? n_vtiles : 1);
+    if (row_pairs * sp >= 4 * n_clusters) return sp;
+  }
+  const int cand[5] = {4, 2, 3, 6, kMaxSplits};
+  int best = 1;
+  int64_t best_items = 0, best_rounds = 1;
+  for (int i = 0; i < 5; ++i) {
+    const int sp = cand[i] < n_vtiles ? cand[i] : (n_vtiles > 0 ? n_vtiles : 1);
+    const int64_t items = row_pairs * sp;
+    const int64_t rounds = (items + n_clusters - 1) / n_clusters;
+    if (items * 10 >= 9 * rounds * n_clusters) return sp;
+    if (best_items == 0 || items * best_rounds > best_items * rounds) {
+      best = sp;
+      best_items = items;
+      best_rounds = rounds;
+    }
+  }
+  return best;
+}
 
 struct LmArgs {
   int64_t rows_cap;             // rows of the A tensor map
   const long long* n_valid_dev; // rows actually present (device), or null = rows_cap
   int32_t H, V;
-  int32_t n_vtiles, splits, tiles_per_split;
+  int32_t n_vtiles;
+  int32_t split_pref;           // preferred vocabulary splits, 0 = automatic
   float scale_log2;             // log2(e) / temperature
   const int32_t* targets;
   const int32_t* rowidx;        // compact row -> original row, or null (identity)
-  float* part_m;                // [rows_cap * splits]
+  float* part_m;                // [rows_cap * kMaxSplits], row r's splits at r * S
   float* part_s;
   float* tgt_logit;             // [rows_cap]
   int32_t* status;
@@ -113,7 +153,9 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
   const int cid = static_cast<int>(blockIdx.x) / CLUSTER;
   const int64_t n_valid = p.n_valid_dev ? static_cast<int64_t>(*p.n_valid_dev) : p.rows_cap;
   const int64_t row_pairs = (n_valid + 2 * BM - 1) / (2 * BM);
-  const int64_t n_items = row_pairs * p.splits;
+  const int n_splits = pick_splits(row_pairs, n_clusters, p.n_vtiles, p.split_pref);
+  const int tiles_per_split = (p.n_vtiles + n_splits - 1) / n_splits;
+  const int64_t n_items = row_pairs * n_splits;
   // both CTAs of a cluster read the same n_valid and cid: the exit is uniform
   if (cid >= n_items) return;
   const int nkb = p.H / BK;
@@ -149,11 +191,11 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
       uint32_t it = 0;
       bool ok = true;
       for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
-        const int64_t rp = c.item / p.splits;
-        const int split = static_cast<int>(c.item % p.splits);
+        const int64_t rp = c.item / n_splits;
+        const int split = static_cast<int>(c.item % n_splits);
         const int32_t row0 = static_cast<int32_t>((rp * CLUSTER + crank) * BM);
-        const int tile0 = split * p.tiles_per_split;
-        const int tile1 = min(tile0 + p.tiles_per_split, p.n_vtiles);
+        const int tile0 = split * tiles_per_split;
+        const int tile1 = min(tile0 + tiles_per_split, p.n_vtiles);
         for (int t = tile0; t < tile1 && ok; ++t) {
           const int32_t nb = t * BN + static_cast<int32_t>(crank) * (BN / CLUSTER);
           for (int kb = 0; kb < nkb; ++kb, ++it) {
@@ -188,9 +230,9 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
       uint32_t it = 0, tcount = 0;
       bool ok = true;
       for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
-        const int split = static_cast<int>(c.item % p.splits);
-        const int tile0 = split * p.tiles_per_split;
-        const int tile1 = min(tile0 + p.tiles_per_split, p.n_vtiles);
+        const int split = static_cast<int>(c.item % n_splits);
+        const int tile0 = split * tiles_per_split;
+        const int tile1 = min(tile0 + tiles_per_split, p.n_vtiles);
         for (int t = tile0; t < tile1 && ok; ++t, ++tcount) {
           const uint32_t acc = tcount & 1u;
           const uint32_t acc_ph = (tcount >> 1) & 1u;
@@ -239,10 +281,10 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
     uint32_t tcount = 0;
     bool ok = true;
     for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
-      const int64_t rp = c.item / p.splits;
-      const int split = static_cast<int>(c.item % p.splits);
-      const int tile0 = split * p.tiles_per_split;
-      const int tile1 = min(tile0 + p.tiles_per_split, p.n_vtiles);
+      const int64_t rp = c.item / n_splits;
+      const int split = static_cast<int>(c.item % n_splits);
+      const int tile0 = split * tiles_per_split;
+      const int tile1 = min(tile0 + tiles_per_split, p.n_vtiles);
       const int64_t row = (rp * CLUSTER + crank) * BM + r_local;
       const bool row_ok = row < n_valid;
       int32_t y = -1;
@@ -296,7 +338,7 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
         mbar_arrive(&tmem_empty[acc]);
       }
       if (row_ok && ok) {
-        const int64_t o = row * p.splits + split;
+        const int64_t o = row * n_splits + split;
         p.part_m[o] = m;
         p.part_s[o] = s;
         if (have_tgt) p.tgt_logit[row] = tgt;
@@ -315,13 +357,17 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
 // Per row in the loss: log-sum-exp from the split partials, then
 // lp = z_y / tau - lse, scattered back to the original row.
 __global__ void lse_merge_kernel(int64_t rows_cap, const long long* __restrict__ n_valid_dev,
-                                 int splits, int32_t V, float inv_temp,
+                                 int lm_clusters, int n_vtiles, int split_pref, int32_t V,
+                                 float inv_temp,
                                  const float* __restrict__ part_m, const float* __restrict__ part_s,
                                  const float* __restrict__ tgt_logit,
                                  const int32_t* __restrict__ targets,
                                  const int32_t* __restrict__ rowidx, float* __restrict__ logprob,
                                  float* __restrict__ lse_out, int32_t* status) {
   const int64_t n_valid = n_valid_dev ? static_cast<int64_t>(*n_valid_dev) : rows_cap;
+  // the split count the LM head used for these rows
+  const int splits =
+      pick_splits((n_valid + 2 * BM - 1) / (2 * BM), lm_clusters, n_vtiles, split_pref);
   for (int64_t r = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; r < n_valid;
        r += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int64_t orig = rowidx ? static_cast<int64_t>(rowidx[r]) : r;
@@ -344,13 +390,6 @@ __global__ void lse_merge_kernel(int64_t rows_cap, const long long* __restrict__
 }
 
 // ---------------------------------------------------------------- host side
-
-int choose_splits(int n_vtiles) {
-  int s = 4;
-  if (s > n_vtiles) s = n_vtiles;
-  if (s < 1) s = 1;
-  return s;
-}
 
 struct LmLaunchInfo {
   int max_clusters = 0;
@@ -394,15 +433,13 @@ pace_status lm_launch_info(LmLaunchInfo* out) {
 
 void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, bool compact,
                  LmWs* w) {
-  const int n_vtiles = (V + BN - 1) / BN;
-  const int S = choose_splits(n_vtiles);
   const int64_t rows_cap = n_rows > BM ? n_rows : BM;
   carve_compact_ws(cv, n_seq, n_rows, &w->cw);
   carve_surrogate_ws(cv, n_seq, &w->sw);
   w->hidden_c = compact ? static_cast<void*>(cv.take<uint16_t>(static_cast<size_t>(rows_cap) * H))
                         : nullptr;
-  w->part_m = cv.take<float>(static_cast<size_t>(rows_cap) * S);
-  w->part_s = cv.take<float>(static_cast<size_t>(rows_cap) * S);
+  w->part_m = cv.take<float>(static_cast<size_t>(rows_cap) * kMaxSplits);
+  w->part_s = cv.take<float>(static_cast<size_t>(rows_cap) * kMaxSplits);
   w->tgt = cv.take<float>(static_cast<size_t>(rows_cap));
 }
 
@@ -448,8 +485,6 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   }
   if (n_rows == 0) return PACE_OK;
   const int n_vtiles = (V + BN - 1) / BN;
-  const int S = choose_splits(n_vtiles);
-  const int tps = (n_vtiles + S - 1) / S;
   CUtensorMap tm_a, tm_b;
   PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, H, BK, BM));
   PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, H, BK, BN / CLUSTER));
@@ -461,8 +496,7 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   a.H = H;
   a.V = V;
   a.n_vtiles = n_vtiles;
-  a.splits = S;
-  a.tiles_per_split = tps;
+  a.split_pref = lmhead_split_pref().load();
   a.scale_log2 = 1.4426950408889634f / temperature;
   a.targets = targets;
   a.rowidx = rowidx;
@@ -470,8 +504,9 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   a.part_s = ws.part_s;
   a.tgt_logit = ws.tgt;
   a.status = status_dev;
-  // persistent: at most one wave of 2-CTA clusters, never more clusters than items
-  const int64_t items = (rows_cap + 2 * BM - 1) / (2 * BM) * S;
+  // persistent: at most one wave of 2-CTA clusters, never more clusters than the
+  // most items the rows could make (the split count is chosen on the device)
+  const int64_t items = (rows_cap + 2 * BM - 1) / (2 * BM) * kMaxSplits;
   const int64_t clusters = items < li.max_clusters ? items : li.max_clusters;
   const int64_t grid = clusters * CLUSTER;
   const ProfileEvents& pe = profile_events(PACE_PROFILE_LMHEAD);
@@ -483,7 +518,9 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   const int64_t cap = static_cast<int64_t>(sm_count()) * 8;
   if (mblocks > cap) mblocks = cap;
   lse_merge_kernel<<<static_cast<unsigned>(mblocks), 256, 0, st>>>(
-      rows_cap, n_valid_dev, S, V, 1.0f / temperature, ws.part_m, ws.part_s, ws.tgt, targets,
+      rows_cap, n_valid_dev, static_cast<int>(clusters), n_vtiles, a.split_pref, V,
+      1.0f / temperature,
+      ws.part_m, ws.part_s, ws.tgt, targets,
       rowidx, logprob, lse, status_dev);
   return last_launch_status();
 }

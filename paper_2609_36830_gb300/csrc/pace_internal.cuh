@@ -4,6 +4,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "pace.h"
 
 #if defined(__CUDA_ARCH__) && (__CUDA_ARCH__ < 1000)
@@ -28,6 +30,10 @@ namespace pace {
 
 // Kernels launched by this library from the calling thread.
 uint64_t& launch_counter();
+
+// Vocabulary splits the LM head should use on large batches (0 = automatic),
+// set by pace_set_lmhead_splits for the whole process.
+std::atomic<int>& lmhead_split_pref();
 
 // Called right after every kernel launch: counts it and checks it started.
 inline pace_status last_launch_status() {

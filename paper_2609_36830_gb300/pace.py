@@ -96,6 +96,7 @@ SIGNATURES = {
                                      _P, _P], _I32),
     "pace_token_logprob_backward_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
     "pace_set_profile_events": ([_I32, _P, _P], _I32),
+    "pace_set_lmhead_splits": ([_I32], _I32),
     "pace_kernel_launches": ([], ctypes.c_uint64),
     "pace_wait_timeout_selftest": ([ctypes.c_uint64, _P, _P], _I32),
 }
@@ -336,6 +337,12 @@ def set_profile_events(kernel: int, begin=None, end=None):
         return ctypes.c_void_p(ev.cuda_event)
     b, e = handle(begin), handle(end)
     _check(lib().pace_set_profile_events(int(kernel), b, e), "pace_set_profile_events")
+
+
+def set_lmhead_splits(splits: int):
+    """pace_set_lmhead_splits: vocabulary splits of the LM head on large batches
+    (0 = automatic), for the whole process."""
+    _check(lib().pace_set_lmhead_splits(int(splits)), "pace_set_lmhead_splits")
 
 
 def kernel_launches() -> int:

@@ -109,6 +109,29 @@ class PaceStep:
         self.r_hat = r_hat
         return k, r_hat
 
+    def tune_lmhead_splits(self, candidates=(2, 4), reps=2):
+        """Time whole steps with each candidate vocabulary-split count of the LM head
+        (pace_set_lmhead_splits) on this GPU, alternating candidates ``reps`` times,
+        and keep the fastest for the process.  The count changes no result beyond
+        rounding order, only the GPU's power-capped clock during the long LM-head
+        launch, which differs from GPU to GPU.  Returns (best, {count: mean ms})."""
+        times = {c: [] for c in candidates}
+        for _ in range(reps):
+            for c in candidates:
+                pace.set_lmhead_splits(c)
+                b = torch.cuda.Event(enable_timing=True)
+                e = torch.cuda.Event(enable_timing=True)
+                self.run()  # settle after the change
+                b.record()
+                self.run()
+                e.record()
+                torch.cuda.synchronize()
+                times[c].append(b.elapsed_time(e))
+        mean = {c: sum(v) / len(v) for c, v in times.items()}
+        best = min(candidates, key=lambda c: (mean[c], c))
+        pace.set_lmhead_splits(best)
+        return best, mean
+
     def capture(self):
         """One step recorded as a CUDA graph (torch.cuda.CUDAGraph) for replay on a
         pool of fixed shape whose inputs are refreshed in place: every call of the

@@ -206,3 +206,30 @@ def test_degenerate_batches(case):
     else:
         assert (lp == 0).all()
         assert float(loss.item()) == 0.0
+
+
+def test_vocabulary_split_counts_agree():
+    """Every split count of the LM head gives the same log-probabilities up to the
+    merge's rounding order (40,000 rows: 157 row pairs, so every preferred count
+    from 2 up gives each resident cluster at least four items)."""
+    H, V, rows = 3584, 152064, 40000
+    hidden = workloads.bf16_normal_device((rows, H), 1.0, 31)
+    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), 32)
+    y = torch.randint(0, V, (rows,), dtype=torch.int32, device=DEV,
+                      generator=torch.Generator(device=DEV).manual_seed(5))
+    so = to_dev(np.array([0, rows], np.int64))
+    b = pace.make_batch(so, rows)
+    out = {}
+    try:
+        for s in (0, 2, 3, 4, 6, 8):
+            pace.set_lmhead_splits(s)
+            status = pace.new_status(DEV)
+            lp = torch.empty(rows, dtype=torch.float32, device=DEV)
+            pace.token_logprob(b, hidden, w, y, 1.0, logprob=lp, status=status)
+            torch.cuda.synchronize()
+            assert int(status.item()) == 0
+            out[s] = lp
+    finally:
+        pace.set_lmhead_splits(0)
+    for s, lp in out.items():
+        assert float((lp - out[0]).abs().max()) <= 2e-5, s

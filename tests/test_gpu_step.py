@@ -117,3 +117,28 @@ def test_repeated_run_advances_ema():
         assert (k, r_hat) == (ok, o)
     torch.cuda.synchronize()
     assert int(st.status.item()) == 0
+
+
+def test_split_tuner_keeps_a_candidate_and_results():
+    """PaceStep.tune_lmhead_splits times the candidates on this GPU, keeps the
+    fastest for the process, and the step's results do not depend on it."""
+    pool = workloads.make_pool("tiny")
+    rw = workloads.make_rows(pool)
+    H, V = pool.spec.hidden, pool.spec.vocab
+    hidden = workloads.bf16_normal_device((rw.n_rows, H), 1.0, 3)
+    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), 4)
+    behav = workloads.behaviour_logprob(rw, pool.trainer_version, workloads.uniform_center(V), 5)
+    st = step.PaceStep(step.build_inputs(pool, rw, hidden, w, behav))
+    st.run()
+    torch.cuda.synchronize()
+    lp0 = st.logprob.clone()
+    try:
+        best, mean = st.tune_lmhead_splits(candidates=(2, 4), reps=1)
+        assert best in (2, 4) and set(mean) == {2, 4}
+        assert all(v > 0 for v in mean.values())
+        st.run()
+        torch.cuda.synchronize()
+        assert int(st.status.item()) == 0
+        assert float((st.logprob - lp0).abs().max()) <= 2e-5
+    finally:
+        pace.set_lmhead_splits(0)

@@ -108,3 +108,12 @@ def test_host_argument_checks_return_before_launch(pace):
     assert st == pace.ERR_INVALID_ARG  # temperature must be > 0
     assert L.pace_token_logprob_workspace_size(1000, 10, 128, 1000) > 1000 * 128 * 2
     assert L.pace_score_pool_workspace_size(1000, 512) >= 16 * 1000
+
+
+def test_lmhead_split_control_range(pace):
+    L = pace.lib()
+    for bad in (-1, 9, 1 << 20):
+        assert L.pace_set_lmhead_splits(bad) == pace.ERR_INVALID_ARG
+    for good in (0, 1, 2, 4, 8):
+        assert L.pace_set_lmhead_splits(good) == pace.OK
+    assert L.pace_set_lmhead_splits(0) == pace.OK  # back to the automatic choice
