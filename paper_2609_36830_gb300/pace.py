@@ -136,21 +136,35 @@ def _check(st: int, where: str):
         raise PaceError(st, where)
 
 
-def _ptr(t: Optional[torch.Tensor]):
-    return None if t is None else ctypes.c_void_p(t.data_ptr())
+def _arg(t: Optional[torch.Tensor], dtype, n: Optional[int] = None, name: str = "tensor"):
+    """Device pointer of a contiguous tensor of `dtype` with at least `n` elements on
+    the current CUDA device; None passes as NULL.  Anything else raises here, before
+    the library sees a pointer its kernels could not use."""
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name}: expected a torch.Tensor, got {type(t).__name__}")
+    if not t.is_cuda:
+        raise ValueError(f"{name}: expected a CUDA tensor")
+    if t.get_device() != torch.cuda.current_device():
+        raise ValueError(f"{name}: on cuda:{t.get_device()}, the current device is "
+                         f"cuda:{torch.cuda.current_device()}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: expected a contiguous tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name}: expected {dtype}, got {t.dtype}")
+    if n is not None and t.numel() < n:
+        raise ValueError(f"{name}: needs at least {n} elements, has {t.numel()}")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+_U8, _I32T, _I64T = torch.uint8, torch.int32, torch.int64
+_F32T, _F64T, _BF16 = torch.float32, torch.float64, torch.bfloat16
 
 
 def _stream(stream=None):
     s = stream if stream is not None else torch.cuda.current_stream()
     return ctypes.c_void_p(s.cuda_stream)
-
-
-def _dev(t: torch.Tensor):
-    if not t.is_cuda:
-        raise ValueError("expected a CUDA tensor")
-    if not t.is_contiguous():
-        raise ValueError("expected a contiguous tensor")
-    return t
 
 
 def workspace(nbytes: int, device) -> torch.Tensor:
@@ -189,11 +203,16 @@ def score_pool(tags, offsets, c_version, s_pre, trainer_version, window, params=
     wl = 0 if window is None else window.numel()
     if ws is None:
         ws = workspace(lib().pace_score_pool_workspace_size(n, wl), dev)
+    units = n // max(p.group_size, 1)
     st = lib().pace_score_pool(
-        _ptr(tags), _ptr(_dev(offsets)), _ptr(_dev(c_version)), _ptr(s_pre), n, tags.numel(),
-        int(trainer_version), _ptr(window), wl, ctypes.byref(p), _ptr(out.get("kgen")),
-        _ptr(out.get("kwait")), _ptr(out.get("weight")), _ptr(out["score"]),
-        _ptr(out.get("unit_score")), _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+        _arg(tags, _I32T, None, "tags"), _arg(offsets, _I64T, n + 1, "offsets"),
+        _arg(c_version, _I32T, n, "c_version"), _arg(s_pre, _F32T, n, "s_pre"), n,
+        tags.numel(), int(trainer_version), _arg(window, _F32T, wl, "window"), wl,
+        ctypes.byref(p), _arg(out.get("kgen"), _F64T, n, "kgen"),
+        _arg(out.get("kwait"), _F64T, n, "kwait"), _arg(out.get("weight"), _F64T, n, "weight"),
+        _arg(out["score"], _F64T, n, "score"),
+        _arg(out.get("unit_score"), _F64T, units, "unit_score"), _arg(ws, _U8, None, "ws"),
+        ws.numel(), _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_score_pool")
     return out
 
@@ -227,10 +246,12 @@ def select(unit_score, group_size, params, out=None, ws=None, status=None, strea
     if ws is None:
         ws = workspace(lib().pace_select_workspace_size(u), dev)
     rh, k = _F64(), _I64()
-    st = lib().pace_select(_ptr(_dev(unit_score)), u, int(group_size), ctypes.byref(params),
-                           ctypes.byref(rh), ctypes.byref(k), _ptr(out["accepted"]),
-                           _ptr(out["rejected"]), _ptr(out["flags"]), _ptr(ws), ws.numel(),
-                           _ptr(status), _stream(stream))
+    st = lib().pace_select(_arg(unit_score, _F64T, u, "unit_score"), u, int(group_size),
+                           ctypes.byref(params), ctypes.byref(rh), ctypes.byref(k),
+                           _arg(out["accepted"], _I32T, n, "accepted"),
+                           _arg(out["rejected"], _I32T, n, "rejected"),
+                           _arg(out["flags"], _U8, n, "flags"), _arg(ws, _U8, None, "ws"),
+                           ws.numel(), _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_select")
     kk = k.value
     return (rh.value, kk, out["accepted"][:(u - kk) * group_size],
@@ -247,9 +268,11 @@ def select_k(unit_score, group_size, k, out=None, ws=None, status=None, stream=N
                "flags": torch.empty(max(n, 1), dtype=torch.uint8, device=dev)}
     if ws is None:
         ws = workspace(lib().pace_select_workspace_size(u), dev)
-    st = lib().pace_select_k(_ptr(_dev(unit_score)), u, int(group_size), int(k),
-                             _ptr(out["accepted"]), _ptr(out["rejected"]), _ptr(out["flags"]),
-                             _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    st = lib().pace_select_k(_arg(unit_score, _F64T, u, "unit_score"), u, int(group_size),
+                             int(k), _arg(out["accepted"], _I32T, n, "accepted"),
+                             _arg(out["rejected"], _I32T, n, "rejected"),
+                             _arg(out["flags"], _U8, n, "flags"), _arg(ws, _U8, None, "ws"),
+                             ws.numel(), _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_select_k")
     return (out["accepted"][:(u - k) * group_size], out["rejected"][:k * group_size],
             out["flags"][:n])
@@ -264,16 +287,20 @@ def loss_params(eps_low=0.2, eps_high=0.28, dual_clip=10.0, adv_eps=1e-6,
 
 
 def make_batch(seq_offsets, n_rows, seq_accepted=None, mask=None):
-    b = PaceBatch(_ptr(_dev(seq_offsets)), _ptr(seq_accepted), _ptr(mask),
-                  seq_offsets.numel() - 1, int(n_rows))
+    n_seq = seq_offsets.numel() - 1
+    b = PaceBatch(_arg(seq_offsets, _I64T, None, "seq_offsets"),
+                  _arg(seq_accepted, _U8, n_seq, "seq_accepted"),
+                  _arg(mask, _U8, int(n_rows), "mask"), n_seq, int(n_rows))
     b._keep = (seq_offsets, seq_accepted, mask)  # keep the tensors alive with the struct
     return b
 
 
 def make_loss_args(behav_lp, reward, group_size, params, loss_out, adv_out=None,
                    ratio_out=None):
-    a = PaceLossArgs(_ptr(_dev(behav_lp)), _ptr(_dev(reward)), int(group_size), params,
-                     _ptr(loss_out), _ptr(adv_out), _ptr(ratio_out))
+    a = PaceLossArgs(_arg(behav_lp, _F32T, None, "behav_lp"), _arg(reward, _F32T, None, "reward"),
+                     int(group_size), params, _arg(loss_out, _F64T, 1, "loss"),
+                     _arg(adv_out, _F32T, reward.numel(), "adv"),
+                     _arg(ratio_out, _F32T, behav_lp.numel(), "ratio"))
     a._keep = (behav_lp, reward, loss_out, adv_out, ratio_out)
     return a
 
@@ -283,9 +310,10 @@ def group_advantages(reward, group_size, seq_accepted=None, adv_eps=1e-6, std_un
     n = reward.numel()
     if out is None:
         out = torch.empty(n, dtype=torch.float32, device=reward.device)
-    st = lib().pace_group_advantages(_ptr(_dev(reward)), _ptr(seq_accepted), n, int(group_size),
-                                     float(adv_eps), int(bool(std_unbiased)), _ptr(out),
-                                     _stream(stream))
+    st = lib().pace_group_advantages(_arg(reward, _F32T, n, "reward"),
+                                     _arg(seq_accepted, _U8, n, "seq_accepted"), n,
+                                     int(group_size), float(adv_eps), int(bool(std_unbiased)),
+                                     _arg(out, _F32T, n, "out"), _stream(stream))
     _check(st, "pace_group_advantages")
     return out
 
@@ -295,23 +323,33 @@ def token_logprob_workspace_size(n_rows, n_seq, hidden, vocab):
                                                    int(vocab))
 
 
+def _head_shapes(batch: PaceBatch, hidden, w_vocab):
+    """(H, V) of a bf16 hidden [>= n_rows, H] / w_vocab [V, H] pair, checked."""
+    if hidden.dim() != 2 or w_vocab.dim() != 2 or hidden.shape[1] != w_vocab.shape[1]:
+        raise ValueError("hidden must be [n_rows, H] and w_vocab [V, H]")
+    if hidden.shape[0] < batch.n_rows:
+        raise ValueError(f"hidden has {hidden.shape[0]} rows, the batch {batch.n_rows}")
+    return int(hidden.shape[1]), int(w_vocab.shape[0])
+
+
 def token_logprob(batch: PaceBatch, hidden, w_vocab, targets, temperature=1.0, loss=None,
                   logprob=None, lse=None, ws=None, status=None, stream=None):
     """pace_token_logprob.  hidden [n_rows, H] and w_vocab [V, H] are bf16 tensors."""
-    if hidden.dtype != torch.bfloat16 or w_vocab.dtype != torch.bfloat16:
-        raise ValueError("hidden and w_vocab must be bf16")
-    n_rows, H = hidden.shape
-    V = w_vocab.shape[0]
+    H, V = _head_shapes(batch, hidden, w_vocab)
+    n_rows = batch.n_rows
     dev = hidden.device
     if logprob is None:
         logprob = torch.empty(n_rows, dtype=torch.float32, device=dev)
     if ws is None:
         ws = workspace(token_logprob_workspace_size(n_rows, batch.n_seq, H, V), dev)
-    st = lib().pace_token_logprob(ctypes.byref(batch), _ptr(_dev(hidden)), _ptr(_dev(w_vocab)),
-                                  _ptr(_dev(targets)), int(H), int(V), float(temperature),
-                                  _ptr(logprob), _ptr(lse),
-                                  ctypes.byref(loss) if loss is not None else None, _ptr(ws),
-                                  ws.numel(), _ptr(status), _stream(stream))
+    st = lib().pace_token_logprob(ctypes.byref(batch), _arg(hidden, _BF16, None, "hidden"),
+                                  _arg(w_vocab, _BF16, None, "w_vocab"),
+                                  _arg(targets, _I32T, n_rows, "targets"), H, V,
+                                  float(temperature), _arg(logprob, _F32T, n_rows, "logprob"),
+                                  _arg(lse, _F32T, n_rows, "lse"),
+                                  ctypes.byref(loss) if loss is not None else None,
+                                  _arg(ws, _U8, None, "ws"), ws.numel(),
+                                  _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_token_logprob")
     return logprob
 
@@ -321,8 +359,10 @@ def surrogate_loss(batch: PaceBatch, logprob, loss: PaceLossArgs, ws=None, statu
     dev = logprob.device
     if ws is None:
         ws = workspace(lib().pace_surrogate_loss_workspace_size(batch.n_rows, batch.n_seq), dev)
-    st = lib().pace_surrogate_loss(ctypes.byref(batch), _ptr(_dev(logprob)), ctypes.byref(loss),
-                                   _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    st = lib().pace_surrogate_loss(ctypes.byref(batch),
+                                   _arg(logprob, _F32T, batch.n_rows, "logprob"),
+                                   ctypes.byref(loss), _arg(ws, _U8, None, "ws"), ws.numel(),
+                                   _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_surrogate_loss")
 
 
@@ -354,20 +394,22 @@ def prefix_score(batch: PaceBatch, hidden, w_vocab, targets, behav_lp, temperatu
                  min_tokens=32, cap_tokens=1024, s_pre=None, logprob=None, ws=None, status=None,
                  stream=None):
     """pace_prefix_score (Eq. 6): float32 s_pre per prefix (NaN = not scored)."""
-    if hidden.dtype != torch.bfloat16 or w_vocab.dtype != torch.bfloat16:
-        raise ValueError("hidden and w_vocab must be bf16")
-    n_rows, H = hidden.shape
-    V = w_vocab.shape[0]
+    H, V = _head_shapes(batch, hidden, w_vocab)
+    n_rows = batch.n_rows
     dev = hidden.device
     if s_pre is None:
         s_pre = torch.empty(batch.n_seq, dtype=torch.float32, device=dev)
     if ws is None:
         ws = workspace(lib().pace_prefix_score_workspace_size(n_rows, batch.n_seq, H, V), dev)
-    st = lib().pace_prefix_score(ctypes.byref(batch), _ptr(_dev(hidden)), _ptr(_dev(w_vocab)),
-                                 _ptr(_dev(targets)), _ptr(_dev(behav_lp)), int(H), int(V),
+    st = lib().pace_prefix_score(ctypes.byref(batch), _arg(hidden, _BF16, None, "hidden"),
+                                 _arg(w_vocab, _BF16, None, "w_vocab"),
+                                 _arg(targets, _I32T, n_rows, "targets"),
+                                 _arg(behav_lp, _F32T, n_rows, "behav_lp"), H, V,
                                  float(temperature), int(min_tokens), int(cap_tokens),
-                                 _ptr(s_pre), _ptr(logprob), _ptr(ws), ws.numel(), _ptr(status),
-                                 _stream(stream))
+                                 _arg(s_pre, _F32T, batch.n_seq, "s_pre"),
+                                 _arg(logprob, _F32T, n_rows, "logprob"),
+                                 _arg(ws, _U8, None, "ws"), ws.numel(),
+                                 _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_prefix_score")
     return s_pre
 
@@ -383,9 +425,11 @@ def stale_k(tags, offsets, trainer_version, k_max, kbar=None, admitted=None, ws=
         admitted = torch.empty(n, dtype=torch.uint8, device=dev)
     if ws is None:
         ws = workspace(lib().pace_stale_k_workspace_size(n), dev)
-    st = lib().pace_stale_k(_ptr(tags), _ptr(_dev(offsets)), n, tags.numel(),
-                            int(trainer_version), float(k_max), _ptr(kbar), _ptr(admitted),
-                            _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    st = lib().pace_stale_k(_arg(tags, _I32T, None, "tags"),
+                            _arg(offsets, _I64T, n + 1, "offsets"), n, tags.numel(),
+                            int(trainer_version), float(k_max), _arg(kbar, _F64T, n, "kbar"),
+                            _arg(admitted, _U8, n, "admitted"), _arg(ws, _U8, None, "ws"),
+                            ws.numel(), _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_stale_k")
     return kbar, admitted
 
@@ -394,9 +438,11 @@ def staleness_histogram(values, flags, lo, hi, n_bins, hist=None, status=None, s
     """pace_staleness_histogram: int32-viewable uint32 counts [2, n_bins] (rejected, accepted)."""
     if hist is None:
         hist = torch.empty(2 * n_bins, dtype=torch.int32, device=values.device)
-    st = lib().pace_staleness_histogram(_ptr(_dev(values)), _ptr(flags), values.numel(),
-                                        float(lo), float(hi), int(n_bins), _ptr(hist),
-                                        _ptr(status), _stream(stream))
+    n = values.numel()
+    st = lib().pace_staleness_histogram(_arg(values, _F64T, n, "values"),
+                                        _arg(flags, _U8, n, "flags"), n, float(lo), float(hi),
+                                        int(n_bins), _arg(hist, _I32T, 2 * int(n_bins), "hist"),
+                                        _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_staleness_histogram")
     return hist.view(2, n_bins)
 
@@ -418,10 +464,14 @@ def quantile_admit(unit_score, r_hat, batch_units, window: ScoreWindow, min_obs=
         decision = torch.empty(max(n, 1), dtype=torch.uint8, device=dev)
     if kappa is None:
         kappa = torch.empty(1, dtype=torch.float64, device=dev)
-    st = lib().pace_quantile_admit(_ptr(_dev(unit_score)), n, float(r_hat), int(batch_units),
-                                   int(min_obs), _ptr(window.values), window.values.numel(),
-                                   _ptr(window.state), _ptr(decision), _ptr(kappa),
-                                   _ptr(status), _stream(stream))
+    st = lib().pace_quantile_admit(_arg(unit_score, _F64T, n, "unit_score"), n, float(r_hat),
+                                   int(batch_units), int(min_obs),
+                                   _arg(window.values, _F64T, None, "window.values"),
+                                   window.values.numel(),
+                                   _arg(window.state, _I64T, 2, "window.state"),
+                                   _arg(decision, _U8, n, "decision"),
+                                   _arg(kappa, _F64T, 1, "kappa"),
+                                   _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_quantile_admit")
     return decision[:n], kappa
 
@@ -435,9 +485,11 @@ def surrogate_backward(batch: PaceBatch, logprob, loss: PaceLossArgs, dlp=None, 
     if ws is None:
         ws = workspace(lib().pace_surrogate_backward_workspace_size(batch.n_rows, batch.n_seq),
                        dev)
-    st = lib().pace_surrogate_backward(ctypes.byref(batch), _ptr(_dev(logprob)),
-                                       ctypes.byref(loss), _ptr(dlp), _ptr(ws), ws.numel(),
-                                       _ptr(status), _stream(stream))
+    st = lib().pace_surrogate_backward(ctypes.byref(batch),
+                                       _arg(logprob, _F32T, batch.n_rows, "logprob"),
+                                       ctypes.byref(loss), _arg(dlp, _F32T, batch.n_rows, "dlp"),
+                                       _arg(ws, _U8, None, "ws"), ws.numel(),
+                                       _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_surrogate_backward")
     return dlp
 
@@ -446,8 +498,8 @@ def token_logprob_backward(batch: PaceBatch, hidden, w_vocab, targets, lse, dlp,
                            temperature=1.0, grad_hidden=None, grad_w=None, ws=None, status=None,
                            stream=None):
     """pace_token_logprob_backward: (grad_hidden fp32 [n_rows, H], grad_w fp32 [V, H])."""
-    n_rows, H = hidden.shape
-    V = w_vocab.shape[0]
+    H, V = _head_shapes(batch, hidden, w_vocab)
+    n_rows = batch.n_rows
     dev = hidden.device
     if grad_hidden is None:
         grad_hidden = torch.empty(n_rows, H, dtype=torch.float32, device=dev)
@@ -456,10 +508,15 @@ def token_logprob_backward(batch: PaceBatch, hidden, w_vocab, targets, lse, dlp,
     if ws is None:
         ws = workspace(lib().pace_token_logprob_backward_workspace_size(n_rows, batch.n_seq, H,
                                                                         V), dev)
-    st = lib().pace_token_logprob_backward(ctypes.byref(batch), _ptr(_dev(hidden)),
-                                           _ptr(_dev(w_vocab)), _ptr(_dev(targets)), int(H),
-                                           int(V), float(temperature), _ptr(_dev(lse)),
-                                           _ptr(_dev(dlp)), _ptr(grad_hidden), _ptr(grad_w),
-                                           _ptr(ws), ws.numel(), _ptr(status), _stream(stream))
+    st = lib().pace_token_logprob_backward(ctypes.byref(batch),
+                                           _arg(hidden, _BF16, None, "hidden"),
+                                           _arg(w_vocab, _BF16, None, "w_vocab"),
+                                           _arg(targets, _I32T, n_rows, "targets"), H, V,
+                                           float(temperature), _arg(lse, _F32T, n_rows, "lse"),
+                                           _arg(dlp, _F32T, n_rows, "dlp"),
+                                           _arg(grad_hidden, _F32T, n_rows * H, "grad_hidden"),
+                                           _arg(grad_w, _F32T, V * H, "grad_w"),
+                                           _arg(ws, _U8, None, "ws"), ws.numel(),
+                                           _arg(status, _I32T, 1, "status"), _stream(stream))
     _check(st, "pace_token_logprob_backward")
     return grad_hidden, grad_w
