@@ -472,17 +472,19 @@ __global__ void count_used_seqs_kernel(const long long* __restrict__ seq_in, int
 template <bool A_MN, bool B_MN, int EPI>
 pace_status launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmArgs a,
                         cudaStream_t st) {
-  static int done_dev = -1;
+  constexpr int kMaxDevices = 64;
+  static bool done[kMaxDevices] = {};  // shared-memory opt-in made on that device
   static std::mutex mu;
   int dev = 0;
   PACE_TRY_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return PACE_ERR_CUDA;
   {
     std::lock_guard<std::mutex> g(mu);
-    if (done_dev != dev) {
+    if (!done[dev]) {
       PACE_TRY_CUDA(cudaFuncSetAttribute(gemm_kernel<A_MN, B_MN, EPI>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(kGSmemBytes)));
-      done_dev = dev;
+      done[dev] = true;
     }
   }
   a.m_tiles = (a.M + GBM - 1) / GBM;
