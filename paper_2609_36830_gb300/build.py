@@ -20,7 +20,8 @@ LIB_PATH = os.path.join(HERE, "libpace.so")
 SOURCES = ["api.cu", "score.cu", "select.cu", "loss.cu", "lmhead.cu", "prefix.cu", "backward.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler",
-              "-ffp-contract=off", "-Xcompiler", "-fvisibility=hidden",
+              "-ffp-contract=off", "-Xcompiler", "-fvisibility=hidden", "-Xcompiler",
+              "-Wall,-Wextra",
               "--expt-relaxed-constexpr", "-I" + INCLUDE]
 
 

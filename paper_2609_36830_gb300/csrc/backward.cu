@@ -510,7 +510,7 @@ int64_t chunk_rows(int64_t n_rows) {
 }
 
 void carve_bw_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, BwWs* w) {
-  carve_lm_ws(cv, n_rows, n_seq, H, V, true, &w->lm);
+  carve_lm_ws(cv, n_rows, n_seq, H, true, &w->lm);
   const int64_t g_cols = (static_cast<int64_t>(V) + 63) / 64 * 64;
   w->g = cv.take<uint16_t>(static_cast<size_t>(chunk_rows(n_rows > 0 ? n_rows : 1)) * g_cols);
   w->n_seq_used = cv.take<int>(1);

@@ -431,7 +431,7 @@ pace_status lm_launch_info(LmLaunchInfo* out) {
 
 }  // namespace
 
-void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, bool compact,
+void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, bool compact,
                  LmWs* w) {
   const int64_t rows_cap = n_rows > BM ? n_rows : BM;
   carve_compact_ws(cv, n_seq, n_rows, &w->cw);
@@ -534,7 +534,7 @@ extern "C" size_t pace_token_logprob_workspace_size(int64_t n_rows, int64_t n_se
   if (n_rows < 0 || n_seq < 0 || hidden_size <= 0 || vocab_size <= 0) return 0;
   Carver cv;
   LmWs w;
-  carve_lm_ws(cv, n_rows, n_seq, hidden_size, vocab_size, true, &w);
+  carve_lm_ws(cv, n_rows, n_seq, hidden_size, true, &w);
   return cv.used;
 }
 
@@ -551,7 +551,7 @@ extern "C" pace_status pace_token_logprob(const PaceBatch* batch, const void* hi
   if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
   Carver cv(workspace, workspace_bytes);
   LmWs ws;
-  carve_lm_ws(cv, batch->n_rows, batch->n_seq, hidden_size, vocab_size,
+  carve_lm_ws(cv, batch->n_rows, batch->n_seq, hidden_size,
               lm_needs_compaction(batch), &ws);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
   cudaStream_t st = as_stream(stream);

@@ -32,7 +32,7 @@ struct LmWs {
 void carve_surrogate_ws(Carver& cv, int64_t n_seq, SurrogateWs* w);
 pace_status launch_group_adv(const float* reward, const uint8_t* accepted, int64_t n_seq, int G,
                              float eps, int unbiased, float* adv, cudaStream_t st);
-void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, bool compact,
+void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, bool compact,
                  LmWs* w);
 bool lm_needs_compaction(const PaceBatch* b);
 pace_status check_lm_args(const PaceBatch* batch, const void* hidden, const void* w_vocab,

@@ -87,8 +87,8 @@ struct PrefixWs {
   float* logprob;
 };
 
-void carve_prefix_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, PrefixWs* w) {
-  carve_lm_ws(cv, n_rows, n_seq, H, V, true, &w->lm);
+void carve_prefix_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, PrefixWs* w) {
+  carve_lm_ws(cv, n_rows, n_seq, H, true, &w->lm);
   w->mask_c = cv.take<uint8_t>(n_rows > 0 ? n_rows : 1);
   w->n_elig = cv.take<long long>(n_seq > 0 ? n_seq : 1);
   w->logprob = cv.take<float>(n_rows > 0 ? n_rows : 1);
@@ -104,7 +104,7 @@ extern "C" size_t pace_prefix_score_workspace_size(int64_t n_rows, int64_t n_seq
   if (n_rows < 0 || n_seq < 0 || hidden_size <= 0 || vocab_size <= 0) return 0;
   Carver cv;
   PrefixWs w;
-  carve_prefix_ws(cv, n_rows, n_seq, hidden_size, vocab_size, &w);
+  carve_prefix_ws(cv, n_rows, n_seq, hidden_size, &w);
   return cv.used;
 }
 
@@ -123,7 +123,7 @@ extern "C" pace_status pace_prefix_score(const PaceBatch* batch, const void* hid
   if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
   Carver cv(workspace, workspace_bytes);
   PrefixWs ws;
-  carve_prefix_ws(cv, batch->n_rows, batch->n_seq, hidden_size, vocab_size, &ws);
+  carve_prefix_ws(cv, batch->n_rows, batch->n_seq, hidden_size, &ws);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
   float* lp = logprob ? logprob : ws.logprob;
   PACE_TRY(check_lm_args(batch, hidden, w_vocab, targets, hidden_size, vocab_size, temperature,
