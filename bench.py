@@ -113,12 +113,11 @@ def _dist():
     return replicas.rank_env()
 
 
-def _make_step(seed_offset, device):
-    import torch
+def _make_step(seed_offset, device, workload=WORKLOAD):
     from paper_2609_36830_gb300 import pace, step, workloads
-    spec = workloads.SPECS[WORKLOAD]
+    spec = workloads.SPECS[workload]
     from paper_2609_36830_gb300 import replicas
-    pool = workloads.make_pool(WORKLOAD, seed=replicas.replica_seed(WORKLOAD, seed_offset))
+    pool = workloads.make_pool(workload, seed=replicas.replica_seed(workload, seed_offset))
     rows = workloads.make_rows(pool)
     H, V = spec.hidden, spec.vocab
     hidden = workloads.bf16_normal_device((rows.n_rows, H), 1.0, pool.seed + 11, device=device)
@@ -375,6 +374,45 @@ def _lmhead_backward(steps, warmup, device):
     return res
 
 
+def _other_workloads(steps, warmup, device, peak_s):
+    """The whole step on the multi-turn tool-use pool (256 trajectories, tool segments
+    masked) and the MoE-shaped pool (1024 trajectories, hidden 2048): the same call
+    sequence and launch configuration as the headline step."""
+    import torch
+    from paper_2609_36830_gb300 import pace
+    res = {}
+    for name in ("multiturn", "moe"):
+        pool, rows, x, st = _make_step(0, device, workload=name)
+        for _ in range(warmup):
+            st.run()
+        torch.cuda.synchronize()
+        M = st.rows_in_loss()
+        H, V = x.hidden.shape[1], x.w_vocab.shape[0]
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        lm = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        for (b, e), (lb, le) in zip(ev, lm):
+            pace.set_profile_events(pace.PROFILE_LMHEAD, lb, le)
+            b.record()
+            st.run()
+            e.record()
+        pace.set_profile_events(pace.PROFILE_LMHEAD)
+        torch.cuda.synchronize()
+        assert int(st.status.item()) == 0, pace.status_string(int(st.status.item()))
+        ms = statistics.mean(b.elapsed_time(e) for b, e in ev)
+        lm_ms = statistics.mean(b.elapsed_time(e) for b, e in lm)
+        tf = 2.0 * H * V * M / (lm_ms / 1e3) / 1e12
+        res[name] = {"workload": f"{name}: {pool.n_traj} trajectories, capacity {pool.n_target}, "
+                                 f"hidden {H}, vocab {V}",
+                     "rows_in_loss_per_step": M, "rows_total": int(rows.n_rows),
+                     "ms_per_step": ms, "tokens_per_s": M / (ms / 1e3),
+                     "lmhead_tflops": tf, "lmhead_frac_of_sustained": tf / peak_s}
+        del pool, rows, x, st
+        torch.cuda.empty_cache()
+    return res
+
+
 def _cpu_baseline(pool, rows, x, step_obj, n_rows_sample):
     """The oracle as it stands on this host's cores: full admission + a row sample."""
     import torch
@@ -620,11 +658,13 @@ def run_gpu(args):
 
     prefix = None
     backward = None
+    others = None
     if not args.no_sweep and rank == 0:
         prefix = _prefix_scoring(max(3, min(K, 5)), 3, device)
         backward = _lmhead_backward(3, 1, device)
         peak_s_b = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
         backward["frac_of_sustained"] = backward["tflops"] / peak_s_b
+        others = _other_workloads(3, 2, device, peak_s_b)
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -665,6 +705,7 @@ def run_gpu(args):
             "pool_scoring": sweep,
             "prefix_scoring": prefix,
             "lmhead_backward": backward,
+            "other_workloads": others,
         }
         print(json.dumps(line), flush=True)
     if ws > 1:
