@@ -60,7 +60,8 @@ def test_surrogate_backward_matches_oracle(rows_spec, agg):
 
 @pytest.mark.parametrize("rows,H,V,masked", [(100, 64, 256, False), (300, 128, 1000, True),
                                              (1000, 256, 2048, False), (700, 192, 4099, True),
-                                             (3000, 512, 2304, True)])
+                                             (3000, 512, 2304, True), (600, 2048, 1000, True),
+                                             (300, 4096, 520, False)])
 def test_lmhead_backward_matches_oracle(rows, H, V, masked):
     rng = np.random.default_rng(rows + H + V)
     hb = workloads.bf16_normal_host((rows, H), 1.0, rows)

@@ -38,7 +38,8 @@ def _run(hidden, w, targets, seq_offsets=None, seq_accepted=None, mask=None, tem
 
 @pytest.mark.parametrize("rows,H,V", [(1, 64, 256), (5, 64, 300), (127, 128, 1000),
                                       (128, 64, 256), (129, 192, 513), (300, 256, 2048),
-                                      (1000, 512, 4099), (2048, 1024, 8192)])
+                                      (1000, 512, 4099), (2048, 1024, 8192),
+                                      (300, 8192, 1000), (260, 16384, 700)])
 @pytest.mark.parametrize("masked", [False, True])
 def test_small_shapes_all_rows(rows, H, V, masked):
     rng = np.random.default_rng(rows * 7 + H + V)
