@@ -2,10 +2,13 @@
 // (Sec. 2: the policy factorises over tokens, log pi_theta(y_t | x, y_<t);
 // training temperature from the shared settings), without writing logits.
 //
-// lmhead_lse_kernel (sm_103a, one CTA per SM, 192 threads, warp-specialised):
-//   warp 0 / lane 0   TMA producer: 128x64 hidden tile + 256x64 vocabulary tile
-//                     per K step into a 4-stage shared-memory ring (128-byte
-//                     swizzle), completion tracked by mbarrier transaction bytes.
+// lmhead_lse_kernel (sm_103a, persistent 2-CTA clusters, one CTA per SM, 192
+// threads, warp-specialised):
+//   warp 0 / lane 0   TMA producer: per K step the CTA's own 128x64 hidden tile
+//                     and one half (128x64) of the pair's 256x64 vocabulary tile,
+//                     multicast into both CTAs of the cluster, into a 4-stage
+//                     shared-memory ring (128-byte swizzle), completion tracked
+//                     by mbarrier transaction bytes.
 //   warp 1 / lane 0   MMA issuer: tcgen05.mma kind::f16 (bf16 x bf16 -> fp32),
 //                     M=128, N=256, K=16 per instruction, accumulating a
 //                     128x256 logit tile in tensor memory; two accumulators
@@ -16,10 +19,11 @@
 //                     tcgen05.ld, keeps a running base-2 max and sum of
 //                     exponentials (online log-sum-exp) and picks out the
 //                     target's logit.
-// A CTA covers 128 rows and one of S contiguous vocabulary splits; it writes
-// one (max, sum) pair per row and split.  Consecutive CTAs share a row block,
-// so the hidden tile they re-read stays in L2 while the vocabulary streams.
-// S is chosen on the device from the rows actually present (pick_splits).
+// A work item is a pair of 128-row blocks (one per CTA of the cluster) and one
+// of S contiguous vocabulary splits; each CTA writes one (max, sum) pair per row
+// and split.  Consecutive items share a row pair, so the hidden tiles re-read
+// for every vocabulary tile stay in L2 while the vocabulary streams.  S is
+// chosen on the device from the rows actually present (pick_splits).
 //
 // lse_merge_kernel: per row, merges the S partial pairs into the log-sum-exp
 //   and writes lp = z_y / tau - lse.
