@@ -8,9 +8,14 @@
 //   small pools (U <= 512): one block ranks every unit against every other
 //     unit in shared memory and compacts the ids (one launch).
 //   large pools: MSB-first radix select over order-preserving 64-bit keys
-//     (six 11/10-bit digit passes, each a histogram + a one-block pick), then
-//     a three-phase scan compaction that rejects the units above the pivot
+//     (six 11/10-bit digit passes; each pass's blocks derive the previous
+//     pass's digit from its histogram themselves), then a three-phase scan
+//     compaction over 256-unit tiles that rejects the units above the pivot
 //     and the lowest-id units equal to it.
+//
+// Also here: the retained-vs-rejected staleness histograms (f4), the literal
+// sliding-window quantile admission (Sec. 3.1, Algorithm 1), and the
+// selection entry point that needs no caller workspace.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
