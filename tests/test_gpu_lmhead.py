@@ -234,3 +234,21 @@ def test_vocabulary_split_counts_agree():
         pace.set_lmhead_splits(0)
     for s, lp in out.items():
         assert float((lp - out[0]).abs().max()) <= 2e-5, s
+
+
+@pytest.mark.parametrize("scale", [8.0, 40.0])
+def test_large_logits(scale):
+    """Logits of tens (sharply peaked softmax): the online log-sum-exp keeps a running
+    maximum, so nothing overflows and lp still matches the oracle's two-pass fp64 LSE
+    within the same 5e-3."""
+    rows, H, V = 300, 256, 2048
+    rng = np.random.default_rng(int(scale))
+    hb = workloads.bf16_normal_host((rows, H), scale, 9)
+    wb = workloads.bf16_normal_host((V, H), 1.0 / math.sqrt(H), 10)
+    y = rng.integers(0, V, size=rows).astype(np.int32)
+    lp, lse = _run(bf16_dev(hb), bf16_dev(wb), to_dev(y))
+    st, olp, olse = oracle.token_logprob(hb, wb, y)
+    assert st == 0
+    assert np.isfinite(lp).all() and np.isfinite(lse).all()
+    assert np.abs(lp - olp).max() <= TOL, np.abs(lp - olp).max()
+    assert np.abs(lse - olse).max() <= TOL, np.abs(lse - olse).max()
