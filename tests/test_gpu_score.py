@@ -47,13 +47,18 @@ def test_workloads(name, n, mode):
 
 def test_group_sizes_and_gammas():
     pool = workloads.make_pool("math7b", n_traj=768)
-    for G in (1, 12, 16, 96):
+    for G in (1, 12, 16, 96, 256, 768):
         for gamma in (1, 2, 4, 7):
             args = (pool.tags, pool.meta["offsets_host"], pool.c_version, pool.s_pre,
                     pool.trainer_version, pool.window)
             g = gpu_score(*args, group_size=G, gamma=gamma)
             o = oracle_score(*args, group_size=G, gamma=gamma)
             _check(g, o, f"G={G} gamma={gamma}")
+    # the largest group the library takes (one group per 1024-thread block)
+    pool = workloads.make_pool("moe")
+    args = (pool.tags, pool.meta["offsets_host"], pool.c_version, pool.s_pre,
+            pool.trainer_version, pool.window)
+    _check(gpu_score(*args, group_size=1024), oracle_score(*args, group_size=1024), "G=1024")
 
 
 def test_sweep_128k_full_and_1m_sampled():
