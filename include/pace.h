@@ -174,7 +174,11 @@ PACE_API pace_status pace_select(const double* unit_score, int64_t n_units, int3
                         uint8_t* traj_accepted, void* workspace, size_t workspace_bytes,
                         int32_t* status_dev, void* stream);
 
-/* Same rejection with k given by the caller (0 <= k_units <= n_units). */
+/* Same rejection with k given by the caller (0 <= k_units <= n_units).
+ * Pools of at most 16,384 units are selected by one block and touch no
+ * workspace (it may be NULL); larger pools need pace_select_workspace_size
+ * bytes.  The first call on a device with more than 512 units sets a kernel
+ * attribute (its shared-memory size): make it before any stream capture. */
 PACE_API pace_status pace_select_k(const double* unit_score, int64_t n_units, int32_t group_size,
                           int64_t k_units, int32_t* accepted_ids, int32_t* rejected_ids,
                           uint8_t* traj_accepted, void* workspace, size_t workspace_bytes,

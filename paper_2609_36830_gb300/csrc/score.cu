@@ -5,10 +5,10 @@
 //                       bound): per trajectory the count T of policy tokens,
 //                       the exact integer sum of their tags and the largest
 //                       tag (+1, for the Lemma 1 premise check).
-//   window_prep_kernel  (pools of 32k trajectories and more) one block: sorts
-//                       the prefix-score window W and tabulates F = phi(count / |W|)
-//                       (Eqs. 9-10) for every possible count 0..|W| (F depends on
-//                       s only through the count).
+//   window_prep_kernel  (pools of 32k trajectories and more) block 0 sorts the
+//                       prefix-score window W; the other blocks tabulate
+//                       F = phi(count / |W|) (Eqs. 9-10) for every possible count
+//                       0..|W| (F depends on s only through the count).
 //   score_finalize_kernel  one thread per trajectory: K_gen, K_wait, the ECDF
 //                       count of s against the window (binary search in the
 //                       sorted window, or a direct count on small pools), F
@@ -279,6 +279,7 @@ struct FinalizeArgs {
   int32_t mode;
   int32_t gamma;
   int32_t group_size;
+  int32_t lanes;                // threads per trajectory for the direct count
   double f_missing;
   double* kgen;
   double* kwait;
@@ -300,13 +301,23 @@ __device__ __forceinline__ double sharpen(double q, int gamma) {
   return __ddiv_rn(a, __dadd_rn(a, b));
 }
 
-// Sorts the window ascending (bitonic, in shared memory, padded to a power of
-// two with +inf, which sorts last and is never read back) and tabulates
-// F[c] = phi_gamma(c / n) for c = 0..n.  NaN in the window is a data error.
+// Block 0 sorts the window ascending (bitonic, in shared memory, padded to a
+// power of two with +inf, which sorts last and is never read back); the other
+// blocks tabulate F[c] = phi_gamma(c / n) for c = 0..n, kFPerBlock entries
+// each, so the table's fp64 divisions and products run on many SMs instead of
+// queueing on one SM's fp64 units.  NaN in the window is a data error.
+constexpr int kFPerBlock = 32;
+
 __global__ void __launch_bounds__(1024) window_prep_kernel(const float* __restrict__ window, int n,
                                                            int gamma, float* __restrict__ sorted,
                                                            double* __restrict__ f_table,
                                                            int32_t* status) {
+  if (blockIdx.x > 0) {
+    const int c = (static_cast<int>(blockIdx.x) - 1) * kFPerBlock + static_cast<int>(threadIdx.x);
+    if (threadIdx.x < kFPerBlock && c <= n)
+      f_table[c] = sharpen(__ddiv_rn(static_cast<double>(c), static_cast<double>(n)), gamma);
+    return;
+  }
   __shared__ float sw[kMaxWindow];
   int np2 = 1;
   while (np2 < n) np2 <<= 1;
@@ -335,34 +346,64 @@ __global__ void __launch_bounds__(1024) window_prep_kernel(const float* __restri
   }
   __syncthreads();
   for (int k = threadIdx.x; k < n; k += blockDim.x) sorted[k] = sw[k];
-  for (int c = threadIdx.x; c <= n; c += blockDim.x)
-    f_table[c] = sharpen(__ddiv_rn(static_cast<double>(c), static_cast<double>(n)), gamma);
 }
 
+// blockDim.x = tpb * lanes: tpb trajectories per block (whole groups) and, on
+// the direct-count path, `lanes` threads per trajectory that each count one
+// strided share of the window (lanes = 1 with the sorted window).  Thread t
+// counts for trajectory slot t % tpb; threads t < tpb then do that
+// trajectory's fp64 work and the group means.
 __global__ void score_finalize_kernel(FinalizeArgs p) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int wpad = (p.window_len + 3) & ~3;
+  const int tpb = static_cast<int>(blockDim.x) / p.lanes;
   float* swin = reinterpret_cast<float*>(smem_raw);
   double* sscore = reinterpret_cast<double*>(smem_raw + align_up(wpad * sizeof(float), 16));
+  int* pcount = reinterpret_cast<int*>(sscore + tpb);  // [lanes][tpb] partial counts
 
   const bool sorted = p.window_sorted != nullptr;
   if (p.window_ready) {
-    if (sorted) {
-      for (int k = threadIdx.x; k < p.window_len; k += blockDim.x) swin[k] = p.window_sorted[k];
-    } else {  // raw window, NaN-padded to a multiple of 4 (NaN never counts as <= s)
-      for (int k = threadIdx.x; k < wpad; k += blockDim.x) {
-        const float w = k < p.window_len ? p.window[k] : __int_as_float(0x7fc00000);
-        swin[k] = w;
-        if (k < p.window_len && isnan(w)) report(p.status, PACE_ERR_NAN_INPUT);
+    // the sorted window, or the raw one NaN-padded to a multiple of 4 (NaN never
+    // counts as <= s); four loads per thread in flight at a time, since small
+    // blocks each copy the whole window
+    const float* src = sorted ? p.window_sorted : p.window;
+    const int nb = static_cast<int>(blockDim.x);
+    for (int k0 = threadIdx.x; k0 < wpad; k0 += 4 * nb) {
+      float w[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int k = k0 + j * nb;
+        w[j] = k < p.window_len ? src[k] : __int_as_float(0x7fc00000);
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int k = k0 + j * nb;
+        if (k < wpad) swin[k] = w[j];
+        if (!sorted && k < p.window_len && isnan(w[j])) report(p.status, PACE_ERR_NAN_INPUT);
       }
     }
   }
   __syncthreads();
 
-  const int G = p.group_size;
-  const int64_t per_block = blockDim.x;  // whole groups per block
-  const int64_t i = static_cast<int64_t>(blockIdx.x) * per_block + threadIdx.x;
-  if (i < p.n_traj) {
+  const int slot = static_cast<int>(threadIdx.x) % tpb;
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * tpb + slot;
+  const bool lead = static_cast<int>(threadIdx.x) < tpb;  // owns trajectory i's results
+  const float s = (i < p.n_traj && p.s_pre) ? p.s_pre[i] : __int_as_float(0x7fc00000);
+  if (p.window_ready && !sorted) {
+    // direct count of window values <= s, one strided share of the window per lane
+    int count = 0;
+    if (!isnan(s)) {
+      const float4* w4 = reinterpret_cast<const float4*>(swin);
+      for (int k = static_cast<int>(threadIdx.x) / tpb; k < wpad / 4; k += p.lanes) {
+        const float4 w = w4[k];
+        count += (w.x <= s) + (w.y <= s) + (w.z <= s) + (w.w <= s);
+      }
+    }
+    pcount[threadIdx.x] = count;
+    __syncthreads();
+  }
+
+  if (lead && i < p.n_traj) {
     const int64_t o0 = p.offsets[i], o1 = p.offsets[i + 1];
     if (o1 < o0 || (i == 0 && o0 != 0) || (i == p.n_traj - 1 && o1 != p.n_tokens))
       report(p.status, PACE_ERR_INVALID_ARG);
@@ -381,32 +422,23 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
     double f;
     if (!p.window_ready) {
       f = 1.0;
-    } else {
-      const float s = p.s_pre ? p.s_pre[i] : __int_as_float(0x7fc00000);
-      if (isnan(s)) {
-        f = p.f_missing;
-      } else {
-        if (sorted) {
-          // count of window values <= s: the first index of the sorted window
-          // holding a value > s
-          int lo = 0, hi = p.window_len;
-          while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (swin[mid] <= s) lo = mid + 1;
-            else hi = mid;
-          }
-          f = p.f_table[lo];
-        } else {  // small pools: count directly, F from the count
-          int count = 0;
-          const float4* w4 = reinterpret_cast<const float4*>(swin);
-          for (int k = 0; k < wpad / 4; ++k) {
-            const float4 w = w4[k];
-            count += (w.x <= s) + (w.y <= s) + (w.z <= s) + (w.w <= s);
-          }
-          f = sharpen(__ddiv_rn(static_cast<double>(count), static_cast<double>(p.window_len)),
-                      p.gamma);
-        }
+    } else if (isnan(s)) {
+      f = p.f_missing;
+    } else if (sorted) {
+      // count of window values <= s: the first index of the sorted window
+      // holding a value > s
+      int lo = 0, hi = p.window_len;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (swin[mid] <= s) lo = mid + 1;
+        else hi = mid;
       }
+      f = p.f_table[lo];
+    } else {  // small pools: F from the summed partial counts
+      int count = 0;
+      for (int l = 0; l < p.lanes; ++l) count += pcount[l * tpb + slot];
+      f = sharpen(__ddiv_rn(static_cast<double>(count), static_cast<double>(p.window_len)),
+                  p.gamma);
     }
     double sc;
     if (p.mode == PACE_SCORE_EFF) sc = __dadd_rn(kwait, __dmul_rn(f, kgen));
@@ -416,13 +448,17 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
     if (p.kwait) p.kwait[i] = kwait;
     if (p.weight) p.weight[i] = f;
     p.score[i] = sc;
-    sscore[threadIdx.x] = sc;
+    sscore[slot] = sc;
   }
   __syncthreads();
-  if (p.unit_score && i < p.n_traj && (threadIdx.x % G) == 0) {
+  const int G = p.group_size;
+  if (p.unit_score && lead && i < p.n_traj && (slot % G) == 0) {
     double acc = 0.0;
-    for (int g = 0; g < G; ++g) acc = __dadd_rn(acc, sscore[threadIdx.x + g]);
-    p.unit_score[i / G] = __ddiv_rn(acc, static_cast<double>(G));
+    for (int g = 0; g < G; ++g) acc = __dadd_rn(acc, sscore[slot + g]);
+    // for G = 2^m, acc * 2^-m is the same correctly rounded value as acc / G
+    // (2^-m is exact), one multiplication instead of a division
+    p.unit_score[i / G] = (G & (G - 1)) == 0 ? __dmul_rn(acc, 1.0 / static_cast<double>(G))
+                                             : __ddiv_rn(acc, static_cast<double>(G));
   }
 }
 
@@ -582,8 +618,11 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   // pools; smaller ones count against the raw window (the same bits either way).
   const bool use_table = window_ready && n_traj >= kTableMinTraj;
   if (use_table) {
-    window_prep_kernel<<<1, 1024, 0, st>>>(window, static_cast<int>(window_len), params->gamma,
-                                          wws.sorted, wws.f_table, status_dev);
+    const unsigned prep_blocks = 1u + static_cast<unsigned>((window_len + 1 + kFPerBlock - 1) /
+                                                            kFPerBlock);
+    window_prep_kernel<<<prep_blocks, 1024, 0, st>>>(window, static_cast<int>(window_len),
+                                                     params->gamma, wws.sorted, wws.f_table,
+                                                     status_dev);
     PACE_TRY(last_launch_status());
   }
   FinalizeArgs a;
@@ -611,11 +650,32 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   a.score = score;
   a.unit_score = unit_score;
   a.status = status_dev;
-  const int units_per_block = G >= 256 ? 1 : 256 / G;
-  const int threads = units_per_block * G;
-  const int64_t blocks = (n_traj + threads - 1) / threads;
+  // Whole groups per block.  With the sorted window: one thread per trajectory,
+  // 64 to 256 threads; small pools take fewer groups per block so that the
+  // per-trajectory fp64 work (GB300's fp64 rate is low) is spread over about two
+  // blocks per SM instead of queueing on a few SMs.  With the direct count, up to
+  // 8 threads per trajectory share the count so its chain is 8 times shorter.
+  const int max_units = G >= 256 ? 1 : 256 / G;
+  const int64_t n_units = n_traj / G;
+  const int64_t spread = 2 * static_cast<int64_t>(sm_count());
+  int64_t want = (n_units + spread - 1) / spread;
+  int min_units = 1;
+  int lanes = 1;
+  if (!use_table && window_ready) {
+    lanes = 8;
+  } else {
+    min_units = G >= 64 ? 1 : (64 + G - 1) / G;
+  }
+  want = want < min_units ? min_units : want;
+  const int units_per_block = want > max_units ? max_units : static_cast<int>(want);
+  const int tpb = units_per_block * G;
+  while (lanes > 1 && tpb * lanes > 1024) lanes /= 2;
+  a.lanes = lanes;
+  const int threads = tpb * lanes;
+  const int64_t blocks = (n_traj + tpb - 1) / tpb;
   const size_t smem = align_up(((window_len + 3) & ~3) * sizeof(float), 16) +
-                      static_cast<size_t>(threads) * sizeof(double);
+                      static_cast<size_t>(tpb) * sizeof(double) +
+                      static_cast<size_t>(threads) * sizeof(int);
   score_finalize_kernel<<<static_cast<unsigned>(blocks), threads, smem, st>>>(a);
   return last_launch_status();
 }

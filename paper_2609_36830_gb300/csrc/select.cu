@@ -7,6 +7,10 @@
 //
 //   small pools (U <= 512): one block ranks every unit against every other
 //     unit in shared memory and compacts the ids (one launch).
+//   mid-size pools (U <= 16,384): one block holds every key in shared memory,
+//     finds the pivot by a radix select that skips the bits all remaining
+//     candidates share and lists the units in output order; a cluster of up to
+//     8 CTAs then writes the ids and flags from that list (one launch).
 //   large pools: MSB-first radix select over order-preserving 64-bit keys
 //     (six 11/10-bit digit passes; each pass's blocks derive the previous
 //     pass's digit from its histogram themselves), then a three-phase scan
@@ -16,6 +20,7 @@
 // Also here: the retained-vs-rejected staleness histograms (f4), the literal
 // sliding-window quantile admission (Sec. 3.1, Algorithm 1), and the
 // selection entry point that needs no caller workspace.
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
@@ -27,6 +32,8 @@
 
 namespace pace {
 namespace {
+
+namespace cg = cooperative_groups;
 
 constexpr int kSmallMax = 512;
 constexpr int kSmallThreads = 512;
@@ -123,25 +130,27 @@ __device__ __forceinline__ void write_unit(int64_t u, bool rejected, int64_t rej
   }
 }
 
-// U <= 512: rank of u = number of units ordered before it.
+// U <= 512: rank of u = number of units ordered before it.  The ranks compare
+// order keys, not doubles: the same order (-0.0 equals +0.0), on the integer
+// pipe instead of GB300's narrow fp64 pipe.
 __global__ void __launch_bounds__(kSmallThreads)
     select_small_kernel(const double* __restrict__ score, int n_units, int G, int64_t k,
                         int32_t* accepted_ids, int32_t* rejected_ids, uint8_t* flags,
                         int32_t* status) {
-  __shared__ double s[kSmallMax];
+  __shared__ uint64_t s[kSmallMax];
   for (int u = threadIdx.x; u < n_units; u += blockDim.x) {
-    double x = score[u];
+    const double x = score[u];
     if (isnan(x)) report(status, PACE_ERR_NAN_INPUT);
-    s[u] = x;
+    s[u] = order_key(x);
   }
   __syncthreads();
   const int u = threadIdx.x;
   int rejected = 0;
   if (u < n_units) {
-    const double x = s[u];
+    const uint64_t x = s[u];
     int rank = 0;
     for (int w = 0; w < n_units; ++w) {
-      const double y = s[w];
+      const uint64_t y = s[w];
       rank += (y > x) || (y == x && w < u);
     }
     rejected = rank < k;
@@ -150,6 +159,255 @@ __global__ void __launch_bounds__(kSmallThreads)
   const int rej_before = block_exclusive_scan<int>(rejected, &n_rej);
   if (u < n_units)
     write_unit(u, rejected, rej_before, u - rej_before, G, accepted_ids, rejected_ids, flags);
+}
+
+// 512 < U <= 16,384: one launch of one thread-block cluster (1 to 8 CTAs).
+// CTA 0 selects: thread t owns the contiguous units [t * per, t * per + per)
+// (per, a power of two, <= 16); their order keys sit in shared memory at
+// [i * (kMidThreads + 1) + t], so a warp's accesses are conflict-free.  The k-th largest key (the pivot) is
+// found by a radix select that adapts to the keys: each round takes the
+// minimum and maximum of the remaining candidates, stops when they are equal,
+// and otherwise histograms the (up to 11) bits just below the highest bit
+// where they differ.  Candidates in one round share every bit above that one,
+// so a round fixes at least one bit and there are at most 64 rounds (two or
+// three for spread-out scores).  One pass in unit order then rejects the keys
+// above the pivot and the lowest-id k_rem keys equal to it, and lists the
+// accepted units followed by the rejected units (both ascending) in CTA 0's
+// shared memory, with a rejected byte per unit.  After a cluster barrier every
+// CTA reads that list through distributed shared memory and writes its share
+// of the ids and flags, consecutive threads at consecutive positions: whole
+// 32-byte sectors per warp store, on up to 8 SMs.
+constexpr int kMidMax = 16384;
+constexpr int kMidThreads = 1024;
+constexpr int kMidPer = kMidMax / kMidThreads;  // units per thread at most
+constexpr int kMidMaxCluster = 8;
+static_assert(kMidPer * kMidThreads == kMidMax, "whole units per thread");
+static_assert(kMidMax <= 65536, "unit numbers are stored in 16 bits");
+
+constexpr int kMidRow = kMidThreads + 1;  // keys per slot row (one pad key)
+
+// log2 of the units per thread: the smallest power of two that covers n_units.
+__host__ __device__ inline int mid_per_log2(int n_units) {
+  int lg = 0;
+  while ((kMidThreads << lg) < n_units) ++lg;
+  return lg;
+}
+
+__host__ __device__ inline size_t mid_smem_bytes(int n_units) {
+  return static_cast<size_t>(1 << mid_per_log2(n_units)) * kMidRow * sizeof(uint64_t) +
+         static_cast<size_t>(n_units) * (sizeof(uint16_t) + 1);
+}
+
+__device__ __forceinline__ void block_min_max(uint64_t& lo, uint64_t& hi, uint64_t* s_lo,
+                                              uint64_t* s_hi) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t a = __shfl_xor_sync(0xffffffffu, lo, o);
+    const uint64_t b = __shfl_xor_sync(0xffffffffu, hi, o);
+    lo = a < lo ? a : lo;
+    hi = b > hi ? b : hi;
+  }
+  if (lane == 0) {
+    s_lo[wid] = lo;
+    s_hi[wid] = hi;
+  }
+  __syncthreads();
+  if (wid == 0) {  // one warp folds the 32 warp results and leaves them in slot 0
+    lo = s_lo[lane];
+    hi = s_hi[lane];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const uint64_t a = __shfl_xor_sync(0xffffffffu, lo, o);
+      const uint64_t b = __shfl_xor_sync(0xffffffffu, hi, o);
+      lo = a < lo ? a : lo;
+      hi = b > hi ? b : hi;
+    }
+    if (lane == 0) {
+      s_lo[0] = lo;
+      s_hi[0] = hi;
+    }
+  }
+  __syncthreads();
+  lo = s_lo[0];
+  hi = s_hi[0];
+  __syncthreads();  // s_lo / s_hi are rewritten by the next call
+}
+
+// CTA 0's part: pivot, then the unit order and rejected bytes.  Every thread
+// of the block calls it; returns false (uniformly) if an invariant failed.
+__device__ bool mid_select_order(const double* __restrict__ score, int n_units, long long k,
+                                 uint64_t* keys, uint16_t* order, uint8_t* rej_u,
+                                 int32_t* status) {
+  __shared__ unsigned hist[kHistBins];
+  __shared__ uint64_t s_lo[kMidThreads / 32], s_hi[kMidThreads / 32];
+  __shared__ int s_digit;
+  __shared__ long long s_left;
+  const int t = threadIdx.x;
+  const int lg = mid_per_log2(n_units);
+  const int per = 1 << lg;
+  const int u0 = t * per;
+  const int n_mine = max(0, min(per, n_units - u0));
+
+  // coalesced loads: unit v (read by thread v % kMidThreads) belongs to thread
+  // v / per, slot v % per; rows of kMidRow keys make both this scatter (two-way)
+  // and the owners' row reads (none) nearly free of bank conflicts
+  for (int v = t; v < n_units; v += kMidThreads) {
+    const double x = score[v];
+    if (isnan(x)) report(status, PACE_ERR_NAN_INPUT);
+    keys[(v & (per - 1)) * kMidRow + (v >> lg)] = order_key(x);
+  }
+  __syncthreads();
+  uint64_t lo = ~0ull, hi = 0ull;
+  for (int i = 0; i < n_mine; ++i) {
+    const uint64_t key = keys[i * kMidRow + t];
+    lo = key < lo ? key : lo;
+    hi = key > hi ? key : hi;
+  }
+  uint64_t prefix = 0ull, mask = 0ull;
+  long long k_rem = k;
+  // each round fixes at least one more bit, so 64 rounds always suffice; the
+  // bound and the digit check only guard against a broken invariant
+  for (int round = 0;; ++round) {
+    block_min_max(lo, hi, s_lo, s_hi);  // every thread: the candidates' min and max
+    if (lo == hi) break;
+    if (round >= 64) {
+      if (t == 0) report(status, PACE_ERR_INVALID_ARG);
+      return false;
+    }
+    const int d = 63 - __clzll(static_cast<long long>(lo ^ hi));
+    const int shift = d >= 10 ? d - 10 : 0;
+    const int nbins = 1 << (d - shift + 1);
+    mask = d == 63 ? 0ull : (~0ull << (d + 1));
+    prefix = lo & mask;
+    for (int b = t; b < nbins; b += kMidThreads) hist[b] = 0u;
+    if (t == 0) s_digit = -1;
+    __syncthreads();
+    for (int i = 0; i < n_mine; ++i) {
+      const uint64_t key = keys[i * kMidRow + t];
+      if ((key & mask) == prefix)
+        atomicAdd(&hist[static_cast<unsigned>(key >> shift) & (nbins - 1)], 1u);
+    }
+    __syncthreads();
+    // thread t owns digits nbins-1-2t and nbins-2-2t: an exclusive scan in thread
+    // order counts the candidates with larger digits
+    const int top = nbins - 1 - 2 * t;
+    const int h0 = top >= 0 ? static_cast<int>(hist[top]) : 0;
+    const int h1 = top >= 1 ? static_cast<int>(hist[top - 1]) : 0;
+    long long run = block_exclusive_scan<long long>(h0 + h1, nullptr);
+    if (top >= 0 && run < k_rem && k_rem <= run + h0) {
+      s_digit = top;
+      s_left = k_rem - run;
+    }
+    run += h0;
+    if (top >= 1 && run < k_rem && k_rem <= run + h1) {
+      s_digit = top - 1;
+      s_left = k_rem - run;
+    }
+    __syncthreads();
+    if (s_digit < 0) {  // uniform: every thread reads the same word
+      if (t == 0) report(status, PACE_ERR_INVALID_ARG);
+      return false;
+    }
+    prefix |= static_cast<uint64_t>(s_digit) << shift;
+    mask |= static_cast<uint64_t>(nbins - 1) << shift;
+    k_rem = s_left;
+    lo = ~0ull;
+    hi = 0ull;
+    for (int i = 0; i < n_mine; ++i) {
+      const uint64_t key = keys[i * kMidRow + t];
+      if ((key & mask) == prefix) {
+        lo = key < lo ? key : lo;
+        hi = key > hi ? key : hi;
+      }
+    }
+  }
+  const uint64_t pivot = lo;  // k_rem of the keys equal to it are rejected, lowest ids first
+
+  int eq = 0;
+  for (int i = 0; i < n_mine; ++i) eq += keys[i * kMidRow + t] == pivot;
+  const long long tie0 = block_exclusive_scan<long long>(eq, nullptr);
+  int nrej = 0;
+  long long tie = tie0;
+  for (int i = 0; i < n_mine; ++i) {
+    const uint64_t key = keys[i * kMidRow + t];
+    nrej += key > pivot || (key == pivot && (tie++) < k_rem);
+  }
+  long long rpos = block_exclusive_scan<long long>(nrej, nullptr);
+  const long long n_acc = n_units - k;
+  tie = tie0;
+  for (int i = 0; i < n_mine; ++i) {
+    const uint64_t key = keys[i * kMidRow + t];
+    const bool r = key > pivot || (key == pivot && (tie++) < k_rem);
+    const int u = u0 + i;
+    order[r ? n_acc + rpos : u - rpos] = static_cast<uint16_t>(u);
+    rej_u[u] = r ? 1 : 0;
+    rpos += r;
+  }
+  return true;
+}
+
+__global__ void __launch_bounds__(kMidThreads, 1)
+    select_mid_kernel(const double* __restrict__ score, int n_units, int G, long long k,
+                      int32_t* accepted_ids, int32_t* rejected_ids, uint8_t* flags,
+                      int32_t* status) {
+  extern __shared__ __align__(16) unsigned char mid_smem[];
+  __shared__ int s_ok;
+  const int per = 1 << mid_per_log2(n_units);
+  uint64_t* keys = reinterpret_cast<uint64_t*>(mid_smem);
+  uint16_t* order =
+      reinterpret_cast<uint16_t*>(mid_smem + static_cast<size_t>(per) * kMidRow * sizeof(uint64_t));
+  uint8_t* rej_u = reinterpret_cast<uint8_t*>(order + n_units);
+  cg::cluster_group cluster = cg::this_cluster();
+  const unsigned rank = cluster.block_rank();
+  if (rank == 0) {  // uniform per block
+    const bool ok = mid_select_order(score, n_units, k, keys, order, rej_u, status);
+    if (threadIdx.x == 0) s_ok = ok ? 1 : 0;
+  }
+  cluster.sync();  // CTA 0's list is complete and visible to the cluster
+
+  const uint16_t* order0 = cluster.map_shared_rank(order, 0);
+  const uint8_t* rej0 = cluster.map_shared_rank(rej_u, 0);
+  if (*cluster.map_shared_rank(&s_ok, 0)) {  // uniform: one word read by every thread
+    const int64_t total = static_cast<int64_t>(n_units) * G;
+    const int nc = static_cast<int>(cluster.num_blocks());
+    const int64_t chunk = (total + nc - 1) / nc;
+    const int64_t p0 = static_cast<int64_t>(rank) * chunk;
+    const int64_t p1 = min(total, p0 + chunk);
+    const int64_t acc_end = (static_cast<int64_t>(n_units) - k) * G;
+    const int sq = kMidThreads / G, sr = kMidThreads % G;
+    // position p of the concatenated output [accepted ids | rejected ids] holds
+    // trajectory order0[p / G] * G + p % G; (q, r) = (p / G, p % G) is advanced
+    // by kMidThreads per step without dividing
+    int64_t p = p0 + threadIdx.x;
+    int q = static_cast<int>(p / G), r = static_cast<int>(p % G);
+    for (; p < p1; p += kMidThreads) {
+      const int32_t id = static_cast<int32_t>(order0[q]) * G + r;
+      if (p < acc_end) accepted_ids[p] = id;
+      else if (rejected_ids) rejected_ids[p - acc_end] = id;
+      q += sq;
+      r += sr;
+      if (r >= G) {
+        r -= G;
+        ++q;
+      }
+    }
+    if (flags) {  // flag of trajectory p: its unit p / G accepted or not
+      p = p0 + threadIdx.x;
+      q = static_cast<int>(p / G);
+      r = static_cast<int>(p % G);
+      for (; p < p1; p += kMidThreads) {
+        flags[p] = rej0[q] ? 0 : 1;
+        q += sq;
+        r += sr;
+        if (r >= G) {
+          r -= G;
+          ++q;
+        }
+      }
+    }
+  }
+  cluster.sync();  // CTA 0's shared memory stays until every CTA has read it
 }
 
 // Pass `pass` of the MSB-first radix select (256 threads per block).  The state
@@ -331,6 +589,72 @@ SelectWs carve_select_ws(Carver& cv, int64_t n_units) {
   return w;
 }
 
+// Opts select_mid_kernel into its largest dynamic shared memory and finds the
+// largest cluster (8, 4, 2 or 1 CTAs) of such blocks the current device can
+// hold, once per device.
+pace_status mid_cluster_limit(int* out) {
+  constexpr int kMaxDevices = 64;
+  static int limit[kMaxDevices] = {};
+  static std::mutex mu;
+  int dev = 0;
+  PACE_TRY_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return PACE_ERR_CUDA;
+  std::lock_guard<std::mutex> g(mu);
+  if (limit[dev] == 0) {
+    const size_t smem = mid_smem_bytes(kMidMax);
+    PACE_TRY_CUDA(cudaFuncSetAttribute(select_mid_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem)));
+    int c = kMidMaxCluster;
+    for (; c > 1; c /= 2) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(static_cast<unsigned>(c), 1, 1);
+      cfg.blockDim = dim3(kMidThreads, 1, 1);
+      cfg.dynamicSmemBytes = smem;
+      cudaLaunchAttribute attr;
+      attr.id = cudaLaunchAttributeClusterDimension;
+      attr.val.clusterDim.x = static_cast<unsigned>(c);
+      attr.val.clusterDim.y = 1;
+      attr.val.clusterDim.z = 1;
+      cfg.attrs = &attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, select_mid_kernel, &cfg) == cudaSuccess && n >= 1)
+        break;
+      (void)cudaGetLastError();  // a refused size is not an error of this call
+    }
+    limit[dev] = c;
+  }
+  *out = limit[dev];
+  return PACE_OK;
+}
+
+// One cluster: 1 CTA up to 16,384 outputs, then one more SM per doubling, up to 8.
+pace_status launch_select_mid(const double* unit_score, int n_units, int G, long long k,
+                              int32_t* accepted_ids, int32_t* rejected_ids, uint8_t* flags,
+                              int32_t* status, cudaStream_t st) {
+  int limit = 1;
+  PACE_TRY(mid_cluster_limit(&limit));
+  const int64_t total = static_cast<int64_t>(n_units) * G;
+  int c = 1;
+  while (c < limit && total > static_cast<int64_t>(c) * 16384) c *= 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(c), 1, 1);
+  cfg.blockDim = dim3(kMidThreads, 1, 1);
+  cfg.dynamicSmemBytes = mid_smem_bytes(n_units);
+  cfg.stream = st;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = static_cast<unsigned>(c);
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  PACE_TRY_CUDA(cudaLaunchKernelEx(&cfg, select_mid_kernel, unit_score, n_units, G, k,
+                                   accepted_ids, rejected_ids, flags, status));
+  return last_launch_status();
+}
+
 int grid_for(int64_t n, int threads, int per_sm) {
   int64_t b = (n + threads - 1) / threads;
   const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;
@@ -413,6 +737,9 @@ extern "C" pace_status pace_select_k(const double* unit_score, int64_t n_units, 
                                                      status_dev);
     return last_launch_status();
   }
+  if (n_units <= kMidMax)
+    return launch_select_mid(unit_score, static_cast<int>(n_units), G, static_cast<long long>(k),
+                             accepted_ids, rejected_ids, traj_accepted, status_dev, st);
   if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
   Carver cv(workspace, workspace_bytes);
   SelectWs ws = carve_select_ws(cv, n_units);

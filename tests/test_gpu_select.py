@@ -28,14 +28,21 @@ def _check_k(scores, G, k):
     np.testing.assert_array_equal(flags, oflag)
 
 
-@pytest.mark.parametrize("U", [1, 2, 7, 64, 511, 512, 513, 2048, 5000, 131072, 1048576])
-@pytest.mark.parametrize("dist", ["ties", "continuous", "constant"])
+# 1..512 units: the one-block rank kernel; 513..16384: the one-block adaptive
+# radix select; above: the multi-block radix select.
+@pytest.mark.parametrize("U", [1, 2, 7, 64, 511, 512, 513, 2048, 5000, 16384, 16385, 131072,
+                               1048576])
+@pytest.mark.parametrize("dist", ["ties", "continuous", "constant", "ulps", "signed_wide"])
 def test_select_k_matches_oracle(U, dist):
     rng = np.random.default_rng(U + len(dist))
     if dist == "ties":
         s = rng.integers(0, 9, size=U).astype(np.float64) / 4.0
     elif dist == "continuous":
         s = rng.random(U) * 40.0
+    elif dist == "ulps":  # keys that differ only in their last two bits
+        s = 1.0 + rng.integers(0, 4, size=U) * np.finfo(np.float64).eps
+    elif dist == "signed_wide":  # both signs, magnitudes from 1e-300 to 1e300
+        s = np.where(rng.random(U) < 0.5, -1.0, 1.0) * 10.0 ** rng.uniform(-300, 300, size=U)
     else:
         s = np.full(U, 2.5)
     ks = sorted({0, 1, U // 3, U // 2, U - 1, U} - {-1})
@@ -45,9 +52,11 @@ def test_select_k_matches_oracle(U, dist):
             _check_k(s, G, k)
 
 
-def test_select_handles_negative_zero_and_subnormals():
-    s = np.array([0.0, -0.0, 5e-324, 1e-310, 0.0, 3.0, -0.0, 5e-324] * 100, np.float64)
-    for k in (1, 3, 100, 401, 799):
+@pytest.mark.parametrize("reps", [50, 100, 1000])  # 400, 800 and 8000 units
+def test_select_handles_negative_zero_and_subnormals(reps):
+    s = np.array([0.0, -0.0, 5e-324, 1e-310, 0.0, 3.0, -0.0, 5e-324] * reps, np.float64)
+    n = s.size
+    for k in (1, 3, 100, n // 2 + 1, n - 1):
         _check_k(s, 1, k)
 
 
@@ -73,9 +82,38 @@ def test_select_with_budget_on_workloads(name, n, beta, r_prev):
 
 
 def test_nan_scores_are_reported():
-    s = np.arange(600, dtype=np.float64)
-    s[17] = np.nan
-    _gpu_select_k(s, 1, 10, expect_status=pace.ERR_NAN_INPUT)
+    for n in (600, 20000):
+        s = np.arange(n, dtype=np.float64)
+        s[17] = np.nan
+        _gpu_select_k(s, 1, 10, expect_status=pace.ERR_NAN_INPUT)
     s = np.arange(40, dtype=np.float64)
     s[3] = np.nan
     _gpu_select_k(s, 2, 5, expect_status=pace.ERR_NAN_INPUT)
+
+
+@pytest.mark.parametrize("U", [513, 16384])
+def test_mid_size_pools_take_no_workspace(U):
+    """Pools of up to 16,384 units are selected by one block without the caller's
+    workspace: a NULL workspace of 0 bytes is accepted and gives the oracle's ids."""
+    import ctypes
+    rng = np.random.default_rng(U)
+    s = rng.integers(0, 50, size=U).astype(np.float64) / 8.0
+    k = U // 3
+    G = 2
+    scores = to_dev(s)
+    acc = torch.full((U * G,), -7, dtype=torch.int32, device=DEV)
+    rej = torch.full((U * G,), -7, dtype=torch.int32, device=DEV)
+    flags = torch.full((U * G,), 9, dtype=torch.uint8, device=DEV)
+    status = pace.new_status(DEV)
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    st = pace.lib().pace_select_k(ctypes.c_void_p(scores.data_ptr()), U, G, k,
+                                  ctypes.c_void_p(acc.data_ptr()), ctypes.c_void_p(rej.data_ptr()),
+                                  ctypes.c_void_p(flags.data_ptr()), None, 0,
+                                  ctypes.c_void_p(status.data_ptr()), stream)
+    assert st == pace.OK, pace.status_string(st)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    _, oacc, orej, oflag = oracle.select(s, G, k)
+    np.testing.assert_array_equal(as_np(acc)[:(U - k) * G], oacc)
+    np.testing.assert_array_equal(as_np(rej)[:k * G], orej)
+    np.testing.assert_array_equal(as_np(flags), oflag)
