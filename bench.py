@@ -194,13 +194,16 @@ def _sweep_scoring(steps, warmup, device, n_traj=SWEEP_N):
     assert int(status.item()) == 0, pace.status_string(int(status.item()))
     k_ms = statistics.mean(b.elapsed_time(e) for b, e in zip(k_b, k_e))
     s_ms = statistics.mean(b.elapsed_time(e) for b, e in zip(s_b, s_e))
+    # the same two calls replayed as one CUDA graph (no host launch gaps)
+    g_ms = _timed(_capture(one, device).replay, steps, warmup, flush)
+    assert int(status.item()) == 0, pace.status_string(int(status.item()))
     # algorithmic bytes of the tag reduction: every tag once, the offsets once,
     # the 16-byte per-trajectory accumulators written once
     k_bytes = 4 * tok + 8 * (n + 1) + 16 * n
     res = {"workload": f"sweep pool {n} trajectories, {tok} tags", "traj_per_s": n / (s_ms / 1e3),
            "tag_reduce_traffic": (TAG_REDUCE_DRAM_BYTES_PER_TAG * tok
                                   if TAG_REDUCE_DRAM_BYTES_PER_TAG else None),
-           "ms_per_call": s_ms, "tag_reduce_ms": k_ms,
+           "ms_per_call": s_ms, "ms_per_call_graph": g_ms, "tag_reduce_ms": k_ms,
            "tag_reduce_gbs": k_bytes / (k_ms / 1e3) / 1e9, "tag_reduce_bytes": k_bytes}
     if n_traj == SWEEP_N:
         res["admission_variants"] = _admission_variants(pool, tok, out, sel, status, flush,
@@ -208,6 +211,21 @@ def _sweep_scoring(steps, warmup, device, n_traj=SWEEP_N):
     del pool, flush
     torch.cuda.empty_cache()
     return res
+
+
+def _capture(fn, device):
+    """fn's stream-ordered calls recorded as one CUDA graph (after one eager call on a
+    side stream, so one-time launch set-up stays outside the capture)."""
+    import torch
+    side = torch.cuda.Stream(device=device)
+    side.wait_stream(torch.cuda.current_stream(device))
+    with torch.cuda.stream(side):
+        fn()
+    torch.cuda.current_stream(device).wait_stream(side)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn()
+    return g
 
 
 def _timed(fn, steps, warmup, flush=None):
@@ -652,6 +670,7 @@ def run_gpu(args):
                 sweep = r_sw
             else:
                 sizes.append({k: r_sw[k] for k in ("workload", "traj_per_s", "ms_per_call",
+                                                   "ms_per_call_graph",
                                                    "tag_reduce_ms", "tag_reduce_gbs",
                                                    "tag_reduce_frac_of_hbm")})
         sweep["smaller_pools"] = sizes
@@ -815,6 +834,13 @@ def run_case(args):
         tf = 3 * 2.0 * rows * H * V / (ms / 1e3) / 1e12
         print(json.dumps({"case": "lmhead_bwd", "rows": rows, "H": H, "V": V, "ms": ms,
                           "tflops": tf}), flush=True)
+    elif args.case == "pool":
+        # pace_score_pool + pace_select on one sweep pool, L2 evicted before each call,
+        # eagerly and as one CUDA-graph replay
+        res = _sweep_scoring(args.steps, args.warmup, device, n_traj=args.case_traj)
+        print(json.dumps({"case": "pool", **res,
+                          "tag_reduce_frac_of_hbm": res["tag_reduce_gbs"] / peaks["hbm_gbs"]}),
+              flush=True)
     else:
         pool = workloads.make_pool("sweep", n_traj=args.case_traj, device=device)
         n = pool.n_traj
@@ -849,7 +875,7 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=512)
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce", "step_tiny"],
+    ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce", "step_tiny", "pool"],
                     default=None,
                     help="time one kernel on a small case (profiler captures)")
     ap.add_argument("--case-rows", type=int, default=4864)
