@@ -175,10 +175,11 @@ PACE_API pace_status pace_select(const double* unit_score, int64_t n_units, int3
                         int32_t* status_dev, void* stream);
 
 /* Same rejection with k given by the caller (0 <= k_units <= n_units).
- * Pools of at most 16,384 units are selected by one block and touch no
- * workspace (it may be NULL); larger pools need pace_select_workspace_size
- * bytes.  The first call on a device with more than 512 units sets a kernel
- * attribute (its shared-memory size): make it before any stream capture. */
+ * Pools of at most 131,072 units are selected by one thread-block cluster and
+ * touch no workspace (it may be NULL); larger pools need
+ * pace_select_workspace_size bytes.  The first call on a device with more than
+ * 512 units sets a kernel attribute (its shared-memory size): make it before
+ * any stream capture. */
 PACE_API pace_status pace_select_k(const double* unit_score, int64_t n_units, int32_t group_size,
                           int64_t k_units, int32_t* accepted_ids, int32_t* rejected_ids,
                           uint8_t* traj_accepted, void* workspace, size_t workspace_bytes,
@@ -191,8 +192,9 @@ PACE_API size_t pace_select_workspace_size(int64_t n_units);
  * a plugin running inside a host framework whose memory pool owns all device
  * memory, or a latency-critical loop where an allocation could synchronise
  * the device.  Such a caller still passes its inputs and outputs; the scratch
- * the radix path needs comes from a fixed array of 128 KB inside the library,
- * which every GPU that loads the library keeps until the process exits.
+ * the radix path (pools above 131,072 units) needs comes from a fixed array of
+ * 128 KB inside the library, which every GPU that loads the library keeps
+ * until the process exits.
  *   - n_units must be at most 2^20 (1,048,576); larger pools get
  *     PACE_ERR_UNSUPPORTED_SHAPE and nothing is launched.
  *   - The first call on a device looks up the array's device address (with

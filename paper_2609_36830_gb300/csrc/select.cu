@@ -7,10 +7,11 @@
 //
 //   small pools (U <= 512): one block ranks every unit against every other
 //     unit in shared memory and compacts the ids (one launch).
-//   mid-size pools (U <= 16,384): one block holds every key in shared memory,
-//     finds the pivot by a radix select that skips the bits all remaining
-//     candidates share and lists the units in output order; a cluster of up to
-//     8 CTAs then writes the ids and flags from that list (one launch).
+//   mid-size pools (U <= 131,072): one cluster of up to 8 CTAs holds every key
+//     in shared memory (16,384 per CTA), finds the pivot by a radix select that
+//     skips the bits all remaining candidates share (histograms combined
+//     through distributed shared memory), and each CTA writes the ids and flags
+//     of its own units (one launch).
 //   large pools: MSB-first radix select over order-preserving 64-bit keys
 //     (six 11/10-bit digit passes; each pass's blocks derive the previous
 //     pass's digit from its histogram themselves), then a three-phase scan
@@ -161,45 +162,58 @@ __global__ void __launch_bounds__(kSmallThreads)
     write_unit(u, rejected, rej_before, u - rej_before, G, accepted_ids, rejected_ids, flags);
 }
 
-// 512 < U <= 16,384: one launch of one thread-block cluster (1 to 8 CTAs).
-// CTA 0 selects: thread t owns the contiguous units [t * per, t * per + per)
-// (per, a power of two, <= 16); their order keys sit in shared memory at
-// [i * (kMidThreads + 1) + t], so a warp's accesses are conflict-free.  The k-th largest key (the pivot) is
-// found by a radix select that adapts to the keys: each round takes the
-// minimum and maximum of the remaining candidates, stops when they are equal,
-// and otherwise histograms the (up to 11) bits just below the highest bit
-// where they differ.  Candidates in one round share every bit above that one,
-// so a round fixes at least one bit and there are at most 64 rounds (two or
-// three for spread-out scores).  One pass in unit order then rejects the keys
-// above the pivot and the lowest-id k_rem keys equal to it, and lists the
-// accepted units followed by the rejected units (both ascending) in CTA 0's
-// shared memory, with a rejected byte per unit.  After a cluster barrier every
-// CTA reads that list through distributed shared memory and writes its share
-// of the ids and flags, consecutive threads at consecutive positions: whole
-// 32-byte sectors per warp store, on up to 8 SMs.
-constexpr int kMidMax = 16384;
-constexpr int kMidThreads = 1024;
-constexpr int kMidPer = kMidMax / kMidThreads;  // units per thread at most
-constexpr int kMidMaxCluster = 8;
-static_assert(kMidPer * kMidThreads == kMidMax, "whole units per thread");
-static_assert(kMidMax <= 65536, "unit numbers are stored in 16 bits");
+// 512 < U <= 131,072: one launch of one thread-block cluster of C CTAs (1, 2,
+// 4 or 8; 1024 threads each).  CTA r owns the contiguous units
+// [r * B, r * B + B) with B = ceil(U / C) <= 16,384; its thread t owns the
+// contiguous units t * per .. t * per + per - 1 of that range (per, a power of
+// two, <= 16), whose order keys sit in shared memory at [i * (1024 + 1) + t], so
+// a warp's accesses are conflict-free.
+//
+// The k-th largest key (the pivot) is found by a radix select that adapts to
+// the keys.  Each round takes the minimum and maximum of the remaining
+// candidates over the whole cluster, stops when they are equal, and otherwise
+// histograms the (up to 11) bits just below the highest bit where they differ;
+// each CTA counts its own keys and sums the C histograms through distributed
+// shared memory.  Candidates in one round share every bit above that one, so a
+// round fixes at least one bit and there are at most 64 rounds (two to four for
+// spread-out scores).  Every CTA computes the same values from the same shared
+// data, so all of them take the same branches and pass the same sequence of
+// cluster barriers.
+//
+// Then each CTA counts its keys above and equal to the pivot, learns the
+// counts of the lower-ranked CTAs (ties are rejected lowest id first), lists
+// its accepted units and then its rejected units in shared memory, and writes
+// its own contiguous runs of the id lists and flags, consecutive threads at
+// consecutive positions (whole 32-byte sectors per warp store).
+constexpr int kSelCtaUnits = 16384;  // units per CTA at most
+constexpr int kSelThreads = 1024;
+constexpr int kSelPer = kSelCtaUnits / kSelThreads;  // units per thread at most
+constexpr int kSelMaxCluster = 8;
+constexpr int64_t kSelMaxUnits = int64_t(kSelCtaUnits) * kSelMaxCluster;
+constexpr int kSelRow = kSelThreads + 1;  // keys per slot row (one pad key)
+static_assert(kSelPer * kSelThreads == kSelCtaUnits, "whole units per thread");
+static_assert(kSelCtaUnits <= 65536, "a CTA's unit numbers are stored in 16 bits");
 
-constexpr int kMidRow = kMidThreads + 1;  // keys per slot row (one pad key)
-
-// log2 of the units per thread: the smallest power of two that covers n_units.
-__host__ __device__ inline int mid_per_log2(int n_units) {
+// log2 of the units per thread: the smallest power of two that covers b units.
+__host__ __device__ inline int sel_per_log2(int b) {
   int lg = 0;
-  while ((kMidThreads << lg) < n_units) ++lg;
+  while ((kSelThreads << lg) < b) ++lg;
   return lg;
 }
 
-__host__ __device__ inline size_t mid_smem_bytes(int n_units) {
-  return static_cast<size_t>(1 << mid_per_log2(n_units)) * kMidRow * sizeof(uint64_t) +
-         static_cast<size_t>(n_units) * (sizeof(uint16_t) + 1);
+// Dynamic shared memory of a CTA holding b units: keys, unit order, rejected bytes.
+__host__ __device__ inline size_t sel_smem_bytes(int b) {
+  return static_cast<size_t>(1 << sel_per_log2(b)) * kSelRow * sizeof(uint64_t) +
+         static_cast<size_t>(b) * (sizeof(uint16_t) + 1);
 }
 
-__device__ __forceinline__ void block_min_max(uint64_t& lo, uint64_t& hi, uint64_t* s_lo,
-                                              uint64_t* s_hi) {
+// Minimum and maximum of (lo, hi) over every thread of every CTA of the
+// cluster; the result is in every thread.  s_mm is this CTA's slot that peers
+// read; s_g holds the cluster result for this CTA's threads.
+template <bool kMulti>
+__device__ __forceinline__ void cluster_min_max(cg::cluster_group& cluster, uint64_t& lo,
+                                                uint64_t& hi, uint64_t* s_wlo, uint64_t* s_whi,
+                                                uint64_t* s_mm, uint64_t* s_g) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -209,13 +223,13 @@ __device__ __forceinline__ void block_min_max(uint64_t& lo, uint64_t& hi, uint64
     hi = b > hi ? b : hi;
   }
   if (lane == 0) {
-    s_lo[wid] = lo;
-    s_hi[wid] = hi;
+    s_wlo[wid] = lo;
+    s_whi[wid] = hi;
   }
   __syncthreads();
-  if (wid == 0) {  // one warp folds the 32 warp results and leaves them in slot 0
-    lo = s_lo[lane];
-    hi = s_hi[lane];
+  if (wid == 0) {  // one warp folds the 32 warp results into this CTA's slot
+    lo = s_wlo[lane];
+    hi = s_whi[lane];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const uint64_t a = __shfl_xor_sync(0xffffffffu, lo, o);
@@ -224,76 +238,147 @@ __device__ __forceinline__ void block_min_max(uint64_t& lo, uint64_t& hi, uint64
       hi = b > hi ? b : hi;
     }
     if (lane == 0) {
-      s_lo[0] = lo;
-      s_hi[0] = hi;
+      s_mm[0] = lo;
+      s_mm[1] = hi;
+      if (!kMulti) {  // one CTA: its result is the cluster's
+        s_g[0] = lo;
+        s_g[1] = hi;
+      }
+    }
+  }
+  if (!kMulti) {
+    __syncthreads();
+    lo = s_g[0];
+    hi = s_g[1];
+    return;
+  }
+  cluster.sync();  // every CTA's slot is written
+  if (wid == 0) {  // lanes < C read the peers' slots; one warp folds them
+    const int nc = static_cast<int>(cluster.num_blocks());
+    lo = ~0ull;
+    hi = 0ull;
+    if (lane < nc) {
+      const uint64_t* peer = cluster.map_shared_rank(s_mm, static_cast<unsigned>(lane));
+      lo = peer[0];
+      hi = peer[1];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const uint64_t a = __shfl_xor_sync(0xffffffffu, lo, o);
+      const uint64_t b = __shfl_xor_sync(0xffffffffu, hi, o);
+      lo = a < lo ? a : lo;
+      hi = b > hi ? b : hi;
+    }
+    if (lane == 0) {
+      s_g[0] = lo;
+      s_g[1] = hi;
     }
   }
   __syncthreads();
-  lo = s_lo[0];
-  hi = s_hi[0];
-  __syncthreads();  // s_lo / s_hi are rewritten by the next call
+  lo = s_g[0];
+  hi = s_g[1];
 }
 
-// CTA 0's part: pivot, then the unit order and rejected bytes.  Every thread
-// of the block calls it; returns false (uniformly) if an invariant failed.
-__device__ bool mid_select_order(const double* __restrict__ score, int n_units, long long k,
-                                 uint64_t* keys, uint16_t* order, uint8_t* rej_u,
-                                 int32_t* status) {
+// kMulti = false: a cluster of one CTA, with block barriers and plain shared
+// memory in place of cluster barriers and distributed shared memory.
+template <bool kMulti>
+__global__ void __launch_bounds__(kSelThreads, 1)
+    select_cluster_kernel(const double* __restrict__ score, int n_units, int G, long long k,
+                          int32_t* accepted_ids, int32_t* rejected_ids, uint8_t* flags,
+                          int32_t* status) {
+  extern __shared__ __align__(16) unsigned char sel_smem[];
   __shared__ unsigned hist[kHistBins];
-  __shared__ uint64_t s_lo[kMidThreads / 32], s_hi[kMidThreads / 32];
+  __shared__ uint64_t s_wlo[kSelThreads / 32], s_whi[kSelThreads / 32];
+  __shared__ uint64_t s_mm[2], s_g[2];
+  __shared__ long long s_cnt[2];  // this CTA's keys equal to / above the pivot (peers read)
+  __shared__ long long s_off[2];  // ties and rejections in lower-ranked CTAs
   __shared__ int s_digit;
   __shared__ long long s_left;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int nc = static_cast<int>(cluster.num_blocks());
+  const int rank = static_cast<int>(cluster.block_rank());
   const int t = threadIdx.x;
-  const int lg = mid_per_log2(n_units);
+  const int B = (n_units + nc - 1) / nc;
+  const int base = rank * B;                        // first unit of this CTA
+  const int nb = max(0, min(B, n_units - base));    // units of this CTA
+  const int lg = sel_per_log2(B);
   const int per = 1 << lg;
+  uint64_t* keys = reinterpret_cast<uint64_t*>(sel_smem);
+  uint16_t* order = reinterpret_cast<uint16_t*>(sel_smem + static_cast<size_t>(per) * kSelRow *
+                                                               sizeof(uint64_t));
+  uint8_t* rej_u = reinterpret_cast<uint8_t*>(order + B);
   const int u0 = t * per;
-  const int n_mine = max(0, min(per, n_units - u0));
+  const int n_mine = max(0, min(per, nb - u0));
 
-  // coalesced loads: unit v (read by thread v % kMidThreads) belongs to thread
-  // v / per, slot v % per; rows of kMidRow keys make both this scatter (two-way)
-  // and the owners' row reads (none) nearly free of bank conflicts
-  for (int v = t; v < n_units; v += kMidThreads) {
-    const double x = score[v];
+  // coalesced loads: unit v (read by thread v % 1024) belongs to thread v / per,
+  // slot v % per; the padded rows make this scatter at most two-way conflicted
+  for (int v = t; v < nb; v += kSelThreads) {
+    const double x = score[base + v];
     if (isnan(x)) report(status, PACE_ERR_NAN_INPUT);
-    keys[(v & (per - 1)) * kMidRow + (v >> lg)] = order_key(x);
+    keys[(v & (per - 1)) * kSelRow + (v >> lg)] = order_key(x);
   }
   __syncthreads();
   uint64_t lo = ~0ull, hi = 0ull;
   for (int i = 0; i < n_mine; ++i) {
-    const uint64_t key = keys[i * kMidRow + t];
+    const uint64_t key = keys[i * kSelRow + t];
     lo = key < lo ? key : lo;
     hi = key > hi ? key : hi;
   }
   uint64_t prefix = 0ull, mask = 0ull;
   long long k_rem = k;
-  // each round fixes at least one more bit, so 64 rounds always suffice; the
-  // bound and the digit check only guard against a broken invariant
+  bool ok = true;
+  // Each round fixes at least one more bit, so 64 rounds always suffice; the
+  // bound and the digit check only guard against a broken invariant.  Every
+  // branch below depends only on cluster-wide values, so it is uniform.
   for (int round = 0;; ++round) {
-    block_min_max(lo, hi, s_lo, s_hi);  // every thread: the candidates' min and max
+    cluster_min_max<kMulti>(cluster, lo, hi, s_wlo, s_whi, s_mm, s_g);
     if (lo == hi) break;
     if (round >= 64) {
-      if (t == 0) report(status, PACE_ERR_INVALID_ARG);
-      return false;
+      ok = false;
+      break;
     }
     const int d = 63 - __clzll(static_cast<long long>(lo ^ hi));
     const int shift = d >= 10 ? d - 10 : 0;
     const int nbins = 1 << (d - shift + 1);
     mask = d == 63 ? 0ull : (~0ull << (d + 1));
     prefix = lo & mask;
-    for (int b = t; b < nbins; b += kMidThreads) hist[b] = 0u;
+    for (int b = t; b < nbins; b += kSelThreads) hist[b] = 0u;
     if (t == 0) s_digit = -1;
     __syncthreads();
     for (int i = 0; i < n_mine; ++i) {
-      const uint64_t key = keys[i * kMidRow + t];
+      const uint64_t key = keys[i * kSelRow + t];
       if ((key & mask) == prefix)
         atomicAdd(&hist[static_cast<unsigned>(key >> shift) & (nbins - 1)], 1u);
     }
-    __syncthreads();
-    // thread t owns digits nbins-1-2t and nbins-2-2t: an exclusive scan in thread
-    // order counts the candidates with larger digits
+    if (kMulti) cluster.sync();  // every CTA's histogram is complete
+    else __syncthreads();
+    // thread t owns digits nbins-1-2t and nbins-2-2t, summed over the cluster: an
+    // exclusive scan in thread order counts the candidates with larger digits
+    // (the loads of all peers are issued together: a fixed-bound loop the
+    // compiler unrolls, one distributed-shared-memory round trip per round)
     const int top = nbins - 1 - 2 * t;
-    const int h0 = top >= 0 ? static_cast<int>(hist[top]) : 0;
-    const int h1 = top >= 1 ? static_cast<int>(hist[top - 1]) : 0;
+    long long h0 = 0, h1 = 0;
+    if (kMulti) {
+      unsigned c0[kSelMaxCluster], c1[kSelMaxCluster];
+#pragma unroll
+      for (int r = 0; r < kSelMaxCluster; ++r) {
+        c0[r] = 0u;
+        c1[r] = 0u;
+        if (r < nc) {
+          const unsigned* ph = cluster.map_shared_rank(hist, static_cast<unsigned>(r));
+          if (top >= 0) c0[r] = ph[top];
+          if (top >= 1) c1[r] = ph[top - 1];
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < kSelMaxCluster; ++r) {
+        h0 += c0[r];
+        h1 += c1[r];
+      }
+    } else {
+      if (top >= 0) h0 = hist[top];
+      if (top >= 1) h1 = hist[top - 1];
+    }
     long long run = block_exclusive_scan<long long>(h0 + h1, nullptr);
     if (top >= 0 && run < k_rem && k_rem <= run + h0) {
       s_digit = top;
@@ -304,10 +389,11 @@ __device__ bool mid_select_order(const double* __restrict__ score, int n_units, 
       s_digit = top - 1;
       s_left = k_rem - run;
     }
-    __syncthreads();
-    if (s_digit < 0) {  // uniform: every thread reads the same word
-      if (t == 0) report(status, PACE_ERR_INVALID_ARG);
-      return false;
+    if (kMulti) cluster.sync();  // every CTA is done reading the histograms; s_digit is set
+    else __syncthreads();
+    if (s_digit < 0) {  // the same in every CTA: the histograms summed are the same
+      ok = false;
+      break;
     }
     prefix |= static_cast<uint64_t>(s_digit) << shift;
     mask |= static_cast<uint64_t>(nbins - 1) << shift;
@@ -315,76 +401,97 @@ __device__ bool mid_select_order(const double* __restrict__ score, int n_units, 
     lo = ~0ull;
     hi = 0ull;
     for (int i = 0; i < n_mine; ++i) {
-      const uint64_t key = keys[i * kMidRow + t];
+      const uint64_t key = keys[i * kSelRow + t];
       if ((key & mask) == prefix) {
         lo = key < lo ? key : lo;
         hi = key > hi ? key : hi;
       }
     }
   }
+  if (!ok && t == 0 && rank == 0) report(status, PACE_ERR_INVALID_ARG);
   const uint64_t pivot = lo;  // k_rem of the keys equal to it are rejected, lowest ids first
 
-  int eq = 0;
-  for (int i = 0; i < n_mine; ++i) eq += keys[i * kMidRow + t] == pivot;
-  const long long tie0 = block_exclusive_scan<long long>(eq, nullptr);
+  int eq = 0, gt = 0;
+  for (int i = 0; i < n_mine; ++i) {
+    const uint64_t key = keys[i * kSelRow + t];
+    eq += key == pivot;
+    gt += key > pivot;
+  }
+  long long cta_eq = 0, cta_gt = 0;
+  const long long tie_local = block_exclusive_scan<long long>(eq, &cta_eq);
+  block_exclusive_scan<long long>(gt, &cta_gt);
+  if (t == 0) {
+    s_cnt[0] = cta_eq;
+    s_cnt[1] = cta_gt;
+  }
+  if (kMulti) cluster.sync();  // every CTA's counts are written
+  else __syncthreads();
+  if (t == 0) {
+    long long ties_before = 0, rej_before = 0;
+    for (int r = 0; r < (kMulti ? rank : 0); ++r) {
+      const long long* pc = cluster.map_shared_rank(s_cnt, static_cast<unsigned>(r));
+      const long long e = pc[0];
+      long long take = k_rem - ties_before;  // ties of CTA r that are rejected
+      take = take < 0 ? 0 : (take > e ? e : take);
+      rej_before += pc[1] + take;
+      ties_before += e;
+    }
+    s_off[0] = ties_before;
+    s_off[1] = rej_before;
+  }
+  if (kMulti) cluster.sync();  // peers' counts are read: no CTA touches another's memory after this
+  else __syncthreads();
+  if (!ok) return;
+
+  const long long tie0 = s_off[0] + tie_local;
+  const long long rej_off = s_off[1];
   int nrej = 0;
   long long tie = tie0;
   for (int i = 0; i < n_mine; ++i) {
-    const uint64_t key = keys[i * kMidRow + t];
+    const uint64_t key = keys[i * kSelRow + t];
     nrej += key > pivot || (key == pivot && (tie++) < k_rem);
   }
-  long long rpos = block_exclusive_scan<long long>(nrej, nullptr);
-  const long long n_acc = n_units - k;
+  long long cta_rej = 0;
+  long long lrpos = block_exclusive_scan<long long>(nrej, &cta_rej);
+  const long long n_acc_cta = nb - cta_rej;
   tie = tie0;
   for (int i = 0; i < n_mine; ++i) {
-    const uint64_t key = keys[i * kMidRow + t];
+    const uint64_t key = keys[i * kSelRow + t];
     const bool r = key > pivot || (key == pivot && (tie++) < k_rem);
     const int u = u0 + i;
-    order[r ? n_acc + rpos : u - rpos] = static_cast<uint16_t>(u);
+    order[r ? n_acc_cta + lrpos : u - lrpos] = static_cast<uint16_t>(u);
     rej_u[u] = r ? 1 : 0;
-    rpos += r;
+    lrpos += r;
   }
-  return true;
-}
+  __syncthreads();
 
-__global__ void __launch_bounds__(kMidThreads, 1)
-    select_mid_kernel(const double* __restrict__ score, int n_units, int G, long long k,
-                      int32_t* accepted_ids, int32_t* rejected_ids, uint8_t* flags,
-                      int32_t* status) {
-  extern __shared__ __align__(16) unsigned char mid_smem[];
-  __shared__ int s_ok;
-  const int per = 1 << mid_per_log2(n_units);
-  uint64_t* keys = reinterpret_cast<uint64_t*>(mid_smem);
-  uint16_t* order =
-      reinterpret_cast<uint16_t*>(mid_smem + static_cast<size_t>(per) * kMidRow * sizeof(uint64_t));
-  uint8_t* rej_u = reinterpret_cast<uint8_t*>(order + n_units);
-  cg::cluster_group cluster = cg::this_cluster();
-  const unsigned rank = cluster.block_rank();
-  if (rank == 0) {  // uniform per block
-    const bool ok = mid_select_order(score, n_units, k, keys, order, rej_u, status);
-    if (threadIdx.x == 0) s_ok = ok ? 1 : 0;
+  // this CTA's runs: accepted ids from position (base - rej_off) * G, rejected
+  // ids from rej_off * G, flags from base * G.  Local position p of the CTA's
+  // [accepted | rejected] list holds trajectory (base + order[p / G]) * G + p % G;
+  // (q, r) = (p / G, p % G) is advanced by 1024 per step without dividing.
+  const int64_t n_out = static_cast<int64_t>(nb) * G;
+  const int64_t acc_end = n_acc_cta * G;
+  int32_t* acc_run = accepted_ids + (static_cast<int64_t>(base) - rej_off) * G;
+  int32_t* rej_run = rejected_ids ? rejected_ids + rej_off * G : nullptr;
+  const int sq = kSelThreads / G, sr = kSelThreads % G;
+  int q = t / G, r = t % G;
+  for (int64_t p = t; p < n_out; p += kSelThreads) {
+    const int32_t id = (base + static_cast<int32_t>(order[q])) * G + r;
+    if (p < acc_end) acc_run[p] = id;
+    else if (rej_run) rej_run[p - acc_end] = id;
+    q += sq;
+    r += sr;
+    if (r >= G) {
+      r -= G;
+      ++q;
+    }
   }
-  cluster.sync();  // CTA 0's list is complete and visible to the cluster
-
-  const uint16_t* order0 = cluster.map_shared_rank(order, 0);
-  const uint8_t* rej0 = cluster.map_shared_rank(rej_u, 0);
-  if (*cluster.map_shared_rank(&s_ok, 0)) {  // uniform: one word read by every thread
-    const int64_t total = static_cast<int64_t>(n_units) * G;
-    const int nc = static_cast<int>(cluster.num_blocks());
-    const int64_t chunk = (total + nc - 1) / nc;
-    const int64_t p0 = static_cast<int64_t>(rank) * chunk;
-    const int64_t p1 = min(total, p0 + chunk);
-    const int64_t acc_end = (static_cast<int64_t>(n_units) - k) * G;
-    const int sq = kMidThreads / G, sr = kMidThreads % G;
-    // position p of the concatenated output [accepted ids | rejected ids] holds
-    // trajectory order0[p / G] * G + p % G; (q, r) = (p / G, p % G) is advanced
-    // by kMidThreads per step without dividing
-    int64_t p = p0 + threadIdx.x;
-    int q = static_cast<int>(p / G), r = static_cast<int>(p % G);
-    for (; p < p1; p += kMidThreads) {
-      const int32_t id = static_cast<int32_t>(order0[q]) * G + r;
-      if (p < acc_end) accepted_ids[p] = id;
-      else if (rejected_ids) rejected_ids[p - acc_end] = id;
+  if (flags) {
+    uint8_t* f_run = flags + static_cast<int64_t>(base) * G;
+    q = t / G;
+    r = t % G;
+    for (int64_t p = t; p < n_out; p += kSelThreads) {
+      f_run[p] = rej_u[q] ? 0 : 1;
       q += sq;
       r += sr;
       if (r >= G) {
@@ -392,22 +499,7 @@ __global__ void __launch_bounds__(kMidThreads, 1)
         ++q;
       }
     }
-    if (flags) {  // flag of trajectory p: its unit p / G accepted or not
-      p = p0 + threadIdx.x;
-      q = static_cast<int>(p / G);
-      r = static_cast<int>(p % G);
-      for (; p < p1; p += kMidThreads) {
-        flags[p] = rej0[q] ? 0 : 1;
-        q += sq;
-        r += sr;
-        if (r >= G) {
-          r -= G;
-          ++q;
-        }
-      }
-    }
   }
-  cluster.sync();  // CTA 0's shared memory stays until every CTA has read it
 }
 
 // Pass `pass` of the MSB-first radix select (256 threads per block).  The state
@@ -589,10 +681,10 @@ SelectWs carve_select_ws(Carver& cv, int64_t n_units) {
   return w;
 }
 
-// Opts select_mid_kernel into its largest dynamic shared memory and finds the
-// largest cluster (8, 4, 2 or 1 CTAs) of such blocks the current device can
+// Opts select_cluster_kernel into its largest dynamic shared memory and finds
+// the largest cluster (8, 4, 2 or 1 CTAs) of such blocks the current device can
 // hold, once per device.
-pace_status mid_cluster_limit(int* out) {
+pace_status sel_cluster_limit(int* out) {
   constexpr int kMaxDevices = 64;
   static int limit[kMaxDevices] = {};
   static std::mutex mu;
@@ -601,15 +693,18 @@ pace_status mid_cluster_limit(int* out) {
   if (dev < 0 || dev >= kMaxDevices) return PACE_ERR_CUDA;
   std::lock_guard<std::mutex> g(mu);
   if (limit[dev] == 0) {
-    const size_t smem = mid_smem_bytes(kMidMax);
-    PACE_TRY_CUDA(cudaFuncSetAttribute(select_mid_kernel,
+    const size_t smem = sel_smem_bytes(kSelCtaUnits);
+    PACE_TRY_CUDA(cudaFuncSetAttribute(select_cluster_kernel<true>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem)));
-    int c = kMidMaxCluster;
+    PACE_TRY_CUDA(cudaFuncSetAttribute(select_cluster_kernel<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem)));
+    int c = kSelMaxCluster;
     for (; c > 1; c /= 2) {
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(static_cast<unsigned>(c), 1, 1);
-      cfg.blockDim = dim3(kMidThreads, 1, 1);
+      cfg.blockDim = dim3(kSelThreads, 1, 1);
       cfg.dynamicSmemBytes = smem;
       cudaLaunchAttribute attr;
       attr.id = cudaLaunchAttributeClusterDimension;
@@ -619,7 +714,8 @@ pace_status mid_cluster_limit(int* out) {
       cfg.attrs = &attr;
       cfg.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, select_mid_kernel, &cfg) == cudaSuccess && n >= 1)
+      if (cudaOccupancyMaxActiveClusters(&n, select_cluster_kernel<true>, &cfg) == cudaSuccess &&
+          n >= 1)
         break;
       (void)cudaGetLastError();  // a refused size is not an error of this call
     }
@@ -629,19 +725,25 @@ pace_status mid_cluster_limit(int* out) {
   return PACE_OK;
 }
 
-// One cluster: 1 CTA up to 16,384 outputs, then one more SM per doubling, up to 8.
-pace_status launch_select_mid(const double* unit_score, int n_units, int G, long long k,
-                              int32_t* accepted_ids, int32_t* rejected_ids, uint8_t* flags,
-                              int32_t* status, cudaStream_t st) {
-  int limit = 1;
-  PACE_TRY(mid_cluster_limit(&limit));
-  const int64_t total = static_cast<int64_t>(n_units) * G;
+// Cluster size for U units of G trajectories: enough CTAs to hold the keys
+// (16,384 each) and one more SM per doubling of the outputs above 16,384, up to
+// the device's limit; 0 when the keys do not fit the largest cluster.
+int sel_cluster_size(int64_t n_units, int G, int limit) {
+  const int64_t total = n_units * G;
   int c = 1;
-  while (c < limit && total > static_cast<int64_t>(c) * 16384) c *= 2;
+  while (c < limit && (n_units > static_cast<int64_t>(c) * kSelCtaUnits ||
+                       total > static_cast<int64_t>(c) * 16384))
+    c *= 2;
+  return n_units <= static_cast<int64_t>(c) * kSelCtaUnits ? c : 0;
+}
+
+pace_status launch_select_cluster(const double* unit_score, int n_units, int G, long long k,
+                                  int c, int32_t* accepted_ids, int32_t* rejected_ids,
+                                  uint8_t* flags, int32_t* status, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(c), 1, 1);
-  cfg.blockDim = dim3(kMidThreads, 1, 1);
-  cfg.dynamicSmemBytes = mid_smem_bytes(n_units);
+  cfg.blockDim = dim3(kSelThreads, 1, 1);
+  cfg.dynamicSmemBytes = sel_smem_bytes((n_units + c - 1) / c);
   cfg.stream = st;
   cudaLaunchAttribute attr;
   attr.id = cudaLaunchAttributeClusterDimension;
@@ -650,8 +752,13 @@ pace_status launch_select_mid(const double* unit_score, int n_units, int G, long
   attr.val.clusterDim.z = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  PACE_TRY_CUDA(cudaLaunchKernelEx(&cfg, select_mid_kernel, unit_score, n_units, G, k,
-                                   accepted_ids, rejected_ids, flags, status));
+  if (c > 1) {
+    PACE_TRY_CUDA(cudaLaunchKernelEx(&cfg, select_cluster_kernel<true>, unit_score, n_units, G,
+                                     k, accepted_ids, rejected_ids, flags, status));
+  } else {
+    PACE_TRY_CUDA(cudaLaunchKernelEx(&cfg, select_cluster_kernel<false>, unit_score, n_units, G,
+                                     k, accepted_ids, rejected_ids, flags, status));
+  }
   return last_launch_status();
 }
 
@@ -737,9 +844,15 @@ extern "C" pace_status pace_select_k(const double* unit_score, int64_t n_units, 
                                                      status_dev);
     return last_launch_status();
   }
-  if (n_units <= kMidMax)
-    return launch_select_mid(unit_score, static_cast<int>(n_units), G, static_cast<long long>(k),
-                             accepted_ids, rejected_ids, traj_accepted, status_dev, st);
+  if (n_units <= kSelMaxUnits) {
+    int limit = 1;
+    PACE_TRY(sel_cluster_limit(&limit));
+    const int c = sel_cluster_size(n_units, G, limit);
+    if (c > 0)
+      return launch_select_cluster(unit_score, static_cast<int>(n_units), G,
+                                   static_cast<long long>(k), c, accepted_ids, rejected_ids,
+                                   traj_accepted, status_dev, st);
+  }
   if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
   Carver cv(workspace, workspace_bytes);
   SelectWs ws = carve_select_ws(cv, n_units);

@@ -28,10 +28,10 @@ def _check_k(scores, G, k):
     np.testing.assert_array_equal(flags, oflag)
 
 
-# 1..512 units: the one-block rank kernel; 513..16384: the one-block adaptive
-# radix select; above: the multi-block radix select.
-@pytest.mark.parametrize("U", [1, 2, 7, 64, 511, 512, 513, 2048, 5000, 16384, 16385, 131072,
-                               1048576])
+# 1..512 units: the one-block rank kernel; 513..131072: the one-cluster adaptive
+# radix select (1-8 CTAs); above: the multi-block radix select.
+@pytest.mark.parametrize("U", [1, 2, 7, 64, 511, 512, 513, 2048, 5000, 16384, 16385, 70001,
+                               131072, 131073, 1048576])
 @pytest.mark.parametrize("dist", ["ties", "continuous", "constant", "ulps", "signed_wide"])
 def test_select_k_matches_oracle(U, dist):
     rng = np.random.default_rng(U + len(dist))
@@ -117,3 +117,14 @@ def test_mid_size_pools_take_no_workspace(U):
     np.testing.assert_array_equal(as_np(acc)[:(U - k) * G], oacc)
     np.testing.assert_array_equal(as_np(rej)[:k * G], orej)
     np.testing.assert_array_equal(as_np(flags), oflag)
+
+
+@pytest.mark.parametrize("U,G", [(600, 3), (3000, 12), (3000, 100), (5000, 7), (16384, 3),
+                                 (700, 1500)])
+def test_select_group_sizes(U, G):
+    """Group sizes that do and do not divide 1024 (the writers step through
+    positions 1024 at a time), clusters of 1 to 8 CTAs on the one-launch path."""
+    rng = np.random.default_rng(U * 31 + G)
+    s = rng.integers(0, 200, size=U).astype(np.float64) / 16.0
+    for k in (1, U // 4, U - 1):
+        _check_k(s, G, k)
