@@ -39,7 +39,7 @@ namespace cg = cooperative_groups;
 constexpr int kSmallMax = 512;
 constexpr int kSmallThreads = 512;
 constexpr int kHistBins = 2048;
-constexpr int kTile = 256;  // units per compaction block (enough blocks to fill the GPU at 16k units)
+constexpr int kTile = 256;  // units per compaction block of the radix path
 constexpr int kTileThreads = 256;
 constexpr int kPerThread = kTile / kTileThreads;
 constexpr int kPasses = 6;

@@ -128,3 +128,30 @@ def test_select_group_sizes(U, G):
     s = rng.integers(0, 200, size=U).astype(np.float64) / 16.0
     for k in (1, U // 4, U - 1):
         _check_k(s, G, k)
+
+
+@pytest.mark.parametrize("U,G", [(5000, 2), (70000, 1), (300000, 1)])
+def test_select_without_optional_outputs(U, G):
+    """rejected_ids and traj_accepted may be NULL: the accepted ids alone, on the
+    one-CTA, multi-CTA and radix paths."""
+    import ctypes
+    rng = np.random.default_rng(U + 3)
+    s = rng.random(U) * 30.0
+    k = U // 5
+    scores = to_dev(s)
+    acc = torch.full((U * G,), -7, dtype=torch.int32, device=DEV)
+    L = pace.lib()
+    ws = pace.workspace(L.pace_select_workspace_size(U), DEV)
+    status = pace.new_status(DEV)
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    st = L.pace_select_k(ctypes.c_void_p(scores.data_ptr()), U, G, k,
+                         ctypes.c_void_p(acc.data_ptr()), None, None,
+                         ctypes.c_void_p(ws.data_ptr()), ws.numel(),
+                         ctypes.c_void_p(status.data_ptr()), stream)
+    assert st == pace.OK, pace.status_string(st)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    _, oacc, _, _ = oracle.select(s, G, k)
+    got = as_np(acc)
+    np.testing.assert_array_equal(got[:(U - k) * G], oacc)
+    assert (got[(U - k) * G:] == -7).all()  # nothing written past the accepted ids
