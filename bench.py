@@ -39,10 +39,11 @@ WORKLOAD = "math7b"
 # DRAM bytes per unit from the committed ncu captures of the current kernels, by the LM head's
 # vocabulary split count (profiles/lmhead_lse_kernel_one_wave.md: 4 splits, 1.130 GB for one
 # full round of 4864 rows, W read once per round, so traffic grows with the rows processed;
-# 2 splits, 18.87 GB for four rounds of 9728 rows; profiles/tag_reduce_kernel_sweep16k.md:
-# 223.4 MB for 54.93 M tags).  Set to None when a kernel changes until it is captured again.
+# 2 splits, 18.87 GB for four rounds of 9728 rows; profiles/tag_reduce_kernel_sweep1m.md:
+# 14.0856 GB read + written for 3.5023 G tags).  Set to None when a kernel changes until it is
+# captured again.
 LMHEAD_DRAM_BYTES_PER_ROW = {4: 1.12978e9 / 4864, 2: 18.8672e9 / 38912}
-TAG_REDUCE_DRAM_BYTES_PER_TAG = 223.412e6 / 54929421
+TAG_REDUCE_DRAM_BYTES_PER_TAG = (14065824512 + 19798528) / 3502330341
 SWEEP_N = 1048576
 SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)
 METRIC = "accepted tokens/sec (logprob+loss) and % bf16 tensor peak; pool scoring traj/s + HBM GB/s"
