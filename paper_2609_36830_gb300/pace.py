@@ -111,6 +111,8 @@ class PaceError(RuntimeError):
 def lib():
     """The loaded libpace.so (raises if it has not been built)."""
     global _lib
+    if _lib is not None:
+        return _lib
     with _lock:
         if _lib is None:
             if not os.path.exists(LIB_PATH):
@@ -162,9 +164,18 @@ _U8, _I32T, _I64T = torch.uint8, torch.int32, torch.int64
 _F32T, _F64T, _BF16 = torch.float32, torch.float64, torch.bfloat16
 
 
+# The current stream's handle without building a torch.cuda.Stream object (0.08 us
+# against ~3 us per call, a tenth of a small pool's scoring call); the public
+# call is the fallback where torch does not provide it.
+_raw_current_stream = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
 def _stream(stream=None):
-    s = stream if stream is not None else torch.cuda.current_stream()
-    return ctypes.c_void_p(s.cuda_stream)
+    if stream is not None:
+        return ctypes.c_void_p(stream.cuda_stream)
+    if _raw_current_stream is not None:
+        return ctypes.c_void_p(_raw_current_stream(torch.cuda.current_device()))
+    return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
 
 
 def workspace(nbytes: int, device) -> torch.Tensor:
