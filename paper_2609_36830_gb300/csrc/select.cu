@@ -285,7 +285,7 @@ template <bool kMulti>
 __global__ void __launch_bounds__(kSelThreads, 1)
     select_cluster_kernel(const double* __restrict__ score, int n_units, int G, long long k,
                           int32_t* accepted_ids, int32_t* rejected_ids, uint8_t* flags,
-                          int32_t* status) {
+                          int32_t* status, int vec4) {
   extern __shared__ __align__(16) unsigned char sel_smem[];
   __shared__ unsigned hist[kHistBins];
   __shared__ uint64_t s_wlo[kSelThreads / 32], s_whi[kSelThreads / 32];
@@ -473,6 +473,46 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   const int64_t acc_end = n_acc_cta * G;
   int32_t* acc_run = accepted_ids + (static_cast<int64_t>(base) - rej_off) * G;
   int32_t* rej_run = rejected_ids ? rejected_ids + rej_off * G : nullptr;
+  if (vec4) {
+    // G % 4 == 0, id lists 16-byte and flags 4-byte aligned (checked on the
+    // host): four consecutive ids (one int4) and four flags (one 32-bit word)
+    // per store, an eighth of the scalar writer's instructions at G = 8.  Every
+    // run starts at a multiple of 4 entries.
+    const int G4 = G / 4;
+    const int64_t n_out4 = static_cast<int64_t>(nb) * G4;
+    const int64_t acc_end4 = n_acc_cta * G4;
+    int4* acc4 = reinterpret_cast<int4*>(acc_run);
+    int4* rej4 = reinterpret_cast<int4*>(rej_run);
+    const int sq4 = kSelThreads / G4, sr4 = kSelThreads % G4;
+    int q = t / G4, r = t % G4;
+    for (int64_t p = t; p < n_out4; p += kSelThreads) {
+      const int32_t id = (base + static_cast<int32_t>(order[q])) * G + 4 * r;
+      const int4 v = make_int4(id, id + 1, id + 2, id + 3);
+      if (p < acc_end4) acc4[p] = v;
+      else if (rej4) rej4[p - acc_end4] = v;
+      q += sq4;
+      r += sr4;
+      if (r >= G4) {
+        r -= G4;
+        ++q;
+      }
+    }
+    if (flags) {
+      uint32_t* f4 = reinterpret_cast<uint32_t*>(flags + static_cast<int64_t>(base) * G);
+      q = t / G4;
+      r = t % G4;
+      for (int64_t p = t; p < n_out4; p += kSelThreads) {
+        f4[p] = rej_u[q] ? 0u : 0x01010101u;
+        q += sq4;
+        r += sr4;
+        if (r >= G4) {
+          r -= G4;
+          ++q;
+        }
+      }
+    }
+    return;
+  }
   const int sq = kSelThreads / G, sr = kSelThreads % G;
   int q = t / G, r = t % G;
   for (int64_t p = t; p < n_out; p += kSelThreads) {
@@ -752,12 +792,14 @@ pace_status launch_select_cluster(const double* unit_score, int n_units, int G, 
   attr.val.clusterDim.z = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
+  const int vec4 = G % 4 == 0 && aligned(accepted_ids, 16) &&
+                   (!rejected_ids || aligned(rejected_ids, 16)) && (!flags || aligned(flags, 4));
   if (c > 1) {
     PACE_TRY_CUDA(cudaLaunchKernelEx(&cfg, select_cluster_kernel<true>, unit_score, n_units, G,
-                                     k, accepted_ids, rejected_ids, flags, status));
+                                     k, accepted_ids, rejected_ids, flags, status, vec4));
   } else {
     PACE_TRY_CUDA(cudaLaunchKernelEx(&cfg, select_cluster_kernel<false>, unit_score, n_units, G,
-                                     k, accepted_ids, rejected_ids, flags, status));
+                                     k, accepted_ids, rejected_ids, flags, status, vec4));
   }
   return last_launch_status();
 }

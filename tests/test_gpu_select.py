@@ -155,3 +155,61 @@ def test_select_without_optional_outputs(U, G):
     got = as_np(acc)
     np.testing.assert_array_equal(got[:(U - k) * G], oacc)
     assert (got[(U - k) * G:] == -7).all()  # nothing written past the accepted ids
+
+
+def test_select_random_shapes():
+    """Random pool sizes across the one-launch range (513..131,072 units, clusters of
+    1-8 CTAs), random group sizes, budgets and score distributions: ids exact."""
+    rng = np.random.default_rng(2026)
+    for case in range(40):
+        U = int(rng.integers(513, 131073)) if case % 4 else int(rng.integers(513, 4096))
+        G = int(rng.choice([1, 2, 3, 8, 12]))
+        if U * G > 600_000:
+            G = 1
+        kind = case % 5
+        if kind == 0:
+            s = rng.random(U) * 40.0
+        elif kind == 1:
+            s = rng.integers(0, 12, size=U).astype(np.float64) / 8.0
+        elif kind == 2:
+            s = np.round(rng.normal(10.0, 3.0, size=U), 3)
+        elif kind == 3:
+            s = rng.choice([0.0, 1.5, 1.5 + 2.0 ** -40, 7.25], size=U)
+        else:
+            s = np.exp(rng.normal(0.0, 20.0, size=U))
+        k = int(rng.integers(1, U))
+        _check_k(s, G, k)
+
+
+@pytest.mark.parametrize("U,G", [(3000, 4), (3000, 8), (20000, 12), (131072, 8)])
+def test_select_outputs_at_unaligned_addresses(U, G):
+    """Groups that are a multiple of 4 are written four ids at a time when the
+    buffers allow it; buffers 4 bytes (ids) or 1 byte (flags) off alignment take
+    the element-wise writer.  Both give the oracle's ids."""
+    import ctypes
+    rng = np.random.default_rng(U * 7 + G)
+    s = rng.integers(0, 300, size=U).astype(np.float64) / 4.0
+    k = U // 3
+    n = U * G
+    scores = to_dev(s)
+    acc = torch.full((n + 4,), -7, dtype=torch.int32, device=DEV)
+    rej = torch.full((n + 4,), -7, dtype=torch.int32, device=DEV)
+    flags = torch.full((n + 4,), 9, dtype=torch.uint8, device=DEV)
+    status = pace.new_status(DEV)
+    L = pace.lib()
+    ws = pace.workspace(L.pace_select_workspace_size(U), DEV)
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    for off_ids, off_flags in ((0, 0), (1, 0), (0, 1)):
+        st = L.pace_select_k(ctypes.c_void_p(scores.data_ptr()), U, G, k,
+                             ctypes.c_void_p(acc.data_ptr() + 4 * off_ids),
+                             ctypes.c_void_p(rej.data_ptr() + 4 * off_ids),
+                             ctypes.c_void_p(flags.data_ptr() + off_flags),
+                             ctypes.c_void_p(ws.data_ptr()), ws.numel(),
+                             ctypes.c_void_p(status.data_ptr()), stream)
+        assert st == pace.OK, pace.status_string(st)
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0
+        _, oacc, orej, oflag = oracle.select(s, G, k)
+        np.testing.assert_array_equal(as_np(acc)[off_ids:off_ids + (U - k) * G], oacc)
+        np.testing.assert_array_equal(as_np(rej)[off_ids:off_ids + k * G], orej)
+        np.testing.assert_array_equal(as_np(flags)[off_flags:off_flags + n], oflag)
