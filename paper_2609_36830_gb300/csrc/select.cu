@@ -184,7 +184,11 @@ __global__ void __launch_bounds__(kSmallThreads)
 // counts of the lower-ranked CTAs (ties are rejected lowest id first), lists
 // its accepted units and then its rejected units in shared memory, and writes
 // its own contiguous runs of the id lists and flags, consecutive threads at
-// consecutive positions (whole 32-byte sectors per warp store).
+// consecutive positions (whole 32-byte sectors per warp store), four ids and
+// four flags per store when G is a multiple of 4 and the buffers are aligned.
+// C is the smallest power of two that keeps each CTA at 16,384 units and
+// 16,384 outputs or fewer; a cluster of one uses block barriers and plain
+// shared memory instead (the kMulti = false instance).
 constexpr int kSelCtaUnits = 16384;  // units per CTA at most
 constexpr int kSelThreads = 1024;
 constexpr int kSelPer = kSelCtaUnits / kSelThreads;  // units per thread at most
