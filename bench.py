@@ -835,6 +835,23 @@ def run_case(args):
         tf = 3 * 2.0 * rows * H * V / (ms / 1e3) / 1e12
         print(json.dumps({"case": "lmhead_bwd", "rows": rows, "H": H, "V": V, "ms": ms,
                           "tflops": tf}), flush=True)
+    elif args.case == "select":
+        # pace_select_k alone: --case-units unit scores drawn uniformly in [0, 30),
+        # groups of 8, half the units rejected
+        U = args.case_units
+        gen = torch.Generator(device=device)
+        gen.manual_seed(104)
+        scores = torch.rand(U, generator=gen, device=device, dtype=torch.float64) * 30.0
+        out = {"accepted": torch.empty(U * 8, dtype=torch.int32, device=device),
+               "rejected": torch.empty(U * 8, dtype=torch.int32, device=device),
+               "flags": torch.empty(U * 8, dtype=torch.uint8, device=device)}
+        ws = pace.workspace(pace.lib().pace_select_workspace_size(U), device)
+        status = pace.new_status(device)
+        ms = _timed(lambda: pace.select_k(scores, 8, U // 2, out=out, ws=ws, status=status),
+                    args.steps, args.warmup)
+        assert int(status.item()) == 0
+        print(json.dumps({"case": "select", "units": U, "group_size": 8, "ms_per_call": ms}),
+              flush=True)
     elif args.case == "pool":
         # pace_score_pool + pace_select on one sweep pool, L2 evicted before each call,
         # eagerly and as one CUDA-graph replay
@@ -876,12 +893,14 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=512)
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce", "step_tiny", "pool"],
+    ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce", "step_tiny", "pool",
+                                       "select"],
                     default=None,
                     help="time one kernel on a small case (profiler captures)")
     ap.add_argument("--case-rows", type=int, default=4864)
     ap.add_argument("--case-workload", default=WORKLOAD, choices=["math7b", "multiturn", "moe"])
     ap.add_argument("--case-traj", type=int, default=16384)
+    ap.add_argument("--case-units", type=int, default=131072)
     ap.add_argument("--case-splits", type=int, default=0,
                     help="LM-head vocabulary splits for --case lmhead (0 = automatic)")
     args = ap.parse_args()
