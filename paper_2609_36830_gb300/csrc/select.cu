@@ -211,13 +211,11 @@ __host__ __device__ inline size_t sel_smem_bytes(int b) {
          static_cast<size_t>(b) * (sizeof(uint16_t) + 1);
 }
 
-// Minimum and maximum of (lo, hi) over every thread of every CTA of the
-// cluster; the result is in every thread.  s_mm is this CTA's slot that peers
-// read; s_g holds the cluster result for this CTA's threads.
-template <bool kMulti>
-__device__ __forceinline__ void cluster_min_max(cg::cluster_group& cluster, uint64_t& lo,
-                                                uint64_t& hi, uint64_t* s_wlo, uint64_t* s_whi,
-                                                uint64_t* s_mm, uint64_t* s_g) {
+// This CTA's minimum and maximum of (lo, hi) over its threads, written to its
+// slot s_mm (read by the other CTAs).  Every thread of the block must call it;
+// the caller's next block or cluster barrier publishes the slot.
+__device__ __forceinline__ void cta_min_max_to_slot(uint64_t lo, uint64_t hi, uint64_t* s_wlo,
+                                                    uint64_t* s_whi, uint64_t* s_mm) {
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -244,19 +242,22 @@ __device__ __forceinline__ void cluster_min_max(cg::cluster_group& cluster, uint
     if (lane == 0) {
       s_mm[0] = lo;
       s_mm[1] = hi;
-      if (!kMulti) {  // one CTA: its result is the cluster's
-        s_g[0] = lo;
-        s_g[1] = hi;
-      }
     }
   }
-  if (!kMulti) {
-    __syncthreads();
-    lo = s_g[0];
-    hi = s_g[1];
+}
+
+// The cluster's minimum and maximum from the CTAs' published slots, in every
+// thread.  Every thread of the block must call it, after the barrier that
+// published the slots.
+template <bool kMulti>
+__device__ __forceinline__ void cluster_fold_slots(cg::cluster_group& cluster, uint64_t& lo,
+                                                   uint64_t& hi, uint64_t* s_mm, uint64_t* s_g) {
+  if (!kMulti) {  // one CTA: its slot is the result
+    lo = s_mm[0];
+    hi = s_mm[1];
     return;
   }
-  cluster.sync();  // every CTA's slot is written
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   if (wid == 0) {  // lanes < C read the peers' slots; one warp folds them
     const int nc = static_cast<int>(cluster.num_blocks());
     lo = ~0ull;
@@ -334,8 +335,15 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   // Each round fixes at least one more bit, so 64 rounds always suffice; the
   // bound and the digit check only guard against a broken invariant.  Every
   // branch below depends only on cluster-wide values, so it is uniform.
+  // Two cluster barriers per round: one after the histograms, and one that
+  // both ends the reading of the histograms and publishes the next round's
+  // minimum / maximum slots (written only after every CTA has passed the
+  // histogram barrier, so after every CTA has read the previous values).
+  cta_min_max_to_slot(lo, hi, s_wlo, s_whi, s_mm);
+  if (kMulti) cluster.sync();
+  else __syncthreads();
   for (int round = 0;; ++round) {
-    cluster_min_max<kMulti>(cluster, lo, hi, s_wlo, s_whi, s_mm, s_g);
+    cluster_fold_slots<kMulti>(cluster, lo, hi, s_mm, s_g);
     if (lo == hi) break;
     if (round >= 64) {
       ok = false;
@@ -393,8 +401,7 @@ __global__ void __launch_bounds__(kSelThreads, 1)
       s_digit = top - 1;
       s_left = k_rem - run;
     }
-    if (kMulti) cluster.sync();  // every CTA is done reading the histograms; s_digit is set
-    else __syncthreads();
+    __syncthreads();  // s_digit and s_left are set
     if (s_digit < 0) {  // the same in every CTA: the histograms summed are the same
       ok = false;
       break;
@@ -411,6 +418,9 @@ __global__ void __launch_bounds__(kSelThreads, 1)
         hi = key > hi ? key : hi;
       }
     }
+    cta_min_max_to_slot(lo, hi, s_wlo, s_whi, s_mm);
+    if (kMulti) cluster.sync();  // histograms read everywhere; the new slots published
+    else __syncthreads();
   }
   if (!ok && t == 0 && rank == 0) report(status, PACE_ERR_INVALID_ARG);
   const uint64_t pivot = lo;  // k_rem of the keys equal to it are rejected, lowest ids first
