@@ -25,8 +25,15 @@ namespace {
 
 constexpr int kReduceThreads = 256;  // 8 warps
 constexpr int kTileTokens = 128;     // one int4 per lane
-constexpr int kTilesPerBatch = 8;    // 1024 tokens (4 KB) per warp batch in flight
-constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
+// Tiles per warp batch (128 tokens each) and resident blocks per SM, by pool
+// size.  Large pools: 8 tiles (1024 tokens, 4 KB in flight per register set),
+// 126 registers, 2 blocks per SM.  Pools of up to kSmallPoolTokens tags: 4
+// tiles, 79 registers, 3 blocks per SM; more warps with half the work each
+// shorten the ramp and the tail where those dominate (16k sweep pool, 55 M
+// tags: 62 -> 52 us), and cost ~0.5 % on long streams (128k and 1M pools).
+constexpr int kTilesLarge = 8, kBlocksLarge = 2;
+constexpr int kTilesSmall = 4, kBlocksSmall = 3;
+constexpr int64_t kSmallPoolTokens = int64_t(1) << 27;
 constexpr int kMaxWindow = 4096;
 constexpr int64_t kTableMinTraj = 32768;  // pools from this size sort W and tabulate F
 
@@ -97,6 +104,7 @@ __device__ __forceinline__ bool small_policy(int bits_or) {
 // Sum, count and max of a batch that lies inside one trajectory and holds only
 // policy tags below 2^26.  Returns false (and leaves acc untouched) when the
 // batch needs the per-group path.
+template <int kTilesPerBatch>
 __device__ __forceinline__ bool acc_batch_fast(LaneAcc& a, const int4 (&v)[kTilesPerBatch]) {
   int o = 0, mx = 0, s = 0;
 #pragma unroll
@@ -128,15 +136,17 @@ __device__ __forceinline__ void acc_group(LaneAcc& a, const int4& q) {
   }
 }
 
-// Each warp owns a contiguous range of 1024-token batches of the flattened
-// tag stream and walks the CSR offsets forward through it, so trajectories of
+// Each warp owns a contiguous range of batches (kTilesPerBatch x 128 tokens) of
+// the flattened tag stream and walks the CSR offsets forward through it, so trajectories of
 // any length mix are balanced across warps.  The walk never leaves
 // [0, n_traj) and loads only tags[0, n_tokens), whatever the offsets hold;
 // inconsistent offsets are reported by the finalize kernel.
-__global__ void __launch_bounds__(kReduceThreads, 2)
+template <int kTilesPerBatch, int kMinBlocks>
+__global__ void __launch_bounds__(kReduceThreads, kMinBlocks)
     tag_reduce_kernel(const int32_t* __restrict__ tags, const int64_t* __restrict__ offsets,
                       int64_t n_traj, int64_t n_tokens, unsigned long long* __restrict__ sumv,
                       unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1) {
+  constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t n_warps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -210,7 +220,7 @@ __global__ void __launch_bounds__(kReduceThreads, 2)
       const int64_t seg_hi = cur_end < bt1 ? cur_end : bt1;
       if (pos == bt0 && seg_hi == bt0 + kBatchTokens) {
         // whole batch inside one trajectory: no position tests
-        if (!acc_batch_fast(acc, v)) {
+        if (!acc_batch_fast<kTilesPerBatch>(acc, v)) {
 #pragma unroll
           for (int u = 0; u < kTilesPerBatch; ++u) acc_group(acc, v[u]);
         }
@@ -519,15 +529,25 @@ pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t 
                            int64_t n_tokens, const ScoreWs& ws, cudaStream_t st) {
   PACE_TRY_CUDA(cudaMemsetAsync(ws.sumv, 0, static_cast<size_t>(n_traj) * 16, st));
   if (n_tokens == 0) return PACE_OK;
-  const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
+  const bool small = n_tokens <= kSmallPoolTokens;
+  const int tiles = small ? kTilesSmall : kTilesLarge;
+  const int per_sm = small ? kBlocksSmall : kBlocksLarge;
+  const int64_t batch_tokens = static_cast<int64_t>(kTileTokens) * tiles;
+  const int64_t n_batches = (n_tokens + batch_tokens - 1) / batch_tokens;
   const int warps_per_block = kReduceThreads / 32;
   int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
-  const int64_t cap = static_cast<int64_t>(sm_count()) * 2;  // one wave at 2 blocks / SM
+  const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;  // one wave
   if (blocks > cap) blocks = cap;
   const ProfileEvents& pe = profile_events(PACE_PROFILE_TAG_REDUCE);
   if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
-  tag_reduce_kernel<<<static_cast<unsigned>(blocks), kReduceThreads, 0, st>>>(
-      tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1);
+  if (small)
+    tag_reduce_kernel<kTilesSmall, kBlocksSmall><<<static_cast<unsigned>(blocks), kReduceThreads,
+                                                   0, st>>>(tags, offsets, n_traj, n_tokens,
+                                                            ws.sumv, ws.cnt, ws.maxp1);
+  else
+    tag_reduce_kernel<kTilesLarge, kBlocksLarge><<<static_cast<unsigned>(blocks), kReduceThreads,
+                                                   0, st>>>(tags, offsets, n_traj, n_tokens,
+                                                            ws.sumv, ws.cnt, ws.maxp1);
   PACE_TRY(last_launch_status());
   if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
   return PACE_OK;
