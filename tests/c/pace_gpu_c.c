@@ -3,17 +3,21 @@
  * device memory comes from cudaMalloc, every call takes the legacy default
  * stream.
  *
- *   pace_gpu_c <input file> <output file>
+ *   pace_gpu_c <input file> <output file> <eps_low> <eps_high>
  *
  * Input (little-endian): int64 n_traj, n_tokens, n_rows, hidden, vocab,
  * window_len, group_size, n_target, trainer_version; then tags int32[n_tokens],
  * offsets int64[n_traj+1], c_version int32[n_traj], s_pre float32[n_traj],
  * window float32[window_len], row_offsets int64[n_traj+1], mask uint8[n_rows],
  * targets int32[n_rows], hidden bf16 bits uint16[n_rows*hidden], w_vocab bf16
- * bits uint16[vocab*hidden].
- * Output: int32 host status of the three calls and the device status word,
+ * bits uint16[vocab*hidden], behav_lp float32[n_rows], reward float32[n_traj].
+ * A second log-prob call also computes the fused loss (GRPO advantages over the
+ * accepted group members and the clipped surrogate, default loss parameters
+ * with the given clip widths).
+ * Output: int32 host status of the four calls and the device status word,
  * int64 k, float64 r_hat, float64 unit_score[n_traj/G], uint8 flags[n_traj],
- * float32 logprob[n_rows].  Exit code 0 when every step ran. */
+ * float32 logprob[n_rows], float64 loss, float32 adv[n_traj].  Exit code 0
+ * when every step ran. */
 #include <stdio.h>
 #include <stdlib.h>
 
@@ -49,7 +53,7 @@ static void* to_device(const void* host, size_t bytes) {
 int main(int argc, char** argv) {
   int64_t hdr[9];
   FILE* f;
-  if (argc != 3) return 1;
+  if (argc != 5) return 1;
   f = fopen(argv[1], "rb");
   if (!f || fread(hdr, sizeof(int64_t), 9, f) != 9) return 1;
   {
@@ -70,7 +74,14 @@ int main(int argc, char** argv) {
     void* h_tgt = read_array(f, (size_t)n_rows * 4);
     void* h_hid = read_array(f, (size_t)n_rows * H * 2);
     void* h_w = read_array(f, (size_t)V * H * 2);
-    int32_t st[4] = {-1, -1, -1, -1};
+    void* h_behav = read_array(f, (size_t)n_rows * 4);
+    void* h_rew = read_array(f, (size_t)n_traj * 4);
+    int32_t st[5] = {-1, -1, -1, -1, -1};
+    PaceLossArgs la;
+    double loss = 0.0;
+    double* d_loss;
+    float *d_lp2, *d_adv, *adv;
+    void *d_behav, *d_rew;
     double r_hat = -1.0;
     int64_t k = -1;
     PaceScoreParams sp;
@@ -89,7 +100,7 @@ int main(int argc, char** argv) {
     void *d_tags, *d_off, *d_c, *d_spre, *d_win, *d_roff, *d_mask, *d_tgt, *d_hid, *d_w;
     fclose(f);
     if (!h_tags || !h_off || !h_c || !h_spre || !h_win || !h_roff || !h_mask || !h_tgt ||
-        !h_hid || !h_w)
+        !h_hid || !h_w || !h_behav || !h_rew)
       return 1;
     d_tags = to_device(h_tags, (size_t)n_tokens * 4);
     d_off = to_device(h_off, (size_t)(n_traj + 1) * 8);
@@ -101,8 +112,10 @@ int main(int argc, char** argv) {
     d_tgt = to_device(h_tgt, (size_t)n_rows * 4);
     d_hid = to_device(h_hid, (size_t)n_rows * H * 2);
     d_w = to_device(h_w, (size_t)V * H * 2);
+    d_behav = to_device(h_behav, (size_t)n_rows * 4);
+    d_rew = to_device(h_rew, (size_t)n_traj * 4);
     if (!d_tags || !d_off || !d_c || !d_spre || !d_win || !d_roff || !d_mask || !d_tgt ||
-        !d_hid || !d_w)
+        !d_hid || !d_w || !d_behav || !d_rew)
       return 2;
     CHECK_CUDA(cudaMalloc((void**)&d_kgen, (size_t)n_traj * 8));
     CHECK_CUDA(cudaMalloc((void**)&d_kwait, (size_t)n_traj * 8));
@@ -142,8 +155,27 @@ int main(int argc, char** argv) {
     CHECK_CUDA(cudaMalloc(&d_ws3, ws_bytes));
     st[2] = pace_token_logprob(&batch, d_hid, d_w, (const int32_t*)d_tgt, H, V, 1.0f, d_lp, NULL,
                                NULL, d_ws3, ws_bytes, d_status, NULL);
+    /* (b) the same rows again with the fused advantages + clipped surrogate */
+    CHECK_CUDA(cudaMalloc((void**)&d_lp2, (size_t)n_rows * 4));
+    CHECK_CUDA(cudaMalloc((void**)&d_adv, (size_t)n_traj * 4));
+    CHECK_CUDA(cudaMalloc((void**)&d_loss, 8));
+    la.behav_lp = (const float*)d_behav;
+    la.reward = (const float*)d_rew;
+    la.group_size = G;
+    pace_loss_params_default(&la.params);
+    la.params.eps_low = (float)atof(argv[3]);
+    la.params.eps_high = (float)atof(argv[4]);
+    la.loss = d_loss;
+    la.adv = d_adv;
+    la.ratio = NULL;
+    st[3] = pace_token_logprob(&batch, d_hid, d_w, (const int32_t*)d_tgt, H, V, 1.0f, d_lp2, NULL,
+                               &la, d_ws3, ws_bytes, d_status, NULL);
     CHECK_CUDA(cudaDeviceSynchronize());
-    CHECK_CUDA(cudaMemcpy(&st[3], d_status, 4, cudaMemcpyDeviceToHost));
+    CHECK_CUDA(cudaMemcpy(&st[4], d_status, 4, cudaMemcpyDeviceToHost));
+    CHECK_CUDA(cudaMemcpy(&loss, d_loss, 8, cudaMemcpyDeviceToHost));
+    adv = (float*)malloc((size_t)n_traj * 4);
+    if (!adv) return 1;
+    CHECK_CUDA(cudaMemcpy(adv, d_adv, (size_t)n_traj * 4, cudaMemcpyDeviceToHost));
     unit = (double*)malloc((size_t)U * 8);
     flags = (uint8_t*)malloc((size_t)n_traj);
     lp = (float*)malloc((size_t)n_rows * 4);
@@ -153,12 +185,14 @@ int main(int argc, char** argv) {
     CHECK_CUDA(cudaMemcpy(lp, d_lp, (size_t)n_rows * 4, cudaMemcpyDeviceToHost));
     o = fopen(argv[2], "wb");
     if (!o) return 1;
-    fwrite(st, 4, 4, o);
+    fwrite(st, 4, 5, o);
     fwrite(&k, 8, 1, o);
     fwrite(&r_hat, 8, 1, o);
     fwrite(unit, 8, (size_t)U, o);
     fwrite(flags, 1, (size_t)n_traj, o);
     fwrite(lp, 4, (size_t)n_rows, o);
+    fwrite(&loss, 8, 1, o);
+    fwrite(adv, 4, (size_t)n_traj, o);
     fclose(o);
   }
   return 0;

@@ -5,9 +5,10 @@
   GPU: version, status strings, defaults and the rejection budget (Eqs. 3-4),
   compared bit for bit with the oracle.
 - tests/c/pace_gpu_c.c (C11) allocates with cudaMalloc and runs scoring,
-  selection and the fused log-probs on the tiny 64-trajectory pool; its
-  outputs are compared with the oracle (scores bit for bit, ids exactly,
-  log-probs within 5e-3)."""
+  selection, the fused log-probs and the fused loss (PaceLossArgs filled in C)
+  on the tiny 64-trajectory pool; its outputs are compared with the oracle
+  (scores bit for bit, ids exactly, log-probs within 5e-3, loss within 1e-3
+  relative)."""
 import math
 import os
 import shutil
@@ -82,6 +83,9 @@ def test_score_select_logprob_from_c(tmp_path):
     offsets = pool.meta["offsets_host"].astype(np.int64)
     tags = np.ascontiguousarray(pool.tags, np.int32)
     n = pool.n_traj
+    st_o, olp, _ = oracle.token_logprob(hb, wb, rows.targets)
+    assert st_o == 0
+    behav = workloads.behaviour_logprob(rows, pool.trainer_version, olp, pool.seed)
     inp = tmp_path / "in.bin"
     with open(inp, "wb") as f:
         np.array([n, tags.size, rows.n_rows, H, V, pool.window.size, G, pool.n_target,
@@ -89,19 +93,26 @@ def test_score_select_logprob_from_c(tmp_path):
         for a, dt in ((tags, np.int32), (offsets, np.int64), (pool.c_version, np.int32),
                       (pool.s_pre, np.float32), (pool.window, np.float32),
                       (rows.row_offsets, np.int64), (rows.mask, np.uint8),
-                      (rows.targets, np.int32), (hb, np.uint16), (wb, np.uint16)):
+                      (rows.targets, np.int32), (hb, np.uint16), (wb, np.uint16),
+                      (behav, np.float32), (pool.reward, np.float32)):
             np.ascontiguousarray(a, dt).tofile(f)
     out = tmp_path / "out.bin"
-    r = subprocess.run([exe, str(inp), str(out)], capture_output=True, text=True)
+    eps_l, eps_h = pool.spec.eps_low, pool.spec.eps_high
+    r = subprocess.run([exe, str(inp), str(out), repr(eps_l), repr(eps_h)], capture_output=True,
+                       text=True)
     assert r.returncode == 0, r.stderr
     raw = out.read_bytes()
     U = n // G
-    st = np.frombuffer(raw, np.int32, 4, 0)
-    k = int(np.frombuffer(raw, np.int64, 1, 16)[0])
-    r_hat = float(np.frombuffer(raw, np.float64, 1, 24)[0])
-    unit = np.frombuffer(raw, np.float64, U, 32)
-    flags = np.frombuffer(raw, np.uint8, n, 32 + 8 * U)
-    lp = np.frombuffer(raw, np.float32, rows.n_rows, 32 + 8 * U + n)
+    st = np.frombuffer(raw, np.int32, 5, 0)
+    k = int(np.frombuffer(raw, np.int64, 1, 20)[0])
+    r_hat = float(np.frombuffer(raw, np.float64, 1, 28)[0])
+    o = 36
+    unit = np.frombuffer(raw, np.float64, U, o)
+    flags = np.frombuffer(raw, np.uint8, n, o + 8 * U)
+    lp = np.frombuffer(raw, np.float32, rows.n_rows, o + 8 * U + n)
+    o2 = o + 8 * U + n + 4 * rows.n_rows
+    loss = float(np.frombuffer(raw, np.float64, 1, o2)[0])
+    adv = np.frombuffer(raw, np.float32, n, o2 + 8)
     assert (st == 0).all(), st
 
     _, *_, ous = oracle.score_pool(tags, offsets, pool.c_version, pool.s_pre,
@@ -111,9 +122,14 @@ def test_score_select_logprob_from_c(tmp_path):
     assert (k, r_hat) == (ok, orh)
     _, _, _, oflag = oracle.select(ous, G, ok)
     np.testing.assert_array_equal(flags, oflag)
-    st_o, olp, _ = oracle.token_logprob(hb, wb, rows.targets)
-    assert st_o == 0
     in_loss = np.repeat(oflag, np.diff(rows.row_offsets)).astype(bool) & rows.mask.astype(bool)
     assert in_loss.any() and (~in_loss).any()
     assert float(np.abs(lp[in_loss] - olp[in_loss]).max()) <= 5e-3
     assert (lp[~in_loss] == 0).all()
+    _, oadv = oracle.group_advantages(pool.reward, G, seq_accepted=oflag,
+                                      eps=float(np.float32(1e-6)))
+    np.testing.assert_allclose(adv, oadv, rtol=1e-5, atol=1e-6)
+    _, oloss, _, _ = oracle.surrogate(olp, behav, rows.row_offsets, oadv, mask=rows.mask,
+                                      seq_accepted=oflag, eps_low=float(np.float32(eps_l)),
+                                      eps_high=float(np.float32(eps_h)))
+    assert abs(loss - oloss) <= 1e-3 * abs(oloss), (loss, oloss)
