@@ -191,15 +191,19 @@ PACE_API size_t pace_select_workspace_size(int64_t n_units);
  * no counterpart: this exists for code that must not call cudaMalloc, such as
  * a plugin running inside a host framework whose memory pool owns all device
  * memory, or a latency-critical loop where an allocation could synchronise
- * the device.  Such a caller still passes its inputs and outputs; the scratch
- * the radix path (pools above 131,072 units) needs comes from a fixed array of
- * 128 KB inside the library, which every GPU that loads the library keeps
- * until the process exits.
+ * the device.  Such a caller still passes its inputs and outputs.  Whenever
+ * the one-cluster selection does not fit on the device (on GB300: pools above
+ * 131,072 units; on a device with a smaller cluster limit, smaller pools too),
+ * the radix path's scratch comes from a fixed array of 128 KB inside the
+ * library (123,136 bytes are used at the 2^20-unit maximum), which every GPU
+ * that loads the library keeps until the process exits.
  *   - n_units must be at most 2^20 (1,048,576); larger pools get
  *     PACE_ERR_UNSUPPORTED_SHAPE and nothing is launched.
  *   - The first call on a device looks up the array's device address (with
  *     that device current) and caches it; make that first call before any
- *     stream capture.
+ *     stream capture.  The cached address belongs to the device's context
+ *     at that time: after cudaDeviceReset on that device the entry point must
+ *     not be called again in the same process.
  *   - All calls on a device share the one array and each call re-initialises
  *     what it needs, so results do not depend on earlier calls; but calls
  *     that overlap on the GPU (different streams, or threads) race on it.

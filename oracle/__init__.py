@@ -71,6 +71,8 @@ def _load():
                 "oracle_surrogate_grad": [_P, _P, _P, _P, _P, _I64, _P, _F64, _F64, _F64, _I32,
                                           _P],
                 "oracle_lmhead_backward": [_P, _P, _P, _P, _I64, _I32, _I32, _F64, _P, _P, _I32],
+                "oracle_lmhead_backward_magnitude": [_P, _P, _P, _P, _I64, _I32, _I32, _F64, _P,
+                                                     _P, _I32],
             }
             for name, args in sig.items():
                 fn = getattr(lib, name)
@@ -275,8 +277,12 @@ def surrogate_grad(logprob, behav_lp, seq_offsets, adv, mask=None, seq_accepted=
 
 
 def lmhead_backward(hidden_bits, w_bits, targets, g, temperature=1.0, with_dw=True,
-                    n_threads=None):
-    """(status, dH fp64 [n_rows, H], dW fp64 [V, H] or None) for dLoss/dlp = g."""
+                    n_threads=None, magnitude=False):
+    """(status, dH fp64 [n_rows, H], dW fp64 [V, H] or None) for dLoss/dlp = g.
+
+    magnitude=True returns instead the error scales sum_v |G_rv| |W_vk| and
+    sum_r |G_rv| |h_rk| (a relative error e in each G_rv moves dH and dW by at
+    most e times these, element by element)."""
     hb, wb = _c(hidden_bits, np.uint16), _c(w_bits, np.uint16)
     tg, gg = _c(targets, np.int32), _c(g, np.float64)
     n, H = hb.shape
@@ -285,6 +291,8 @@ def lmhead_backward(hidden_bits, w_bits, targets, g, temperature=1.0, with_dw=Tr
     dw = np.zeros((V, H), np.float64) if with_dw else None
     if n_threads is None:
         n_threads = min(os.cpu_count() or 1, 64)
-    st = _load().oracle_lmhead_backward(_ptr(hb), _ptr(wb), _ptr(tg), _ptr(gg), n, H, V,
+    fn = (_load().oracle_lmhead_backward_magnitude if magnitude
+          else _load().oracle_lmhead_backward)
+    st = fn(_ptr(hb), _ptr(wb), _ptr(tg), _ptr(gg), n, H, V,
                                         float(temperature), _ptr(dh), _ptr(dw), int(n_threads))
     return st, dh, dw

@@ -14,10 +14,14 @@
 //                             fp32 rows scattered back to their original row;
 //   3. gemm_kernel<EPI_ACC>:  dW += G^T H_c (A = G and B = H_c, both read
 //                             MN-major), fp32 accumulation in place.
-// The GEMM is one warp-specialised tcgen05 kernel: warp 0 issues TMA into a
-// 4-stage ring (128-byte swizzle), warp 1 issues tcgen05.mma (M 128, N 256,
-// K 16; the instruction descriptor's major bits select K- or MN-major operand
-// layouts), warps 2-5 drain the two TMEM accumulators.  Every wait is bounded.
+// The GEMM is one warp-specialised tcgen05 kernel on CTA pairs: in each CTA
+// warp 0 issues TMA for the CTA's own A tile and its own half of the B tile
+// into a 6-stage ring (128-byte swizzle), both CTAs' bytes completing on the
+// even CTA's barrier; warp 1 of the even CTA issues tcgen05.mma.cta_group::2
+// (M 256 = 128 rows per CTA, N 256 = 128 columns from each CTA, K 16; the
+// instruction descriptor's major bits select K- or MN-major operand layouts);
+// warps 2-5 of each CTA drain its two TMEM accumulators.  No operand is
+// multicast.  Every wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -36,10 +40,10 @@ namespace {
 constexpr int GBM = 128;
 constexpr int GBN = 256;
 constexpr int GBK = 64;
-constexpr int GSTAGES = 4;
+constexpr int GSTAGES = 6;
 constexpr int kGemmThreads = 192;
 constexpr uint32_t kGStageA = GBM * GBK * 2;  // 16 KB
-constexpr uint32_t kGStageB = GBN * GBK * 2;  // 32 KB
+constexpr uint32_t kGStageB = GBN / 2 * GBK * 2;  // 16 KB: this CTA's half of the B tile
 constexpr uint32_t kGStageBytes = kGStageA + kGStageB;
 constexpr uint32_t kGTmemCols = 2 * GBN;
 constexpr size_t kGSmemBytes = 1024 + GSTAGES * kGStageBytes + 256;
@@ -79,8 +83,8 @@ struct GemmArgs {
 };
 
 // Work items are (pair of M tiles, N tile); the two CTAs of a cluster take the
-// two M tiles of a pair and share every B tile, each loading half of it and
-// multicasting it to both.
+// two M tiles of a pair and share every B tile through the 2-CTA MMA, each
+// loading its own half of it.
 __device__ __forceinline__ void item_of(const GemmArgs& p, int64_t m_tiles, int64_t item,
                                         int64_t* mp, int64_t* n) {
   const int64_t pairs = (m_tiles + 1) / 2;
@@ -114,10 +118,11 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t saddr, bool mn_major) 
   return d;
 }
 
+// M = 256: the pair's two 128-row tiles.
 __host__ __device__ constexpr uint32_t idesc_bf16(bool a_mn, bool b_mn) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) |
          ((b_mn ? 1u : 0u) << 16) | ((static_cast<uint32_t>(GBN) >> 3) << 17) |
-         ((static_cast<uint32_t>(GBM) >> 4) << 24);
+         ((static_cast<uint32_t>(2 * GBM) >> 4) << 24);
 }
 
 __device__ __forceinline__ uint16_t f32_to_bf16_rn(float x) {
@@ -145,6 +150,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t crank = cluster_ctarank();
+  const bool leader = crank == 0;
   // The host sizes a chunk by its row capacity; the rows of it that are in the
   // loss are known only on the device (the compaction's count).  Tiles past
   // them hold zero rows: M (G, dH) or K (dW) is cut to the count rounded up to
@@ -166,31 +172,38 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
   const int64_t n_items = (m_tiles + 1) / 2 * p.n_tiles;
   const int64_t cid = blockIdx.x / 2, n_clusters = gridDim.x / 2;
   const int nkb = static_cast<int>((K + GBK - 1) / GBK);
-  if (nkb == 0 || n_items == 0) return;  // uniform over the grid
+  // uniform over the grid, and before the pair's collective TMEM allocation
+  if (nkb == 0 || n_items == 0) return;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < GSTAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 2);  // both CTAs' MMAs (each stage holds the peer's half of B)
+      mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tmem_full[b], 1);
-      mbar_init(&tmem_empty[b], 4 * 32);
+      mbar_init(&tmem_empty[b], 2 * 4);  // one arrival per epilogue warp of the pair
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
+  cluster_sync();  // both CTAs run and their barriers exist
   if (warp == 1) {
-    tmem_alloc(tmem_slot, kGTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(tmem_slot, kGTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  cluster_sync();
+  cluster_sync();  // both CTAs' tensor memory is allocated before any MMA writes it
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   constexpr uint32_t kIdesc = idesc_bf16(A_MN, B_MN);
-  constexpr uint16_t kPair = 0x3;
+  const uint32_t peer_abort = cluster_addr(const_cast<int*>(abort_flag), crank ^ 1u);
+  auto give_up = [&]() {
+    if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+    *abort_flag = 1;
+    st_cluster_u32(peer_abort, 1u);
+  };
 
   if (warp == 0) {
     if (lane == 0) {
@@ -213,51 +226,54 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           }
           unsigned char* sa = smem + s * kGStageBytes;
           unsigned char* sb = sa + kGStageA;
-          mbar_arrive_expect_tx(&full[s], kGStageBytes);
+          const uint32_t bar = cluster_addr(&full[s], 0);
+          if (leader) mbar_arrive_expect_tx(&full[s], 2 * kGStageBytes);
           const int32_t k0 = kb * GBK;
           if (p.a_pitch > 0) {  // blocked G: one 64-wide block is the inner dimension
             const int64_t ap = p.a_pitch;
             if (A_MN) {  // M = vocabulary: blocks m0 / 64 and m0 / 64 + 1, rows k0..k0+63
               const int64_t b0 = m0 / 64;
-              tma_load_2d(sa, &tm_a, &full[s], 0, static_cast<int32_t>(b0 * ap + k0), pol);
-              tma_load_2d(sa + 8192, &tm_a, &full[s], 0,
-                          static_cast<int32_t>((b0 + 1) * ap + k0), pol);
+              tma_load_2d_pair(sa, &tm_a, bar, 0, static_cast<int32_t>(b0 * ap + k0), pol);
+              tma_load_2d_pair(sa + 8192, &tm_a, bar, 0,
+                               static_cast<int32_t>((b0 + 1) * ap + k0), pol);
             } else {     // K = vocabulary: block kb, rows m0..m0+127
-              tma_load_2d(sa, &tm_a, &full[s], 0, static_cast<int32_t>(kb * ap + m0), pol);
+              tma_load_2d_pair(sa, &tm_a, bar, 0, static_cast<int32_t>(kb * ap + m0), pol);
             }
           } else if (A_MN) {  // box {64 MN, 64 K}: two along M
-            tma_load_2d(sa, &tm_a, &full[s], m0, k0, pol);
-            tma_load_2d(sa + 8192, &tm_a, &full[s], m0 + 64, k0, pol);
+            tma_load_2d_pair(sa, &tm_a, bar, m0, k0, pol);
+            tma_load_2d_pair(sa + 8192, &tm_a, bar, m0 + 64, k0, pol);
           } else {     // box {64 K, 128 rows}
-            tma_load_2d(sa, &tm_a, &full[s], k0, m0, pol);
+            tma_load_2d_pair(sa, &tm_a, bar, k0, m0, pol);
           }
-          // this CTA's half of B, multicast into both CTAs of the pair
-          if (B_MN) {  // four {64 N, 64 K} boxes along N; this CTA loads two
-#pragma unroll
-            for (int q = 2 * static_cast<int>(crank); q < 2 * static_cast<int>(crank) + 2; ++q)
-              tma_load_2d_multicast(sb + q * 8192, &tm_b, &full[s], n0 + 64 * q, k0, kPair, pol);
-          } else {     // {64 K, 128 rows}, one half of the 256 rows
-            tma_load_2d_multicast(sb + crank * (kGStageB / 2), &tm_b, &full[s], k0,
-                                  n0 + static_cast<int32_t>(crank) * (GBN / 2), kPair, pol);
+          // this CTA's half of B: columns n0 + 128 * crank .. + 127
+          const int32_t nh = n0 + static_cast<int32_t>(crank) * (GBN / 2);
+          if (B_MN) {  // two {64 N, 64 K} boxes along N
+            tma_load_2d_pair(sb, &tm_b, bar, nh, k0, pol);
+            tma_load_2d_pair(sb + 8192, &tm_b, bar, nh + 64, k0, pol);
+          } else {     // {64 K, 128 rows}
+            tma_load_2d_pair(sb, &tm_b, bar, k0, nh, pol);
           }
         }
       }
-      if (!ok) {
-        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
-        *abort_flag = 1;
-      }
+      if (!ok) give_up();
+      // every copy issued has landed before the CTA exits: the even CTA sees
+      // both CTAs' bytes on its full barriers, the odd CTA its stages consumed
+      const uint64_t lim = *abort_flag ? 1000000ull : kWaitLimitNs;
       for (uint32_t s = 0; s < GSTAGES && s < it; ++s) {
         const uint32_t last = it - 1 - ((it - 1 - s) % GSTAGES);
-        mbar_wait_bounded(&full[s], (last / GSTAGES) & 1u, nullptr);
+        if (leader)
+          mbar_wait_bounded(&full[s], (last / GSTAGES) & 1u, nullptr, lim);
+        else
+          mbar_wait_bounded(&empty[s], (last / GSTAGES) & 1u, nullptr, lim);
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && leader) {
       uint32_t it = 0, tc = 0;
       bool ok = true;
       for (int64_t t = cid; t < n_items && ok; t += n_clusters, ++tc) {
         const uint32_t acc = tc & 1u, acc_ph = (tc >> 1) & 1u;
-        if (!mbar_wait_bounded(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
+        if (!mbar_wait_bounded_cluster(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
           ok = false;
           break;
         }
@@ -276,33 +292,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           for (int k = 0; k < GBK / 16; ++k) {
             const uint32_t ka = A_MN ? sa + k * 2048 : sa + k * 32;
             const uint32_t kbb = B_MN ? sb + k * 2048 : sb + k * 32;
-            tc_mma_f16(d_tmem, operand_desc(ka, A_MN), operand_desc(kbb, B_MN), kIdesc,
-                       (kb > 0 || k > 0) ? 1u : 0u);
+            tc_mma_f16_pair(d_tmem, operand_desc(ka, A_MN), operand_desc(kbb, B_MN), kIdesc,
+                            (kb > 0 || k > 0) ? 1u : 0u);
           }
-          tc_commit_multicast(&empty[s], kPair);
+          tc_commit_pair(cluster_addr(&empty[s], 0));
+          tc_commit_pair(cluster_addr(&empty[s], 1));
         }
         if (!ok) break;
-        tc_commit(&tmem_full[acc]);
+        tc_commit_pair(cluster_addr(&tmem_full[acc], 0));
+        tc_commit_pair(cluster_addr(&tmem_full[acc], 1));
       }
-      if (!ok) {
-        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
-        *abort_flag = 1;
-      }
-      tc_commit(mma_done);
+      if (!ok) give_up();
+      tc_commit_pair(cluster_addr(mma_done, 0));
       mbar_wait_bounded(mma_done, 0, nullptr);
     }
   } else {
     const int quad = warp & 3;
     const int r_local = quad * 32 + lane;
+    const uint32_t empty0 = cluster_addr(&tmem_empty[0], 0);
+    const uint32_t empty1 = cluster_addr(&tmem_empty[1], 0);
     uint32_t tc = 0;
     for (int64_t t = cid; t < n_items; t += n_clusters, ++tc) {
       int64_t mp, nt;
       item_of(p, m_tiles, t, &mp, &nt);
       const int64_t mt = 2 * mp + crank;
       const uint32_t acc = tc & 1u, acc_ph = (tc >> 1) & 1u;
-      if (!mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag)) {
-        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
-        *abort_flag = 1;
+      // one outcome for the whole warp (tcgen05.ld below is warp-collective)
+      const bool got = __all_sync(0xffffffffu,
+                                  mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag));
+      if (!got) {
+        give_up();
         break;
       }
       tc_fence_after();
@@ -387,16 +406,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
           }
         }
       }
+      // one arrival per warp on the even CTA's barrier, after every lane's loads
       tc_fence_before();
-      mbar_arrive(&tmem_empty[acc]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(acc ? empty1 : empty0);
     }
   }
 
   tc_fence_before();
   __syncthreads();
-  cluster_sync();  // the peer may still multicast into this CTA until it is done too
+  // neither CTA frees its tensor memory or leaves while the pair's MMAs, copies
+  // or arrivals may still reach it
+  cluster_sync();
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, kGTmemCols);
+  if (warp == 1) tmem_dealloc_pair(tmem_base, kGTmemCols);
+  cluster_sync();  // the collective release is complete in both CTAs
 }
 
 // Zero the gathered rows from n_valid up to the next multiple of GBM (at most

@@ -2,23 +2,26 @@
 // (Sec. 2: the policy factorises over tokens, log pi_theta(y_t | x, y_<t);
 // training temperature from the shared settings), without writing logits.
 //
-// lmhead_lse_kernel (sm_103a, persistent 2-CTA clusters, one CTA per SM, 192
-// threads, warp-specialised):
-//   warp 0 / lane 0   TMA producer: per K step the CTA's own 128x64 hidden tile
-//                     and one half (128x64) of the pair's 256x64 vocabulary tile,
-//                     multicast into both CTAs of the cluster, into a 4-stage
-//                     shared-memory ring (128-byte swizzle), completion tracked
-//                     by mbarrier transaction bytes.
-//   warp 1 / lane 0   MMA issuer: tcgen05.mma kind::f16 (bf16 x bf16 -> fp32),
-//                     M=128, N=256, K=16 per instruction, accumulating a
-//                     128x256 logit tile in tensor memory; two accumulators
-//                     (512 TMEM columns) so the epilogue of tile n overlaps
-//                     the MMAs of tile n+1.
-//   warps 2..5        epilogue: each thread owns one row (one TMEM lane),
-//                     reads its 256 logits 32 columns at a time with
-//                     tcgen05.ld, keeps a running base-2 max and sum of
+// lmhead_lse_kernel (sm_103a, persistent CTA pairs, one CTA per SM, 192
+// threads, warp-specialised, tcgen05 on the pair):
+//   warp 0 / lane 0   TMA producer, in both CTAs: per K step the CTA's own
+//                     128x64 hidden tile and its own half (128x64) of the pair's
+//                     256x64 vocabulary tile, into its own 6-stage shared-memory
+//                     ring (128-byte swizzle); the transaction bytes of both
+//                     CTAs complete on the even CTA's mbarrier.
+//   warp 1 / lane 0   MMA issuer, even CTA only: tcgen05.mma.cta_group::2
+//                     kind::f16 (bf16 x bf16 -> fp32), M=256 (128 rows from each
+//                     CTA), N=256 (128 vocabulary rows from each CTA), K=16 per
+//                     instruction; each CTA's tensor memory receives its own
+//                     128x256 logit tile; two accumulators (512 TMEM columns)
+//                     so the epilogue of tile n overlaps the MMAs of tile n+1.
+//   warps 2..5        epilogue, in both CTAs: each thread owns one row (one
+//                     TMEM lane), reads its 256 logits 32 columns at a time
+//                     with tcgen05.ld, keeps a running base-2 max and sum of
 //                     exponentials (online log-sum-exp) and picks out the
 //                     target's logit.
+// No operand is multicast: every CTA reads only its own tiles; the pair shares
+// the vocabulary tile through the 2-CTA MMA itself.
 // A work item is a pair of 128-row blocks (one per CTA of the cluster) and one
 // of S contiguous vocabulary splits; each CTA writes one (max, sum) pair per row
 // and split.  Consecutive items share a row pair, so the hidden tiles re-read
@@ -29,8 +32,8 @@
 //   and writes lp = z_y / tau - lse.
 //
 // Every mbarrier wait is bounded (2 s); on timeout the CTA reports
-// PACE_ERR_TIMEOUT, stops issuing, waits (bounded) for its in-flight copies
-// and MMAs, frees its tensor memory and returns.
+// PACE_ERR_TIMEOUT, tells its peer to stop, waits (bounded) for its in-flight
+// copies and MMAs, frees its tensor memory and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -46,19 +49,17 @@
 namespace pace {
 namespace {
 
-constexpr int BM = 128;
-constexpr int BN = 256;
+constexpr int BM = 128;                         // rows per CTA; the pair's MMA covers 256
+constexpr int BN = 256;                         // vocabulary rows per MMA tile (both CTAs)
 constexpr int BK = 64;
-constexpr int STAGES = 4;
-constexpr int CLUSTER = 2;                      // CTAs sharing each vocabulary tile
+constexpr int STAGES = 6;
+constexpr int CLUSTER = 2;                      // the CTA pair of one 2-CTA MMA
 constexpr int kThreads = 192;
 constexpr uint32_t kStageA = BM * BK * 2;       // 16 KB: this CTA's 128 hidden rows
-constexpr uint32_t kStageB = BN * BK * 2;       // 32 KB: 256 vocabulary rows
-constexpr uint32_t kHalfB = kStageB / CLUSTER;  // each CTA of the pair loads one half
+constexpr uint32_t kStageB = BN / CLUSTER * BK * 2;  // 16 KB: this CTA's half of the vocabulary tile
 constexpr uint32_t kStageBytes = kStageA + kStageB;
 constexpr uint32_t kTmemCols = 2 * BN;          // two fp32 accumulators of 256 columns
-constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
-constexpr uint16_t kPairMask = 0x3;
+constexpr uint32_t kIdesc = idesc_bf16_f32(CLUSTER * BM, BN);
 constexpr size_t kSmemBytes = 1024 /* alignment slack */ + STAGES * kStageBytes + 256;
 constexpr int kMaxSplits = 8;
 
@@ -122,10 +123,9 @@ __device__ __forceinline__ uint64_t make_policy_evict_normal() {
 
 // A work item is (row pair, vocabulary split): the two CTAs of a cluster take
 // the two 128-row blocks of the pair and sweep the same vocabulary tiles, each
-// loading half of every 256-row vocabulary tile and multicasting it to both.
-// Clusters are persistent and take items round-robin, so all clusters sweep
-// their splits in step and each vocabulary tile is read from HBM about once per
-// round of items.
+// loading its half of every 256-row vocabulary tile.  Clusters are persistent
+// and take items round-robin, so all clusters sweep their splits in step and
+// each vocabulary tile is read from HBM about once per round of items.
 struct ItemCursor {
   int64_t item, n_items;
   int n_clusters;
@@ -138,14 +138,16 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
     lmhead_lse_kernel(const __grid_constant__ CUtensorMap tm_a,
                       const __grid_constant__ CUtensorMap tm_b, LmArgs p) {
   extern __shared__ unsigned char smem_raw[];
+  // the same offsets in both CTAs: the pair's MMA reads each CTA's operand
+  // tiles at the addresses the even CTA's descriptors name
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* stage_base = smem;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * kStageBytes);
-  uint64_t* full = bars;                     // [STAGES] this CTA's A + both halves of B landed
-  uint64_t* empty = bars + STAGES;           // [STAGES] both CTAs' MMAs done with the stage
-  uint64_t* tmem_full = bars + 2 * STAGES;   // [2]
-  uint64_t* tmem_empty = tmem_full + 2;      // [2]
+  uint64_t* full = bars;                     // [STAGES] even CTA: both CTAs' tiles landed
+  uint64_t* empty = bars + STAGES;           // [STAGES] the pair's MMAs are done with the stage
+  uint64_t* tmem_full = bars + 2 * STAGES;   // [2] this CTA's accumulator is ready
+  uint64_t* tmem_empty = tmem_full + 2;      // [2] even CTA: both CTAs' epilogues drained it
   uint64_t* mma_done = tmem_empty + 2;       // [1]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -153,6 +155,7 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const uint32_t crank = cluster_ctarank();
+  const bool leader = crank == 0;
   const int n_clusters = static_cast<int>(gridDim.x) / CLUSTER;
   const int cid = static_cast<int>(blockIdx.x) / CLUSTER;
   const int64_t n_valid = p.n_valid_dev ? static_cast<int64_t>(*p.n_valid_dev) : p.rows_cap;
@@ -160,35 +163,44 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
   const int n_splits = pick_splits(row_pairs, n_clusters, p.n_vtiles, p.split_pref);
   const int tiles_per_split = (p.n_vtiles + n_splits - 1) / n_splits;
   const int64_t n_items = row_pairs * n_splits;
-  // both CTAs of a cluster read the same n_valid and cid: the exit is uniform
+  // both CTAs of a cluster read the same n_valid and cid: the exit is uniform,
+  // and comes before the pair's collective tensor-memory allocation
   if (cid >= n_items) return;
   const int nkb = p.H / BK;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], CLUSTER);
+      mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tmem_full[b], 1);
-      mbar_init(&tmem_empty[b], 4 * 32);
+      mbar_init(&tmem_empty[b], CLUSTER * 4);  // one arrival per epilogue warp of the pair
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
+  cluster_sync();  // both CTAs run and their barriers exist
   if (warp == 1) {
-    tmem_alloc(tmem_slot, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(tmem_slot, kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  cluster_sync();  // both CTAs' barriers exist before any multicast reaches them
+  cluster_sync();  // both CTAs' tensor memory is allocated before any MMA writes it
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  const uint32_t peer_abort = cluster_addr(const_cast<int*>(abort_flag), crank ^ 1u);
+  // first timeout: report it, and make both CTAs of the pair stop issuing
+  auto give_up = [&]() {
+    if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
+    *abort_flag = 1;
+    st_cluster_u32(peer_abort, 1u);
+  };
 
   if (warp == 0) {
     if (lane == 0) {
-      // ------------------------------------------------ TMA producer
+      // ------------------------------------------------ TMA producer (both CTAs)
       tma_prefetch_desc(&tm_a);
       tma_prefetch_desc(&tm_b);
       const uint64_t pol = make_policy_evict_normal();
@@ -211,26 +223,30 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
             }
             unsigned char* sa = stage_base + s * kStageBytes;
             unsigned char* sb = sa + kStageA;
-            mbar_arrive_expect_tx(&full[s], kStageBytes);
-            tma_load_2d(sa, &tm_a, &full[s], kb * BK, row0, pol);
-            tma_load_2d_multicast(sb + crank * kHalfB, &tm_b, &full[s], kb * BK, nb, kPairMask,
-                                  pol);
+            const uint32_t bar = cluster_addr(&full[s], 0);
+            if (leader) mbar_arrive_expect_tx(&full[s], CLUSTER * kStageBytes);
+            tma_load_2d_pair(sa, &tm_a, bar, kb * BK, row0, pol);
+            tma_load_2d_pair(sb, &tm_b, bar, kb * BK, nb, pol);
           }
         }
       }
-      if (!ok) {
-        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
-        *abort_flag = 1;
-      }
-      // Drain: every copy issued must have landed before the CTA exits.
+      if (!ok) give_up();
+      // Drain: every copy issued must have landed before the CTA exits.  The
+      // even CTA sees both CTAs' bytes on its full barriers; the odd CTA sees
+      // its stages consumed on its empty barriers.  After a timeout anywhere
+      // the waits are short: copies land in microseconds.
+      const uint64_t lim = *abort_flag ? 1000000ull : kWaitLimitNs;
       for (uint32_t s = 0; s < STAGES && s < it; ++s) {
         const uint32_t last = it - 1 - ((it - 1 - s) % STAGES);  // last index with stage s
-        mbar_wait_bounded(&full[s], (last / STAGES) & 1u, nullptr);
+        if (leader)
+          mbar_wait_bounded(&full[s], (last / STAGES) & 1u, nullptr, lim);
+        else
+          mbar_wait_bounded(&empty[s], (last / STAGES) & 1u, nullptr, lim);
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer
+    if (lane == 0 && leader) {
+      // ------------------------------------------------ MMA issuer (even CTA)
       uint32_t it = 0, tcount = 0;
       bool ok = true;
       for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
@@ -240,7 +256,7 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
         for (int t = tile0; t < tile1 && ok; ++t, ++tcount) {
           const uint32_t acc = tcount & 1u;
           const uint32_t acc_ph = (tcount >> 1) & 1u;
-          if (!mbar_wait_bounded(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
+          if (!mbar_wait_bounded_cluster(&tmem_empty[acc], acc_ph ^ 1u, abort_flag)) {
             ok = false;
             break;
           }
@@ -258,30 +274,30 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
             const uint32_t sb = sa + kStageA;
 #pragma unroll
             for (int k = 0; k < BK / 16; ++k) {
-              tc_mma_f16(d_tmem, smem_desc_k128(sa + k * 32), smem_desc_k128(sb + k * 32),
-                         kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
+              tc_mma_f16_pair(d_tmem, smem_desc_k128(sa + k * 32), smem_desc_k128(sb + k * 32),
+                              kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
             }
-            // frees the stage in both CTAs once these MMAs have read it: the peer
-            // multicasts its half of B into this CTA's stage too
-            tc_commit_multicast(&empty[s], kPairMask);
+            // the stage is free in both CTAs once these MMAs have read it
+            tc_commit_pair(cluster_addr(&empty[s], 0));
+            tc_commit_pair(cluster_addr(&empty[s], 1));
           }
           if (!ok) break;
-          tc_commit(&tmem_full[acc]);
+          tc_commit_pair(cluster_addr(&tmem_full[acc], 0));
+          tc_commit_pair(cluster_addr(&tmem_full[acc], 1));
         }
       }
-      if (!ok) {
-        if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
-        *abort_flag = 1;
-      }
+      if (!ok) give_up();
       // all MMAs issued by this thread complete before tensor memory is freed
-      tc_commit(mma_done);
+      tc_commit_pair(cluster_addr(mma_done, 0));
       mbar_wait_bounded(mma_done, 0, nullptr);
     }
   } else {
-    // ------------------------------------------------ epilogue (4 warps)
+    // ------------------------------------------------ epilogue (4 warps, both CTAs)
     const int quad = warp & 3;  // TMEM lanes this warp may access
     const int r_local = quad * 32 + lane;
     const float scale = p.scale_log2;
+    const uint32_t empty0 = cluster_addr(&tmem_empty[0], 0);
+    const uint32_t empty1 = cluster_addr(&tmem_empty[1], 0);
     uint32_t tcount = 0;
     bool ok = true;
     for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
@@ -301,9 +317,12 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
       for (int t = tile0; t < tile1; ++t, ++tcount) {
         const uint32_t acc = tcount & 1u;
         const uint32_t acc_ph = (tcount >> 1) & 1u;
-        if (!mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag)) {
-          if (!*abort_flag) report(p.status, PACE_ERR_TIMEOUT);
-          *abort_flag = 1;
+        // one outcome for the whole warp: tcgen05.ld below is warp-collective,
+        // and a lane that saw the peer's abort must not leave its warp behind
+        const bool got = __all_sync(0xffffffffu,
+                                    mbar_wait_bounded(&tmem_full[acc], acc_ph, abort_flag));
+        if (!got) {
+          give_up();
           ok = false;
           break;
         }
@@ -338,8 +357,11 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
             have_tgt = true;
           }
         }
+        // this warp is done reading the accumulator: one arrival per warp on the
+        // even CTA's barrier, after every lane's loads have completed
         tc_fence_before();
-        mbar_arrive(&tmem_empty[acc]);
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(acc ? empty1 : empty0);
       }
       if (row_ok && ok) {
         const int64_t o = row * n_splits + split;
@@ -352,10 +374,12 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
-  // neither CTA leaves while its peer may still multicast into it or arrive on it
+  // neither CTA frees its tensor memory or leaves while the pair's MMAs, copies
+  // or arrivals may still reach it
   cluster_sync();
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
+  if (warp == 1) tmem_dealloc_pair(tmem_base, kTmemCols);
+  cluster_sync();  // the collective release is complete in both CTAs
 }
 
 // Per row in the loss: log-sum-exp from the split partials, then
@@ -491,7 +515,7 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   const int n_vtiles = (V + BN - 1) / BN;
   CUtensorMap tm_a, tm_b;
   PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, H, BK, BM));
-  PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, H, BK, BN / CLUSTER));
+  PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, H, BK, BN / CLUSTER));  // one CTA's half tile
   LmLaunchInfo li;
   PACE_TRY(lm_launch_info(&li));
   LmArgs a;

@@ -1150,7 +1150,9 @@ namespace {
 
 // Device address of g_select_scratch on the current device.  In host code the
 // array's name is only a host-side stand-in, so the address is asked from the
-// runtime once per device (with that device current) and cached.
+// runtime once per device (with that device current) and cached.  The cached
+// address belongs to the device's context at that time; after cudaDeviceReset
+// the entry point is not to be used again in the process (stated in pace.h).
 pace_status select_scratch_address(void** out) {
   constexpr int kMaxDevices = 64;
   static void* addr[kMaxDevices] = {};

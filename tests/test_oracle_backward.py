@@ -74,3 +74,28 @@ def test_lmhead_backward_matches_autograd(rows, H, V, tau):
     np.testing.assert_allclose(dw, w.grad.numpy(), rtol=1e-10, atol=1e-12)
     assert np.abs(dw.sum(axis=0)).max() < 1e-12  # sum over the vocabulary is zero
     assert (dh[2] == 0).all()
+
+
+@pytest.mark.parametrize("rows,H,V,tau", [(6, 16, 37, 1.0), (9, 32, 70, 0.8)])
+def test_lmhead_backward_magnitude_matches_autograd(rows, H, V, tau):
+    """The element-wise error scales sum_v |G_rv||W_vk| and sum_r |G_rv||h_rk|, with G
+    the library's autograd gradient of the logits (a different route to G), and the
+    triangle-inequality bound they put on dH and dW."""
+    rng = np.random.default_rng(rows * V)
+    hb, hf = _bits(rng.standard_normal((rows, H)))
+    wb, wf = _bits(rng.standard_normal((V, H)) / math.sqrt(H) * 2)
+    y = rng.integers(0, V, size=rows).astype(np.int32)
+    g = rng.standard_normal(rows)
+    g[1] = 0.0
+    st, mh, mw = oracle.lmhead_backward(hb, wb, y, g, temperature=tau, n_threads=2,
+                                        magnitude=True)
+    assert st == 0
+    z = torch.from_numpy(hf @ wf.T).requires_grad_(True)
+    lp = torch.log_softmax(z / tau, dim=-1)[torch.arange(rows), torch.from_numpy(y).long()]
+    (lp * torch.from_numpy(g)).sum().backward()
+    G = np.abs(z.grad.numpy())
+    np.testing.assert_allclose(mh, G @ np.abs(wf), rtol=1e-10, atol=1e-14)
+    np.testing.assert_allclose(mw, G.T @ np.abs(hf), rtol=1e-10, atol=1e-14)
+    _, dh, dw = oracle.lmhead_backward(hb, wb, y, g, temperature=tau, n_threads=2)
+    assert (np.abs(dh) <= mh * (1 + 1e-12)).all() and (np.abs(dw) <= mw * (1 + 1e-12)).all()
+    assert (mh[1] == 0).all()

@@ -2,14 +2,16 @@
 allocate device memory (for example a plugin inside a framework whose memory
 pool owns all device memory).  Its scratch is a fixed 128 KB array inside the
 library, so it must give exactly the ids of pace_select_k, which uses a
-caller-provided workspace, and keep doing so on back-to-back calls that reuse
-the shared array.  This file is collected last on purpose."""
+caller-provided workspace, and of the CPU oracle's top-k, and keep doing so on
+back-to-back calls that reuse the shared array.  This file is collected last on
+purpose."""
 import ctypes
 
 import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_2609_36830_gb300 import pace
 
 pytestmark = pytest.mark.gpu
@@ -65,6 +67,12 @@ def test_noalloc_matches_workspace_entry_point_twice(U, G):
         b = _call_workspace(s, G, k)
         for x, y in zip(a, b):
             np.testing.assert_array_equal(x, y)
+        # and the oracle's (score desc, id asc) top-k on the same scores
+        st, acc, rej, flag = oracle.select(s.cpu().numpy(), G, k)
+        assert st == 0
+        np.testing.assert_array_equal(a[0][: acc.size], acc)
+        np.testing.assert_array_equal(a[1][: rej.size], rej)
+        np.testing.assert_array_equal(a[2], flag)
         assert a[1][: k * G].size == k * G and (a[1][: k * G] >= 0).all()
 
 
