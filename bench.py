@@ -3,20 +3,26 @@
 A step is one pass of the whole path over one pool: pool scoring
 (pace_score_pool), budget + rejection (pace_select), then the fused LM-head
 log-probs, GRPO advantages and clipped surrogate of the accepted rows
-(pace_token_logprob).  The workload is the 7B-shaped single-turn math pool
-(512 trajectories = 64 prompts x 8, 256 masked prompt rows + lognormal
-responses, hidden 3584, vocab 152064, capacity 384): the metric is accepted
-tokens per second (rows in the loss / step time).  Further line items time
-pool scoring + selection alone on the sweep pools (1k, 16k, 128k and 1M
-trajectories) against HBM bandwidth, prefix rescoring (Eq. 6) and the LM-head
-backward.
+(pace_token_logprob).  The headline workload is the largest step that fits one
+GPU, the MoE-shaped policy head (1024 trajectories = 128 prompts x 8, lognormal
+responses of median 4096 capped at 16384, hidden 2048, vocab 151936, capacity
+768): the metric is accepted tokens per second (rows in the loss / step time).
+Further line items time the same step on the 7B-shaped math pool and the
+multi-turn tool-use pool, pool scoring + selection alone on the sweep pools
+(1k, 16k, 128k and 1M trajectories) against HBM bandwidth, prefix rescoring
+(Eq. 6) and the LM-head backward.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
-With N > 1 (torchrun), every rank runs an independent pool (its own seed): the
-path has no exchange, so the job is weak-scaled replicas with a barrier and a
-max-over-ranks clock.  ``--impl reference`` times the CPU oracle on a bounded
-sample of the same workload (rank 0 only).
+With N > 1 (torchrun, one process per GPU) the pool is partitioned by prompt
+group across the ranks (each rank holds 1024 trajectories, the whole pool
+N x 1024 with capacity N x 768): the ranks score their groups, reject the k
+top-scored groups of the whole pool (six all-reduces of a 2048-bin histogram
+and one exclusive sum of tie counts) and compute log-probs and loss on their
+accepted rows, the loss from one all-reduce of two partial sums; weak scaling,
+a barrier around the timed region and the slowest rank's clock.
+``--impl reference`` times the CPU oracle on a bounded sample of the same
+workload (rank 0 only).
 """
 from __future__ import annotations
 
@@ -35,14 +41,14 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-WORKLOAD = "math7b"
-# DRAM bytes per unit from the committed ncu captures of the current kernels, by the LM head's
-# vocabulary split count (profiles/lmhead_lse_kernel_one_wave.md: 4 splits, 1.130 GB for one
-# full round of 4864 rows, W read once per round, so traffic grows with the rows processed;
-# 2 splits, 18.87 GB for four rounds of 9728 rows; profiles/tag_reduce_kernel_sweep1m.md:
-# 14.0856 GB read + written for 3.5023 G tags).  Set to None when a kernel changes until it is
-# captured again.
-LMHEAD_DRAM_BYTES_PER_ROW = {4: 1.12978e9 / 4864, 2: 18.8672e9 / 38912}
+WORKLOAD = "moe"
+OTHER_WORKLOADS = ("math7b", "multiturn")
+PREFIX_WORKLOAD = "math7b"  # prefix rescoring and the backward are timed on the 7B math pool
+# DRAM bytes (read + written) per row in the loss of the LM-head kernel, by workload, from a
+# one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of one launch of the
+# current kernel; None until the current kernel has been captured.  The tag reduction's per
+# tag: 14.0656 GB read + 19.8 MB written for the 3.5023 G tags of the 1M sweep pool.
+LMHEAD_DRAM_BYTES_PER_ROW = {}
 TAG_REDUCE_DRAM_BYTES_PER_TAG = (14065824512 + 19798528) / 3502330341
 SWEEP_N = 1048576
 SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)
@@ -114,20 +120,37 @@ def _dist():
     return replicas.rank_env()
 
 
-def _make_step(seed_offset, device, workload=WORKLOAD):
-    from paper_2609_36830_gb300 import pace, step, workloads
+def _make_inputs(seed_offset, device, workload=WORKLOAD):
+    """The pool of rank seed_offset (its own seed), its rows and the step's device inputs."""
+    from paper_2609_36830_gb300 import pace, replicas, step, workloads
     spec = workloads.SPECS[workload]
-    from paper_2609_36830_gb300 import replicas
     pool = workloads.make_pool(workload, seed=replicas.replica_seed(workload, seed_offset))
     rows = workloads.make_rows(pool)
     H, V = spec.hidden, spec.vocab
     hidden = workloads.bf16_normal_device((rows.n_rows, H), 1.0, pool.seed + 11, device=device)
-    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), pool.seed + 12, device=device)
+    # the vocabulary matrix is the same on every rank (the policy's lm_head.weight)
+    w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H),
+                                     replicas.replica_seed(workload, 0) + 12, device=device)
     behav = workloads.behaviour_logprob(rows, pool.trainer_version, workloads.uniform_center(V),
                                         pool.seed)
     x = step.build_inputs(pool, rows, hidden, w, behav, device=device)
     lp_params = pace.loss_params(eps_low=spec.eps_low, eps_high=spec.eps_high)
-    return pool, rows, x, step.PaceStep(x, loss_params=lp_params, device=device)
+    return pool, rows, x, lp_params
+
+
+def _step_for(x, pool, lp_params, ws, rank, device):
+    """One GPU: the whole pool's step.  N ranks: this rank's part of the step over
+    the pool partitioned by prompt group (every rank holds pool.n_traj trajectories)."""
+    from paper_2609_36830_gb300 import sharded, step
+    if ws == 1:
+        return step.PaceStep(x, loss_params=lp_params, device=device)
+    return sharded.ShardedPaceStep(x, rank * (pool.n_traj // pool.group_size), ws * pool.n_traj,
+                                   ws * pool.n_target, loss_params=lp_params, device=device)
+
+
+def _make_step(seed_offset, device, workload=WORKLOAD):
+    pool, rows, x, lp_params = _make_inputs(seed_offset, device, workload)
+    return pool, rows, x, _step_for(x, pool, lp_params, 1, 0, device)
 
 
 class _L2Flush:
@@ -302,8 +325,8 @@ def _prefix_scoring(steps, warmup, device):
     rollout-side overhead the paper measures for PACE (prefix rescoring)."""
     import torch
     from paper_2609_36830_gb300 import pace, workloads
-    spec = workloads.SPECS[WORKLOAD]
-    pool = workloads.make_pool(WORKLOAD)
+    spec = workloads.SPECS[PREFIX_WORKLOAD]
+    pool = workloads.make_pool(PREFIX_WORKLOAD)
     rows = workloads.make_rows(pool)
     pre = workloads.make_prefixes(pool, rows)
     H, V = spec.hidden, spec.vocab
@@ -339,7 +362,7 @@ def _prefix_scoring(steps, warmup, device):
     assert int(status.item()) == 0, pace.status_string(int(status.item()))
     ms = statistics.mean(a.elapsed_time(z) for a, z in ev)
     k_ms = statistics.mean(a.elapsed_time(z) for a, z in kv)
-    res = {"workload": f"{len(pre.traj)} interrupted prefixes of the {WORKLOAD} pool, "
+    res = {"workload": f"{len(pre.traj)} interrupted prefixes of the {PREFIX_WORKLOAD} pool, "
                        f"{pre.n_rows} rows, first 1024 eligible tokens scored",
            "prefixes": len(pre.traj), "rows_scored": scored, "ms_per_call": ms,
            "rows_scored_per_s": scored / (ms / 1e3), "lmhead_ms": k_ms,
@@ -354,7 +377,7 @@ def _lmhead_backward(steps, warmup, device):
     3 x 2 H V FLOP per row in the loss (recomputed logits, G W, G^T H)."""
     import torch
     from paper_2609_36830_gb300 import pace
-    pool, rows, x, st = _make_step(0, device)
+    pool, rows, x, st = _make_step(0, device, workload=PREFIX_WORKLOAD)
     st.run()
     torch.cuda.synchronize()
     M = st.rows_in_loss()
@@ -385,7 +408,7 @@ def _lmhead_backward(steps, warmup, device):
     assert int(st.status.item()) == 0, pace.status_string(int(st.status.item()))
     ms = statistics.mean(b.elapsed_time(e) for b, e in ev)
     flops = 3 * 2.0 * H * V * M
-    res = {"workload": f"{WORKLOAD} step's {M} rows in the loss, H {H}, V {V}",
+    res = {"workload": f"{PREFIX_WORKLOAD} step's {M} rows in the loss, H {H}, V {V}",
            "ms_per_call": ms, "rows_per_s": M / (ms / 1e3),
            "tflops": flops / (ms / 1e3) / 1e12, "flops_per_call": flops}
     del gh, gw, ws, x, st
@@ -394,13 +417,13 @@ def _lmhead_backward(steps, warmup, device):
 
 
 def _other_workloads(steps, warmup, device, peak_s):
-    """The whole step on the multi-turn tool-use pool (256 trajectories, tool segments
-    masked) and the MoE-shaped pool (1024 trajectories, hidden 2048): the same call
-    sequence and launch configuration as the headline step."""
+    """The whole step on the 7B-shaped math pool (512 trajectories, hidden 3584) and
+    the multi-turn tool-use pool (256 trajectories, tool segments masked): the same
+    call sequence and launch configuration as the headline step."""
     import torch
     from paper_2609_36830_gb300 import pace
     res = {}
-    for name in ("multiturn", "moe"):
+    for name in OTHER_WORKLOADS:
         pool, rows, x, st = _make_step(0, device, workload=name)
         for _ in range(warmup):
             st.run()
@@ -432,43 +455,85 @@ def _other_workloads(steps, warmup, device, peak_s):
     return res
 
 
-def _cpu_baseline(pool, rows, x, step_obj, n_rows_sample):
-    """The oracle as it stands on this host's cores: full admission + a row sample."""
-    import torch
-    import oracle
-    t0 = time.perf_counter()
-    st, *_, us = oracle.score_pool(pool.tags, pool.meta["offsets_host"], pool.c_version,
-                                   pool.s_pre, pool.trainer_version, pool.window,
-                                   group_size=pool.group_size)
-    U = pool.n_traj // pool.group_size
-    _, _, _, k = oracle.budget(pool.n_traj, pool.n_target, 0.0, 0.9, 0.0, U)
-    _, _, _, flags = oracle.select(us, pool.group_size, k)
-    t_adm = time.perf_counter() - t0
-    in_loss = np.repeat(flags, np.diff(rows.row_offsets)).astype(bool) & rows.mask.astype(bool)
-    M = int(in_loss.sum())
-    rng = np.random.default_rng(0)
-    sample = np.sort(rng.choice(np.nonzero(in_loss)[0], size=n_rows_sample, replace=False))
-    hb = x.hidden[torch.from_numpy(sample).to(x.hidden.device)].view(torch.int16).cpu().numpy()
-    wb = x.w_vocab.view(torch.int16).cpu().numpy()
+class OracleSampleStep:
+    """The oracle's step on a bounded sample of the workload's batch: full admission of
+    the pool (scores, budget, top-k) then the fp64 log-probs of n_rows sampled rows in
+    the loss and their clipped-surrogate terms.  The vocabulary matrix comes from the
+    same seeded generator as the GPU arm's; hidden rows are drawn on the host."""
+
+    def __init__(self, workload, n_rows, seed_offset=0):
+        import oracle
+        from paper_2609_36830_gb300 import replicas, workloads
+        oracle.build()
+        spec = workloads.SPECS[workload]
+        self.spec = spec
+        self.pool = workloads.make_pool(workload,
+                                        seed=replicas.replica_seed(workload, seed_offset))
+        self.rows = workloads.make_rows(self.pool)
+        H, V = spec.hidden, spec.vocab
+        seed_w = replicas.replica_seed(workload, 0) + 12
+        try:
+            import torch
+            has_gpu = torch.cuda.is_available()
+        except ImportError:
+            has_gpu = False
+        if has_gpu:
+            w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), seed_w)
+            self.wb = w.view(torch.int16).cpu().numpy().view(np.uint16)
+            del w
+        else:
+            self.wb = workloads.bf16_normal_host((V, H), 1.0 / math.sqrt(H), seed_w)
+        self.behav = workloads.behaviour_logprob(self.rows, self.pool.trainer_version,
+                                                 workloads.uniform_center(V), self.pool.seed)
+        self.n_rows = n_rows
+        self.M = None
+
+    def run(self, i, n_threads):
+        """One sample step; returns (seconds, rows in the loss of the whole batch)."""
+        import oracle
+        from paper_2609_36830_gb300 import workloads
+        pool, rows = self.pool, self.rows
+        t0 = time.perf_counter()
+        st, *_, us = oracle.score_pool(pool.tags, pool.meta["offsets_host"], pool.c_version,
+                                       pool.s_pre, pool.trainer_version, pool.window,
+                                       group_size=pool.group_size)
+        U = pool.n_traj // pool.group_size
+        _, _, _, k = oracle.budget(pool.n_traj, pool.n_target, 0.0, 0.9, 0.0, U)
+        _, _, _, flags = oracle.select(us, pool.group_size, k)
+        in_loss = np.repeat(flags, np.diff(rows.row_offsets)).astype(bool) & \
+            rows.mask.astype(bool)
+        self.M = int(in_loss.sum())
+        rng = np.random.default_rng(i)
+        sample = np.sort(rng.choice(np.nonzero(in_loss)[0], size=self.n_rows, replace=False))
+        hb = workloads.bf16_normal_host((self.n_rows, self.spec.hidden), 1.0,
+                                        pool.seed + 11 + i)
+        _, lp, _ = oracle.token_logprob(hb, self.wb, rows.targets[sample], n_threads=n_threads)
+        _, adv = oracle.group_advantages(pool.reward, pool.group_size, seq_accepted=flags)
+        so = np.arange(self.n_rows + 1, dtype=np.int64)
+        seq = np.searchsorted(rows.row_offsets, sample, side="right") - 1
+        oracle.surrogate(lp, self.behav[sample], so, adv[seq],
+                         eps_low=float(np.float32(self.spec.eps_low)),
+                         eps_high=float(np.float32(self.spec.eps_high)))
+        return time.perf_counter() - t0, self.M
+
+
+def _cpu_baseline(n_rows_sample):
+    """The oracle as it stands on this host's cores: one sample step of the headline
+    workload on every core, and a smaller one on one core."""
     cores = os.cpu_count() or 1
-    t0 = time.perf_counter()
-    st, lp, _ = oracle.token_logprob(hb.view(np.uint16), wb.view(np.uint16),
-                                     rows.targets[sample], n_threads=cores)
-    t_lp = time.perf_counter() - t0
-    t_step = t_adm + t_lp * (M / n_rows_sample)
-    # the same oracle on one core, on a 16x smaller row sample
+    ref = OracleSampleStep(WORKLOAD, n_rows_sample)
+    t, M = ref.run(0, cores)
     n1 = max(n_rows_sample // 16, 1)
-    t0 = time.perf_counter()
-    oracle.token_logprob(hb[:n1].view(np.uint16), wb.view(np.uint16),
-                         rows.targets[sample[:n1]], n_threads=1)
-    t_lp1 = time.perf_counter() - t0
-    return {"value": M / t_step, "unit": UNIT, "cores": cores, "kind": "oracle",
+    one = OracleSampleStep(WORKLOAD, n1)
+    t1, _ = one.run(1, 1)
+    return {"value": n_rows_sample / t, "unit": UNIT, "cores": cores, "kind": "oracle",
             "cpu": _cpu_model(),
-            "sample": f"full admission of the {pool.n_traj}-trajectory pool ({t_adm:.3f} s) + "
-                      f"fp64 log-probs of {n_rows_sample} of the {M} rows in the loss "
-                      f"({t_lp:.1f} s), extrapolated to all rows",
-            "single_core": {"value": M / (t_adm + t_lp1 * (M / n1)), "unit": UNIT, "cores": 1,
-                            "sample": f"fp64 log-probs of {n1} rows on one thread ({t_lp1:.1f} s)"}}
+            "sample": f"one step of the {WORKLOAD} pool: full admission of its "
+                      f"{ref.pool.n_traj} trajectories, then fp64 log-probs and surrogate "
+                      f"terms of {n_rows_sample} of the {M} rows in the loss ({t:.1f} s); "
+                      f"value = sampled rows per second of that step",
+            "single_core": {"value": n1 / t1, "unit": UNIT, "cores": 1,
+                            "sample": f"the same with {n1} rows on one thread ({t1:.1f} s)"}}
 
 
 def _cpu_model():
@@ -482,76 +547,55 @@ def _cpu_model():
     return None
 
 
+def _config(ws):
+    """The workload both arms name (the same object in the GPU and reference lines)."""
+    from paper_2609_36830_gb300 import workloads
+    spec = workloads.SPECS[WORKLOAD]
+    return {"workload": "moe: 1024 trajectories (128 prompts x 8) per GPU, lognormal responses "
+                        "(median 4096, cap 16384), capacity 768, hidden 2048, vocab 151936, "
+                        "j=300, EFF scoring gamma 4, groups of 8, clip 0.2/0.28",
+            "global_batch": spec.n_traj * ws,
+            "parallelism": ("dp1: one GPU, whole pool" if ws == 1 else
+                            f"dp{ws}: pool partitioned by prompt group across {ws} GPUs, "
+                            "global top-k by histogram all-reduce, loss by partial-sum "
+                            "all-reduce"),
+            "l2": "inputs larger than L2 (hidden states 21.7 GB per GPU per step)"}
+
+
 def run_reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
         return
-    import torch
-    import oracle
-    from paper_2609_36830_gb300 import workloads
-    spec = workloads.SPECS[WORKLOAD]
-    pool = workloads.make_pool(WORKLOAD)
-    rows = workloads.make_rows(pool)
-    H, V = spec.hidden, spec.vocab
-    oracle.build()
-    # vocabulary and hidden rows from the same seeded generators as the GPU arm
-    if torch.cuda.is_available():
-        w = workloads.bf16_normal_device((V, H), 1.0 / math.sqrt(H), pool.seed + 12)
-        wb = w.view(torch.int16).cpu().numpy().view(np.uint16)
-        del w
-    else:
-        wb = workloads.bf16_normal_host((V, H), 1.0 / math.sqrt(H), pool.seed + 12)
     cores = os.cpu_count() or 1
-    rows_per_step = 64
+    rows_per_step = args.ref_rows
+    ref = OracleSampleStep(WORKLOAD, rows_per_step)
     times = []
     M = None
     for i in range(args.warmup + args.steps):
-        t0 = time.perf_counter()
-        st, *_, us = oracle.score_pool(pool.tags, pool.meta["offsets_host"], pool.c_version,
-                                       pool.s_pre, pool.trainer_version, pool.window,
-                                       group_size=pool.group_size)
-        U = pool.n_traj // pool.group_size
-        _, _, _, k = oracle.budget(pool.n_traj, pool.n_target, 0.0, 0.9, 0.0, U)
-        _, _, _, flags = oracle.select(us, pool.group_size, k)
-        in_loss = np.repeat(flags, np.diff(rows.row_offsets)).astype(bool) & \
-            rows.mask.astype(bool)
-        M = int(in_loss.sum())
-        rng = np.random.default_rng(i)
-        sample = np.sort(rng.choice(np.nonzero(in_loss)[0], size=rows_per_step, replace=False))
-        hb = workloads.bf16_normal_host((rows_per_step, H), 1.0, pool.seed + 11 + i)
-        t_adm = time.perf_counter() - t0
-        t1 = time.perf_counter()
-        oracle.token_logprob(hb, wb, rows.targets[sample], n_threads=cores)
-        t_lp = time.perf_counter() - t1
+        t, M = ref.run(i, cores)
         if i >= args.warmup:
-            times.append(t_adm + t_lp * (M / rows_per_step))
+            times.append(t)
     t = statistics.mean(times)
-    value = M / t
-    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 1,
+    value = rows_per_step / t
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic",
-            "config": {"workload": _workload_name(), "global_batch": pool.n_traj,
-                       "parallelism": "none (CPU oracle)"},
+            "data": "synthetic", "config": _config(ws),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": f"per step: full admission + fp64 log-probs of "
-                                       f"{rows_per_step} of {M} rows in the loss, "
-                                       f"extrapolated to all rows"},
+                             "cpu": _cpu_model(),
+                             "sample": f"per step: full admission of the {ref.pool.n_traj}-"
+                                       f"trajectory pool, then fp64 log-probs and surrogate "
+                                       f"terms of {rows_per_step} of its {M} rows in the loss; "
+                                       f"value = sampled rows per second of the timed steps"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
-def _workload_name():
-    return ("math7b: 512 trajectories (64 prompts x 8), 256 masked prompt rows + lognormal "
-            "responses (median 2048, cap 8192), capacity 384, hidden 3584, vocab 152064, "
-            "j=200, EFF scoring gamma 4, groups of 8")
-
-
 def run_gpu(args):
     import torch
     import torch.distributed as dist
-    from paper_2609_36830_gb300 import pace, step
+    from paper_2609_36830_gb300 import pace, replicas
     ws, rank, local = _dist()
     if ws > 1:
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
@@ -559,10 +603,12 @@ def run_gpu(args):
     device = f"cuda:{local}"
     peaks, peak_src = _peaks()
 
-    pool, rows, x, st = _make_step(rank, device)
+    pool, rows, x, lp_params = _make_inputs(rank, device)
+    st = _step_for(x, pool, lp_params, ws, rank, device)
     H, V = x.hidden.shape[1], x.w_vocab.shape[0]
-    # the LM head's vocabulary split count, measured on this GPU (untimed)
-    splits, split_ms = st.tune_lmhead_splits()
+    # the LM head's vocabulary split count, measured on this GPU (untimed; one GPU:
+    # the ranks of a sharded step keep the automatic choice so that they agree)
+    splits, split_ms = (st.tune_lmhead_splits() if ws == 1 else (0, {}))
     k_units = None
     for _ in range(args.warmup):
         k_units, _ = st.run()
@@ -590,7 +636,6 @@ def run_gpu(args):
     launches = pace.kernel_launches() - launches0
     assert int(st.status.item()) == 0, pace.status_string(int(st.status.item()))
     ms = t_b.elapsed_time(t_e) / K
-    from paper_2609_36830_gb300 import replicas
     job_rows, ms = replicas.job_totals(M, ms, device)
     if ws > 1:
         dist.barrier()
@@ -600,6 +645,7 @@ def run_gpu(args):
     achieved = flops / (lm_ms / 1e3) / 1e12
     peak_s = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
     value = job_rows / (ms / 1e3)
+    loss_value = float(st.loss.item())
 
     # End to end through the same C ABI with host buffers: every step's inputs are
     # copied from pinned host memory and its log-probs and loss copied back.  The
@@ -616,7 +662,7 @@ def run_gpu(args):
         h.copy_(t)
         host[name] = h
     x2 = dataclasses.replace(x, **{name: torch.empty_like(getattr(x, name)) for name in names})
-    st2 = step.PaceStep(x2, loss_params=st.lp_params, device=device)
+    st2 = _step_for(x2, pool, lp_params, ws, rank, device)
     sets = [(x, st), (x2, st2)]
     h2d = sum(h.numel() * h.element_size() for h in host.values())
     lp_host = torch.empty(x.mask.numel(), dtype=torch.float32, pin_memory=True)
@@ -637,6 +683,8 @@ def run_gpu(args):
                 getattr(xi, name).copy_(host[name], non_blocking=True)
             staged[i].record(copy_stream)
 
+    if ws > 1:
+        dist.barrier()
     torch.cuda.synchronize()
     e_b = torch.cuda.Event(enable_timing=True)
     e_e = torch.cuda.Event(enable_timing=True)
@@ -658,8 +706,8 @@ def run_gpu(args):
     _, e_ms = replicas.job_totals(M, e_ms, device)
     del host, x2, st2, sets
 
-    sweep = None
-    if not args.no_sweep and rank == 0:
+    sweep = prefix = backward = others = cpu = None
+    if not args.no_sweep and rank == 0 and ws == 1:
         del x, st
         torch.cuda.empty_cache()
         sizes = []
@@ -675,48 +723,36 @@ def run_gpu(args):
                                                    "tag_reduce_ms", "tag_reduce_gbs",
                                                    "tag_reduce_frac_of_hbm")})
         sweep["smaller_pools"] = sizes
-
-    prefix = None
-    backward = None
-    others = None
-    if not args.no_sweep and rank == 0:
         prefix = _prefix_scoring(max(3, min(K, 5)), 3, device)
         backward = _lmhead_backward(3, 1, device)
-        peak_s_b = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
-        backward["frac_of_sustained"] = backward["tflops"] / peak_s_b
-        others = _other_workloads(3, 2, device, peak_s_b)
-
-    cpu = None
+        backward["frac_of_sustained"] = backward["tflops"] / peak_s
+        others = _other_workloads(3, 2, device, peak_s)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        if sweep is not None:
-            pool, rows, x, st = _make_step(0, device)
-        cpu = _cpu_baseline(pool, rows, x, st, args.cpu_rows)
+        cpu = _cpu_baseline(args.cpu_rows)
 
     if rank == 0:
+        traffic = LMHEAD_DRAM_BYTES_PER_ROW.get(WORKLOAD)
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": K,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": _workload_name(), "global_batch": pool.n_traj * ws,
-                       "rows_in_loss_per_step": M, "rows_total": int(rows.n_rows),
-                       "k_units_rejected": k_units,
-                       "parallelism": f"{ws} independent pool replica(s), no collective",
-                       "l2": "inputs larger than L2 (hidden states 10.7 GB per step)",
-                       "lmhead_splits": {"chosen": splits,
-                                         "tuning_ms_per_step": {str(k): v
-                                                                for k, v in split_ms.items()}}},
+            "config": _config(ws),
+            "step_detail": {"rows_in_loss_per_step": job_rows, "rows_in_loss_rank0": M,
+                            "rows_total_rank0": int(rows.n_rows), "k_units_rejected": k_units,
+                            "loss": loss_value,
+                            "lmhead_splits": {"chosen": splits,
+                                              "tuning_ms_per_step": {str(k): v for k, v
+                                                                     in split_ms.items()}}},
             "roofline": {"bound": "tensor", "kernel": "lmhead_lse_kernel", "achieved": achieved,
                          "peak": peak_s, "unit": "TFLOP/s", "frac": achieved / peak_s,
                          "peak_source": f"{peak_src} bf16_tflops_sustained",
                          "frac_of_burst": achieved / peaks["bf16_tflops"],
-                         "frac_of_nominal_2250": achieved / 2250.0,
                          "kernel_ms": lm_ms, "kernel_ms_each": lm_each,
                          "flops_per_launch": flops,
-                         "traffic": (LMHEAD_DRAM_BYTES_PER_ROW[splits] * M
-                                     if LMHEAD_DRAM_BYTES_PER_ROW
-                                     and splits in LMHEAD_DRAM_BYTES_PER_ROW else None),
-                         "traffic_note": "dram read+write bytes per launch, scaled by rows from "
-                                         "the one-round ncu capture"},
+                         "traffic": traffic * M if traffic else None,
+                         "traffic_note": "dram read+write bytes per launch: bytes per row in the "
+                                         "loss from a one-pass ncu capture of the current kernel, "
+                                         "times the rows of this launch"},
             "cpu_baseline": cpu,
             "e2e": {"value": job_rows / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e_ms},
@@ -891,6 +927,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--cpu-rows", type=int, default=512)
+    ap.add_argument("--ref-rows", type=int, default=96,
+                    help="rows of the batch the reference arm's oracle computes per step")
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", choices=["lmhead", "lmhead_bwd", "tagreduce", "step_tiny", "pool",

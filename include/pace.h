@@ -187,6 +187,60 @@ PACE_API pace_status pace_select_k(const double* unit_score, int64_t n_units, in
 
 PACE_API size_t pace_select_workspace_size(int64_t n_units);
 
+/* ---- Sharded rejection: the pool's units partitioned across ranks --------
+ * The rule of pace_select_k over the WHOLE pool (Sec. 3.1, Algorithm 1: the
+ * k top-scored units are rejected, ties lowest id first), when rank r holds
+ * the contiguous units [u0_r, u0_r + n_units_r) and their unit scores, u0
+ * increasing with r.  Every rank computes the same k (pace_budget on the
+ * whole pool's counts).  The calls run an MSB-first radix select of the
+ * order-preserving 64-bit keys of the scores; the caller sums the histograms
+ * over the ranks between the calls, with any collective:
+ *   for pass in 0..PACE_SHARD_PASSES-1:
+ *     pace_select_shard_pass(.., pass, k, hist_sum_prev, hist_mine, ..)
+ *     hist_sum = sum over ranks of hist_mine         (all-reduce, uint32 bins)
+ *   pace_select_shard_ties(.., hist_sum, &tied_mine, ..)
+ *   tied_before = sum of tied_mine over lower ranks  (exclusive scan)
+ *   pace_select_shard_write(.., k, tied_before, u0 * G, ..)
+ * The union of the ranks' lists is exactly pace_select_k's on the whole pool.
+ * Every call is stream-ordered and needs no host synchronisation; the
+ * workspace (pace_select_shard_workspace_size, 256-byte aligned) carries the
+ * select state from call to call and must not be shared by concurrent calls.
+ *   hist_prev, hist_out, hist_last   device uint32 [PACE_SHARD_HIST_BINS];
+ *                    hist_prev is the summed histogram of pass - 1 (NULL at
+ *                    pass 0); hist_out is this shard's histogram of pass
+ *                    (cleared by the call).
+ *   n_tied_out       device int64 [1]: this shard's units tied at the pivot.
+ *   tied_before      device int64 [1]: units tied at the pivot on lower ranks.
+ *   id_base          the global id of this shard's first trajectory (u0 * G);
+ *                    ids written are id_base + local ids; traj_accepted is
+ *                    indexed locally (n_units * G entries).
+ *   n_rejected_out   device int64 [1] or NULL: units rejected on this shard.
+ * A shard may hold no units (it still takes part in every pass).  NaN scores
+ * report PACE_ERR_NAN_INPUT through status_dev at pass 0. */
+#define PACE_SHARD_PASSES 6
+#define PACE_SHARD_HIST_BINS 2048
+
+PACE_API size_t pace_select_shard_workspace_size(int64_t n_units);
+
+PACE_API pace_status pace_select_shard_pass(const double* unit_score, int64_t n_units,
+                                            int32_t pass, int64_t k_units,
+                                            const uint32_t* hist_prev, uint32_t* hist_out,
+                                            void* workspace, size_t workspace_bytes,
+                                            int32_t* status_dev, void* stream);
+
+PACE_API pace_status pace_select_shard_ties(const double* unit_score, int64_t n_units,
+                                            const uint32_t* hist_last, int64_t* n_tied_out,
+                                            void* workspace, size_t workspace_bytes,
+                                            int32_t* status_dev, void* stream);
+
+PACE_API pace_status pace_select_shard_write(const double* unit_score, int64_t n_units,
+                                             int32_t group_size, int64_t k_units,
+                                             const int64_t* tied_before, int64_t id_base,
+                                             int32_t* accepted_ids, int32_t* rejected_ids,
+                                             uint8_t* traj_accepted, int64_t* n_rejected_out,
+                                             void* workspace, size_t workspace_bytes,
+                                             int32_t* status_dev, void* stream);
+
 /* pace_select_k for callers that cannot allocate device memory.  The paper has
  * no counterpart: this exists for code that must not call cudaMalloc, such as
  * a plugin running inside a host framework whose memory pool owns all device
@@ -257,6 +311,12 @@ typedef struct {
   float* adv;            /* device float32 [n_seq] or NULL: advantages used (output) */
   float* ratio;          /* device float32 [n_rows] or NULL: rho_t of rows in the loss,
                             0 elsewhere (output) */
+  double* partial;       /* device float64 [2] or NULL: the aggregate's numerator and
+                            denominator before the division (output): sum_t m_t L_t
+                            and sum_t m_t (TOKEN_MEAN), or the sum of the sequences'
+                            token means and the number of sequences with tokens
+                            (SEQ_MEAN_TOKEN_MEAN).  Batches split across ranks by
+                            whole prompt groups add these, then divide. */
 } PaceLossArgs;
 
 /* GRPO within-group standardisation over the accepted members of each group:
@@ -313,6 +373,14 @@ PACE_API pace_status pace_surrogate_loss(const PaceBatch* batch, const float* lo
                                 size_t workspace_bytes, int32_t* status_dev, void* stream);
 
 PACE_API size_t pace_surrogate_loss_workspace_size(int64_t n_rows, int64_t n_seq);
+
+/* The loss of a batch split across ranks by whole prompt groups: each rank's
+ * pace_token_logprob / pace_surrogate_loss fills PaceLossArgs.partial; the
+ * caller sums the two values over the ranks (one all-reduce) and this writes
+ * loss = numerator / denominator (0 when the denominator is 0), the division
+ * of the unsplit batch's aggregate.  partial: device float64 [2]; loss: device
+ * float64 [1]. */
+PACE_API pace_status pace_loss_from_partial(const double* partial, double* loss, void* stream);
 
 /* The literal admission rule of Sec. 3.1 and Algorithm 1 (trainer side), kept
  * across steps with a sliding window of recently observed unit scores:

@@ -16,7 +16,7 @@
 //                             MN-major), fp32 accumulation in place.
 // The GEMM is one warp-specialised tcgen05 kernel on CTA pairs: in each CTA
 // warp 0 issues TMA for the CTA's own A tile and its own half of the B tile
-// into a 6-stage ring (128-byte swizzle), both CTAs' bytes completing on the
+// into a 4-stage ring (128-byte swizzle), both CTAs' bytes completing on the
 // even CTA's barrier; warp 1 of the even CTA issues tcgen05.mma.cta_group::2
 // (M 256 = 128 rows per CTA, N 256 = 128 columns from each CTA, K 16; the
 // instruction descriptor's major bits select K- or MN-major operand layouts);
@@ -40,7 +40,7 @@ namespace {
 constexpr int GBM = 128;
 constexpr int GBN = 256;
 constexpr int GBK = 64;
-constexpr int GSTAGES = 6;
+constexpr int GSTAGES = 4;
 constexpr int kGemmThreads = 192;
 constexpr uint32_t kGStageA = GBM * GBK * 2;  // 16 KB
 constexpr uint32_t kGStageB = GBN / 2 * GBK * 2;  // 16 KB: this CTA's half of the B tile

@@ -6,7 +6,7 @@
 // threads, warp-specialised, tcgen05 on the pair):
 //   warp 0 / lane 0   TMA producer, in both CTAs: per K step the CTA's own
 //                     128x64 hidden tile and its own half (128x64) of the pair's
-//                     256x64 vocabulary tile, into its own 6-stage shared-memory
+//                     256x64 vocabulary tile, into its own 4-stage shared-memory
 //                     ring (128-byte swizzle); the transaction bytes of both
 //                     CTAs complete on the even CTA's mbarrier.
 //   warp 1 / lane 0   MMA issuer, even CTA only: tcgen05.mma.cta_group::2
@@ -52,7 +52,7 @@ namespace {
 constexpr int BM = 128;                         // rows per CTA; the pair's MMA covers 256
 constexpr int BN = 256;                         // vocabulary rows per MMA tile (both CTAs)
 constexpr int BK = 64;
-constexpr int STAGES = 6;
+constexpr int STAGES = 4;
 constexpr int CLUSTER = 2;                      // the CTA pair of one 2-CTA MMA
 constexpr int kThreads = 192;
 constexpr uint32_t kStageA = BM * BK * 2;       // 16 KB: this CTA's 128 hidden rows

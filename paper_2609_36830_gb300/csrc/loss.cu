@@ -123,7 +123,7 @@ __global__ void __launch_bounds__(kSurThreads)
 __global__ void __launch_bounds__(kSurThreads)
     surrogate_reduce_kernel(const double* __restrict__ seq_sum,
                             const double* __restrict__ seq_cnt, int64_t n_seq, int agg,
-                            double* __restrict__ loss) {
+                            double* __restrict__ loss, double* __restrict__ partial) {
   __shared__ double sh[kSurThreads];
   double a = 0.0, b = 0.0;
   for (int64_t i = threadIdx.x; i < n_seq; i += kSurThreads) {
@@ -137,7 +137,21 @@ __global__ void __launch_bounds__(kSurThreads)
   }
   const double ta = block_sum_fixed<kSurThreads>(a, sh);
   const double tb = block_sum_fixed<kSurThreads>(b, sh);
-  if (threadIdx.x == 0) *loss = tb > 0.0 ? __ddiv_rn(ta, tb) : 0.0;
+  if (threadIdx.x == 0) {
+    *loss = tb > 0.0 ? __ddiv_rn(ta, tb) : 0.0;
+    if (partial) {
+      partial[0] = ta;
+      partial[1] = tb;
+    }
+  }
+}
+
+// loss = numerator / denominator of partials summed over the parts of a batch
+// (0 for an empty loss), the same correctly rounded division as above.
+__global__ void loss_from_partial_kernel(const double* __restrict__ partial,
+                                         double* __restrict__ loss) {
+  if (threadIdx.x == 0 && blockIdx.x == 0)
+    *loss = partial[1] > 0.0 ? __ddiv_rn(partial[0], partial[1]) : 0.0;
 }
 
 void carve_surrogate_ws(Carver& cv, int64_t n_seq, SurrogateWs* w) {
@@ -183,7 +197,7 @@ pace_status run_surrogate(const PaceBatch* b, const float* logprob, const PaceLo
     PACE_TRY(last_launch_status());
   }
   surrogate_reduce_kernel<<<1, kSurThreads, 0, st>>>(ws.seq_sum, ws.seq_cnt, b->n_seq,
-                                                     l->params.agg, l->loss);
+                                                     l->params.agg, l->loss, l->partial);
   return last_launch_status();
 }
 
@@ -393,4 +407,11 @@ extern "C" pace_status pace_surrogate_loss(const PaceBatch* batch, const float* 
   carve_surrogate_ws(cv, batch->n_seq, &ws);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
   return run_surrogate(batch, logprob, loss, ws, status_dev, as_stream(stream));
+}
+
+extern "C" pace_status pace_loss_from_partial(const double* partial, double* loss,
+                                              void* stream) {
+  if (!partial || !loss) return PACE_ERR_INVALID_ARG;
+  pace::loss_from_partial_kernel<<<1, 32, 0, pace::as_stream(stream)>>>(partial, loss);
+  return pace::last_launch_status();
 }

@@ -117,15 +117,17 @@ __device__ void block_pick(const unsigned* __restrict__ hist, int pass, SelectSt
   __syncthreads();  // s_digit and s_left may be rewritten by the next call
 }
 
+// Unit u's G trajectories: ids id_base + u * G + g in the lists, flags at u * G + g.
 __device__ __forceinline__ void write_unit(int64_t u, bool rejected, int64_t rej_pos,
-                                           int64_t acc_pos, int G, int32_t* accepted_ids,
-                                           int32_t* rejected_ids, uint8_t* flags) {
+                                           int64_t acc_pos, int G, int64_t id_base,
+                                           int32_t* accepted_ids, int32_t* rejected_ids,
+                                           uint8_t* flags) {
   for (int g = 0; g < G; ++g) {
     const int64_t id = u * G + g;
     if (rejected) {
-      if (rejected_ids) rejected_ids[rej_pos * G + g] = static_cast<int32_t>(id);
+      if (rejected_ids) rejected_ids[rej_pos * G + g] = static_cast<int32_t>(id_base + id);
     } else {
-      accepted_ids[acc_pos * G + g] = static_cast<int32_t>(id);
+      accepted_ids[acc_pos * G + g] = static_cast<int32_t>(id_base + id);
     }
     if (flags) flags[id] = rejected ? 0 : 1;
   }
@@ -159,7 +161,7 @@ __global__ void __launch_bounds__(kSmallThreads)
   int n_rej = 0;
   const int rej_before = block_exclusive_scan<int>(rejected, &n_rej);
   if (u < n_units)
-    write_unit(u, rejected, rej_before, u - rej_before, G, accepted_ids, rejected_ids, flags);
+    write_unit(u, rejected, rej_before, u - rej_before, G, 0, accepted_ids, rejected_ids, flags);
 }
 
 // 512 < U <= 131,072: one launch of one thread-block cluster of C CTAs (1, 2,
@@ -563,20 +565,26 @@ __global__ void __launch_bounds__(kSelThreads, 1)
 // buffers: pass p adds into hist[p % 3], reads hist[(p - 1) % 3] and clears
 // hist[(p + 1) % 3] (last read by pass p - 1) for pass p + 1.  State slots
 // alternate: pass p reads slot (p - 1) & 1 and writes slot p & 1.
+//
+// hist_prev is the previous pass's histogram (unused at pass 0), hist_out the
+// cleared histogram this pass adds into, hist_clear (or null) a histogram to
+// clear for the next pass.  The sharded entry points pass the caller's
+// histograms, summed over the ranks between passes.
 __global__ void __launch_bounds__(256)
     radix_pass_kernel(const double* __restrict__ score, int64_t n_units, int pass,
-                      SelectState* states, unsigned* hist3, int32_t* status) {
+                      SelectState* states, const unsigned* hist_prev, unsigned* hist_out,
+                      unsigned* hist_clear, int32_t* status) {
   __shared__ unsigned h[kHistBins];
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x) h[b] = 0;
   SelectState st = states[pass == 0 ? 0 : (pass - 1) & 1];
   if (pass > 0) {
-    block_pick(hist3 + ((pass - 1) % 3) * kHistBins, pass - 1, st);
+    block_pick(hist_prev, pass - 1, st);
     if (blockIdx.x == 0 && threadIdx.x == 0) states[pass & 1] = st;
   }
-  unsigned* clear = hist3 + ((pass + 1) % 3) * kHistBins;
-  for (int64_t b = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < kHistBins;
-       b += static_cast<int64_t>(gridDim.x) * blockDim.x)
-    clear[b] = 0u;
+  if (hist_clear)
+    for (int64_t b = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < kHistBins;
+         b += static_cast<int64_t>(gridDim.x) * blockDim.x)
+      hist_clear[b] = 0u;
   __syncthreads();
   const unsigned long long prefix = st.prefix, mask = st.mask;
   const int shift = c_shift[pass];
@@ -589,9 +597,8 @@ __global__ void __launch_bounds__(256)
     if ((key & mask) == prefix) atomicAdd(&h[(key >> shift) & dmask], 1u);
   }
   __syncthreads();
-  unsigned* out = hist3 + (pass % 3) * kHistBins;
   for (int b = threadIdx.x; b < kHistBins; b += blockDim.x)
-    if (h[b]) atomicAdd(&out[b], h[b]);
+    if (h[b]) atomicAdd(&hist_out[b], h[b]);
 }
 
 // Phase 1: per tile, units equal to the pivot and above it.  The pivot is the
@@ -599,9 +606,9 @@ __global__ void __launch_bounds__(256)
 // state slot kPasses & 1 for the later phases).
 __global__ void __launch_bounds__(kTileThreads)
     count_tile_kernel(const double* __restrict__ score, int64_t n_units, SelectState* states,
-                      const unsigned* hist3, int* eq_cnt, int* gt_cnt) {
+                      const unsigned* hist_last, int* eq_cnt, int* gt_cnt) {
   SelectState st = states[(kPasses - 1) & 1];
-  block_pick(hist3 + ((kPasses - 1) % 3) * kHistBins, kPasses - 1, st);
+  block_pick(hist_last, kPasses - 1, st);
   if (blockIdx.x == 0 && threadIdx.x == 0) states[kPasses & 1] = st;
   const unsigned long long pivot = st.prefix;
   int eq = 0, gt = 0;
@@ -624,12 +631,16 @@ __global__ void __launch_bounds__(kTileThreads)
 }
 
 // Phase 2 (one block): per tile, ties before it and rejections before it.
+// eq_start (or null = 0) counts the ties at the pivot held before this pool's
+// first unit (on lower ranks of a sharded pool); rej_total (or null) receives
+// the number of units rejected here.
 __global__ void __launch_bounds__(1024)
     scan_tiles_kernel(int n_tiles, const SelectState* __restrict__ state, const int* eq_cnt,
-                      const int* gt_cnt, long long* eq_before, long long* rej_before) {
+                      const int* gt_cnt, long long* eq_before, long long* rej_before,
+                      const long long* eq_start, long long* rej_total) {
   __shared__ long long carry_eq, carry_rej;
   if (threadIdx.x == 0) {
-    carry_eq = 0;
+    carry_eq = eq_start ? *eq_start : 0;
     carry_rej = 0;
   }
   __syncthreads();
@@ -656,11 +667,12 @@ __global__ void __launch_bounds__(1024)
     }
     __syncthreads();
   }
+  if (rej_total && threadIdx.x == 0) *rej_total = carry_rej;
 }
 
 // Phase 3: flags and output positions inside each tile.
 __global__ void __launch_bounds__(kTileThreads)
-    write_tile_kernel(const double* __restrict__ score, int64_t n_units, int G,
+    write_tile_kernel(const double* __restrict__ score, int64_t n_units, int G, int64_t id_base,
                       const SelectState* __restrict__ state, const long long* eq_before,
                       const long long* rej_before, int32_t* accepted_ids,
                       int32_t* rejected_ids, uint8_t* flags) {
@@ -693,17 +705,18 @@ __global__ void __launch_bounds__(kTileThreads)
     const int64_t u = base + i;
     if (u >= n_units) break;
     const long long apos = u - rpos;
-    write_unit(u, rej[i], rpos, apos, G, accepted_ids, rejected_ids, flags);
+    write_unit(u, rej[i], rpos, apos, G, id_base, accepted_ids, rejected_ids, flags);
     rpos += rej[i];
   }
 }
 
-__global__ void fill_identity_kernel(int64_t n_units, int G, bool accept, int32_t* accepted_ids,
-                                     int32_t* rejected_ids, uint8_t* flags) {
+__global__ void fill_identity_kernel(int64_t n_units, int G, bool accept, int64_t id_base,
+                                     int32_t* accepted_ids, int32_t* rejected_ids,
+                                     uint8_t* flags) {
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_units * G;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    if (accept) accepted_ids[i] = static_cast<int32_t>(i);
-    else if (rejected_ids) rejected_ids[i] = static_cast<int32_t>(i);
+    if (accept) accepted_ids[i] = static_cast<int32_t>(id_base + i);
+    else if (rejected_ids) rejected_ids[i] = static_cast<int32_t>(id_base + i);
     if (flags) flags[i] = accept ? 1 : 0;
   }
 }
@@ -891,7 +904,7 @@ extern "C" pace_status pace_select_k(const double* unit_score, int64_t n_units, 
     nan_check_kernel<<<grid_for(n_units, 256, 4), 256, 0, st>>>(unit_score, n_units, status_dev);
     PACE_TRY(last_launch_status());
     fill_identity_kernel<<<grid_for(n_units * G, 256, 8), 256, 0, st>>>(
-        n_units, G, k == 0, accepted_ids, rejected_ids, traj_accepted);
+        n_units, G, k == 0, 0, accepted_ids, rejected_ids, traj_accepted);
     return last_launch_status();
   }
   if (n_units <= kSmallMax) {
@@ -916,22 +929,177 @@ extern "C" pace_status pace_select_k(const double* unit_score, int64_t n_units, 
   select_init_kernel<<<1, 256, 0, st>>>(ws.states, static_cast<long long>(k), ws.hist);
   PACE_TRY(last_launch_status());
   const int hist_grid = grid_for(n_units, 256, 2);
+  // histograms rotate through three buffers: pass p adds into hist[p % 3],
+  // reads hist[(p - 1) % 3] and clears hist[(p + 1) % 3] (last read by pass p - 1)
   for (int pass = 0; pass < kPasses; ++pass) {
-    radix_pass_kernel<<<hist_grid, 256, 0, st>>>(unit_score, n_units, pass, ws.states, ws.hist,
-                                                 status_dev);
+    radix_pass_kernel<<<hist_grid, 256, 0, st>>>(
+        unit_score, n_units, pass, ws.states, ws.hist + ((pass + 2) % 3) * kHistBins,
+        ws.hist + (pass % 3) * kHistBins, ws.hist + ((pass + 1) % 3) * kHistBins, status_dev);
     PACE_TRY(last_launch_status());
   }
   const int64_t n_tiles = (n_units + kTile - 1) / kTile;
   const SelectState* final_state = ws.states + (kPasses & 1);
   count_tile_kernel<<<static_cast<unsigned>(n_tiles), kTileThreads, 0, st>>>(
-      unit_score, n_units, ws.states, ws.hist, ws.eq_cnt, ws.gt_cnt);
+      unit_score, n_units, ws.states, ws.hist + ((kPasses - 1) % 3) * kHistBins, ws.eq_cnt,
+      ws.gt_cnt);
   PACE_TRY(last_launch_status());
   scan_tiles_kernel<<<1, 1024, 0, st>>>(static_cast<int>(n_tiles), final_state, ws.eq_cnt,
-                                        ws.gt_cnt, ws.eq_before, ws.rej_before);
+                                        ws.gt_cnt, ws.eq_before, ws.rej_before, nullptr, nullptr);
   PACE_TRY(last_launch_status());
   write_tile_kernel<<<static_cast<unsigned>(n_tiles), kTileThreads, 0, st>>>(
-      unit_score, n_units, G, final_state, ws.eq_before, ws.rej_before, accepted_ids, rejected_ids,
-      traj_accepted);
+      unit_score, n_units, G, 0, final_state, ws.eq_before, ws.rej_before, accepted_ids,
+      rejected_ids, traj_accepted);
+  return last_launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// Sharded rejection (the pool's units partitioned across ranks in contiguous
+// id ranges).  The rule is unchanged: the k top-scored units of the WHOLE pool
+// are rejected, ties lowest id first (Sec. 3.1, Algorithm 1).  The radix
+// select above runs on each shard with the histogram of every pass summed over
+// the ranks by the caller between the calls; then each shard counts its units
+// tied at the pivot, the caller turns those counts into the ties held by lower
+// ranks, and each shard writes its own id lists.
+// ---------------------------------------------------------------------------
+
+namespace pace {
+namespace {
+
+struct ShardWs {
+  SelectState* states;  // two slots, alternating between passes
+  int* eq_cnt;
+  int* gt_cnt;
+  long long* eq_before;
+  long long* rej_before;
+};
+
+ShardWs carve_shard_ws(Carver& cv, int64_t n_units) {
+  const int64_t n_tiles = (n_units + kTile - 1) / kTile;
+  const int64_t t = n_tiles > 0 ? n_tiles : 1;
+  ShardWs w;
+  w.states = cv.take<SelectState>(2);
+  w.eq_cnt = cv.take<int>(t);
+  w.gt_cnt = cv.take<int>(t);
+  w.eq_before = cv.take<long long>(t);
+  w.rej_before = cv.take<long long>(t);
+  return w;
+}
+
+pace_status shard_ws(void* workspace, size_t bytes, int64_t n_units, ShardWs* out) {
+  if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
+  Carver cv(workspace, bytes);
+  *out = carve_shard_ws(cv, n_units);
+  return cv.fits() ? PACE_OK : PACE_ERR_WORKSPACE;
+}
+
+// A shard's number of units tied at the pivot: the sum of the per-tile counts.
+__global__ void tile_total_kernel(int n_tiles, const int* __restrict__ cnt,
+                                  long long* __restrict__ total) {
+  __shared__ long long sh[1024];
+  long long a = 0;
+  for (int t = threadIdx.x; t < n_tiles; t += blockDim.x) a += cnt[t];
+  sh[threadIdx.x] = a;
+  __syncthreads();
+  for (int o = 512; o > 0; o >>= 1) {
+    if (static_cast<int>(threadIdx.x) < o) sh[threadIdx.x] += sh[threadIdx.x + o];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *total = sh[0];
+}
+
+bool shard_shape_ok(int64_t n_units) { return n_units >= 0 && n_units <= (int64_t(1) << 30); }
+
+}  // namespace
+}  // namespace pace
+
+extern "C" size_t pace_select_shard_workspace_size(int64_t n_units) {
+  if (!shard_shape_ok(n_units)) return 0;
+  Carver cv;
+  carve_shard_ws(cv, n_units);
+  return cv.used;
+}
+
+extern "C" pace_status pace_select_shard_pass(const double* unit_score, int64_t n_units,
+                                              int32_t pass, int64_t k_units,
+                                              const uint32_t* hist_prev, uint32_t* hist_out,
+                                              void* workspace, size_t workspace_bytes,
+                                              int32_t* status_dev, void* stream) {
+  if (!shard_shape_ok(n_units) || pass < 0 || pass >= kPasses || k_units < 0 || !hist_out ||
+      (pass > 0 && !hist_prev) || (n_units > 0 && !unit_score))
+    return PACE_ERR_INVALID_ARG;
+  ShardWs ws;
+  PACE_TRY(shard_ws(workspace, workspace_bytes, n_units, &ws));
+  cudaStream_t st = as_stream(stream);
+  unsigned* out = reinterpret_cast<unsigned*>(hist_out);
+  if (pass == 0) {
+    select_init_kernel<<<1, 256, 0, st>>>(ws.states, static_cast<long long>(k_units), out);
+    PACE_TRY(last_launch_status());
+  } else {
+    PACE_TRY_CUDA(cudaMemsetAsync(out, 0, kHistBins * sizeof(unsigned), st));
+  }
+  radix_pass_kernel<<<grid_for(n_units, 256, 2), 256, 0, st>>>(
+      unit_score, n_units, pass, ws.states, reinterpret_cast<const unsigned*>(hist_prev), out,
+      nullptr, status_dev);
+  return last_launch_status();
+}
+
+extern "C" pace_status pace_select_shard_ties(const double* unit_score, int64_t n_units,
+                                              const uint32_t* hist_last, int64_t* n_tied_out,
+                                              void* workspace, size_t workspace_bytes,
+                                              int32_t* status_dev, void* stream) {
+  (void)status_dev;
+  if (!shard_shape_ok(n_units) || !hist_last || !n_tied_out || (n_units > 0 && !unit_score))
+    return PACE_ERR_INVALID_ARG;
+  ShardWs ws;
+  PACE_TRY(shard_ws(workspace, workspace_bytes, n_units, &ws));
+  cudaStream_t st = as_stream(stream);
+  long long* tied = reinterpret_cast<long long*>(n_tied_out);
+  if (n_units == 0) {
+    PACE_TRY_CUDA(cudaMemsetAsync(tied, 0, sizeof(long long), st));
+    return PACE_OK;
+  }
+  const int64_t n_tiles = (n_units + kTile - 1) / kTile;
+  count_tile_kernel<<<static_cast<unsigned>(n_tiles), kTileThreads, 0, st>>>(
+      unit_score, n_units, ws.states, reinterpret_cast<const unsigned*>(hist_last), ws.eq_cnt,
+      ws.gt_cnt);
+  PACE_TRY(last_launch_status());
+  tile_total_kernel<<<1, 1024, 0, st>>>(static_cast<int>(n_tiles), ws.eq_cnt, tied);
+  return last_launch_status();
+}
+
+extern "C" pace_status pace_select_shard_write(const double* unit_score, int64_t n_units,
+                                               int32_t group_size, int64_t k_units,
+                                               const int64_t* tied_before, int64_t id_base,
+                                               int32_t* accepted_ids, int32_t* rejected_ids,
+                                               uint8_t* traj_accepted, int64_t* n_rejected_out,
+                                               void* workspace, size_t workspace_bytes,
+                                               int32_t* status_dev, void* stream) {
+  (void)status_dev;
+  if (!shard_shape_ok(n_units) || group_size < 1 || k_units < 0 || id_base < 0 || !tied_before)
+    return PACE_ERR_INVALID_ARG;
+  if (id_base + n_units * static_cast<int64_t>(group_size) > (int64_t(1) << 31) - 1)
+    return PACE_ERR_INVALID_ARG;
+  if (n_units > 0 && (!unit_score || !accepted_ids)) return PACE_ERR_INVALID_ARG;
+  ShardWs ws;
+  PACE_TRY(shard_ws(workspace, workspace_bytes, n_units, &ws));
+  cudaStream_t st = as_stream(stream);
+  long long* n_rej = reinterpret_cast<long long*>(n_rejected_out);
+  if (n_units == 0 || k_units == 0) {
+    if (n_rej) PACE_TRY_CUDA(cudaMemsetAsync(n_rej, 0, sizeof(long long), st));
+    if (n_units == 0) return PACE_OK;
+    fill_identity_kernel<<<grid_for(n_units * group_size, 256, 8), 256, 0, st>>>(
+        n_units, group_size, true, id_base, accepted_ids, rejected_ids, traj_accepted);
+    return last_launch_status();
+  }
+  const int64_t n_tiles = (n_units + kTile - 1) / kTile;
+  const SelectState* final_state = ws.states + (kPasses & 1);
+  scan_tiles_kernel<<<1, 1024, 0, st>>>(static_cast<int>(n_tiles), final_state, ws.eq_cnt,
+                                        ws.gt_cnt, ws.eq_before, ws.rej_before,
+                                        reinterpret_cast<const long long*>(tied_before), n_rej);
+  PACE_TRY(last_launch_status());
+  write_tile_kernel<<<static_cast<unsigned>(n_tiles), kTileThreads, 0, st>>>(
+      unit_score, n_units, group_size, id_base, final_state, ws.eq_before, ws.rej_before,
+      accepted_ids, rejected_ids, traj_accepted);
   return last_launch_status();
 }
 

@@ -59,7 +59,8 @@ class PaceBatch(ctypes.Structure):
 
 class PaceLossArgs(ctypes.Structure):
     _fields_ = [("behav_lp", _P), ("reward", _P), ("group_size", _I32),
-                ("params", PaceLossParams), ("loss", _P), ("adv", _P), ("ratio", _P)]
+                ("params", PaceLossParams), ("loss", _P), ("adv", _P), ("ratio", _P),
+                ("partial", _P)]
 
 
 # every symbol include/pace.h declares, with its C signature
@@ -76,6 +77,11 @@ SIGNATURES = {
     "pace_select_k": ([_P, _I64, _I32, _I64, _P, _P, _P, _P, _SZ, _P, _P], _I32),
     "pace_select_workspace_size": ([_I64], _SZ),
     "pace_select_k_noalloc": ([_P, _I64, _I32, _I64, _P, _P, _P, _P, _P], _I32),
+    "pace_select_shard_workspace_size": ([_I64], _SZ),
+    "pace_select_shard_pass": ([_P, _I64, _I32, _I64, _P, _P, _P, _SZ, _P, _P], _I32),
+    "pace_select_shard_ties": ([_P, _I64, _P, _P, _P, _SZ, _P, _P], _I32),
+    "pace_select_shard_write": ([_P, _I64, _I32, _I64, _P, _I64, _P, _P, _P, _P, _P, _SZ, _P,
+                                 _P], _I32),
     "pace_loss_params_default": ([_P], None),
     "pace_group_advantages": ([_P, _P, _I64, _I32, _F32, _I32, _P, _P], _I32),
     "pace_token_logprob": ([_P, _P, _P, _P, _I32, _I32, _F32, _P, _P, _P, _P, _SZ, _P, _P],
@@ -83,6 +89,7 @@ SIGNATURES = {
     "pace_token_logprob_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
     "pace_surrogate_loss": ([_P, _P, _P, _P, _SZ, _P, _P], _I32),
     "pace_surrogate_loss_workspace_size": ([_I64, _I64], _SZ),
+    "pace_loss_from_partial": ([_P, _P, _P], _I32),
     "pace_prefix_score": ([_P, _P, _P, _P, _P, _I32, _I32, _F32, _I32, _I32, _P, _P, _P, _SZ,
                            _P, _P], _I32),
     "pace_prefix_score_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
@@ -289,6 +296,53 @@ def select_k(unit_score, group_size, k, out=None, ws=None, status=None, stream=N
             out["flags"][:n])
 
 
+# Sharded rejection (pool partitioned by unit across ranks); histograms are
+# int32 tensors of SHARD_HIST_BINS (the library's uint32 bins; counts < 2^31).
+SHARD_PASSES = 6
+SHARD_HIST_BINS = 2048
+
+
+def select_shard_workspace(n_units, device):
+    return workspace(lib().pace_select_shard_workspace_size(int(n_units)), device)
+
+
+def select_shard_pass(unit_score, pass_, k, hist_prev, hist_out, ws, status=None, stream=None):
+    u = unit_score.numel()
+    st = lib().pace_select_shard_pass(_arg(unit_score, _F64T, u, "unit_score"), u, int(pass_),
+                                      int(k), _arg(hist_prev, _I32T, SHARD_HIST_BINS, "hist_prev"),
+                                      _arg(hist_out, _I32T, SHARD_HIST_BINS, "hist_out"),
+                                      _arg(ws, _U8, None, "ws"), ws.numel(),
+                                      _arg(status, _I32T, 1, "status"), _stream(stream))
+    _check(st, "pace_select_shard_pass")
+
+
+def select_shard_ties(unit_score, hist_last, n_tied_out, ws, status=None, stream=None):
+    u = unit_score.numel()
+    st = lib().pace_select_shard_ties(_arg(unit_score, _F64T, u, "unit_score"), u,
+                                      _arg(hist_last, _I32T, SHARD_HIST_BINS, "hist_last"),
+                                      _arg(n_tied_out, _I64T, 1, "n_tied"),
+                                      _arg(ws, _U8, None, "ws"), ws.numel(),
+                                      _arg(status, _I32T, 1, "status"), _stream(stream))
+    _check(st, "pace_select_shard_ties")
+
+
+def select_shard_write(unit_score, group_size, k, tied_before, id_base, out, ws,
+                       n_rejected_out=None, status=None, stream=None):
+    """out: {"accepted", "rejected", "flags"} of n_units * group_size entries."""
+    u = unit_score.numel()
+    n = u * group_size
+    st = lib().pace_select_shard_write(_arg(unit_score, _F64T, u, "unit_score"), u,
+                                       int(group_size), int(k),
+                                       _arg(tied_before, _I64T, 1, "tied_before"), int(id_base),
+                                       _arg(out["accepted"], _I32T, n, "accepted"),
+                                       _arg(out["rejected"], _I32T, n, "rejected"),
+                                       _arg(out["flags"], _U8, n, "flags"),
+                                       _arg(n_rejected_out, _I64T, 1, "n_rejected"),
+                                       _arg(ws, _U8, None, "ws"), ws.numel(),
+                                       _arg(status, _I32T, 1, "status"), _stream(stream))
+    _check(st, "pace_select_shard_write")
+
+
 # ---------------------------------------------------------------- (b) batch
 
 def loss_params(eps_low=0.2, eps_high=0.28, dual_clip=10.0, adv_eps=1e-6,
@@ -307,13 +361,23 @@ def make_batch(seq_offsets, n_rows, seq_accepted=None, mask=None):
 
 
 def make_loss_args(behav_lp, reward, group_size, params, loss_out, adv_out=None,
-                   ratio_out=None):
+                   ratio_out=None, partial_out=None):
+    """partial_out (float64 [2], optional) receives the aggregate's numerator and
+    denominator, which ranks holding parts of one batch add before dividing."""
     a = PaceLossArgs(_arg(behav_lp, _F32T, None, "behav_lp"), _arg(reward, _F32T, None, "reward"),
                      int(group_size), params, _arg(loss_out, _F64T, 1, "loss"),
                      _arg(adv_out, _F32T, reward.numel(), "adv"),
-                     _arg(ratio_out, _F32T, behav_lp.numel(), "ratio"))
-    a._keep = (behav_lp, reward, loss_out, adv_out, ratio_out)
+                     _arg(ratio_out, _F32T, behav_lp.numel(), "ratio"),
+                     _arg(partial_out, _F64T, 2, "partial"))
+    a._keep = (behav_lp, reward, loss_out, adv_out, ratio_out, partial_out)
     return a
+
+
+def loss_from_partial(partial, loss_out, stream=None):
+    """loss = partial[0] / partial[1] (0 if the denominator is 0), on the device."""
+    st = lib().pace_loss_from_partial(_arg(partial, _F64T, 2, "partial"),
+                                      _arg(loss_out, _F64T, 1, "loss"), _stream(stream))
+    _check(st, "pace_loss_from_partial")
 
 
 def group_advantages(reward, group_size, seq_accepted=None, adv_eps=1e-6, std_unbiased=True,

@@ -1,10 +1,11 @@
-"""Host-side logic of multi-GPU runs: one process per GPU, each running an
-independent replica of the PACE step on its own pool.
+"""Host-side helpers of multi-GPU runs (one process per GPU): the launcher's
+rank environment, the seed of each rank's part of the pool, and the job's
+totals.
 
-The path has no exchange step between replicas (each trainer replica admits
-from its own pool), so a job of N ranks is N weak-scaled replicas: distinct
-seeds per rank, a barrier around the timed region, the maximum of the ranks'
-step times as the job's time, and the sum of the ranks' rows as the job's work.
+A data-parallel step (sharded.ShardedPaceStep) partitions the pool by prompt
+group: rank r draws its groups with its own seed, and the whole pool is the
+union of the ranks' parts.  The job's work is the sum of the ranks' rows in the
+loss and its time the slowest rank's, with a barrier around the timed region.
 """
 from __future__ import annotations
 
@@ -21,7 +22,7 @@ def rank_env() -> Tuple[int, int, int]:
 
 
 def replica_seed(workload: str, rank: int) -> int:
-    """Seed of rank's pool: rank 0 draws the workload's default pool."""
+    """Seed of rank's part of the pool: rank 0 draws the workload's default pool."""
     return workloads.SEED_BASE + workloads.SPECS[workload].index + 1000 * rank
 
 

@@ -168,6 +168,7 @@ int main(int argc, char** argv) {
     la.loss = d_loss;
     la.adv = d_adv;
     la.ratio = NULL;
+    la.partial = NULL;
     st[3] = pace_token_logprob(&batch, d_hid, d_w, (const int32_t*)d_tgt, H, V, 1.0f, d_lp2, NULL,
                                &la, d_ws3, ws_bytes, d_status, NULL);
     CHECK_CUDA(cudaDeviceSynchronize());

@@ -47,3 +47,19 @@ def test_peaks_are_the_measured_file_when_present():
     else:
         assert src == "fallback" and peaks["hbm_gbs"] == 6800.0
     assert peaks["bf16_tflops_sustained"] <= peaks["bf16_tflops"]
+
+
+def test_both_arms_name_the_same_config():
+    """The GPU line and the reference line take their config from one function:
+    the workload, the whole job's batch and the partition at each N."""
+    c1, c8 = bench._config(1), bench._config(8)
+    assert c1["global_batch"] == 1024 and c8["global_batch"] == 8 * 1024
+    assert c1["workload"] == c8["workload"] and c1["workload"].startswith("moe:")
+    assert c1["parallelism"].startswith("dp1") and c8["parallelism"].startswith("dp8")
+
+
+def test_oracle_sample_step_on_the_tiny_pool():
+    """The reference arm's step (full admission + a row sample) runs on the host alone."""
+    ref = bench.OracleSampleStep("tiny", 8)
+    t, M = ref.run(0, 2)
+    assert t > 0 and M == ref.M and 8 <= M <= int(ref.rows.mask.sum())

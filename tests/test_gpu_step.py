@@ -2,9 +2,11 @@
 the full-size workloads (7B single-turn at occupancies 1.0 / 1.33 / 2.0 of
 capacity, multi-turn with tool segments at 1.0 / 2.5, the MoE head), in
 exactly the launch configuration bench.py times: the selection must match the
-oracle id for id, sampled log-probs within 5e-3, and the fused loss must equal
-the standalone surrogate on the same log-probs (whose parity with the oracle
-is pinned in test_gpu_loss.py at these sizes).  Then the occupancy EMA
+oracle id for id, sampled log-probs within 5e-3, the fused loss must equal
+the standalone surrogate on the same log-probs, and it must match the oracle's
+surrogate computed over every row from the GPU log-probs (verified on the
+sample) and the same behaviour log-probs, within 1e-3 relative (to the larger
+of |loss| and the mean |term| of the rows in the loss).  Then the occupancy EMA
 (Eq. 4) carried across steps."""
 import math
 
@@ -62,6 +64,18 @@ def test_full_size_step(name, n_traj):
     assert float(st.loss.item()) == float(loss2.item())
     assert math.isfinite(float(st.loss.item()))
     assert st.rows_in_loss() == int(in_loss.sum())
+    # fused loss against the oracle's surrogate over all rows (GRPO
+    # advantages over the accepted members of each group)
+    _, oadv = oracle.group_advantages(pool.reward, pool.group_size, seq_accepted=oflag,
+                                      eps=float(np.float32(1e-6)))
+    sst, oloss, _, oterm = oracle.surrogate(lp, behav, rw.row_offsets, oadv, mask=rw.mask,
+                                            seq_accepted=oflag,
+                                            eps_low=float(np.float32(pool.spec.eps_low)),
+                                            eps_high=float(np.float32(pool.spec.eps_high)),
+                                            dual_clip=10.0)
+    assert sst == 0
+    scale = max(abs(oloss), float(np.abs(oterm[in_loss]).mean()))
+    assert abs(float(st.loss.item()) - oloss) <= 1e-3 * scale, (float(st.loss.item()), oloss)
 
 
 def test_ema_budget_carried_across_steps():

@@ -1,6 +1,6 @@
-"""Multi-rank host logic of bench.py on CPU: two gloo ranks, each with its own
-pool, reduce their work and time the way the GPU job does (sum of rows, max of
-step times), and their pools are distinct replicas."""
+"""Multi-rank bookkeeping of bench.py on CPU: two gloo ranks, each with its own
+part of the pool, reduce their work and time the way the GPU job does (sum of
+rows, max of step times), and their parts are distinct draws."""
 import os
 import socket
 
