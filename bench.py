@@ -44,11 +44,15 @@ sys.path.insert(0, ROOT)
 WORKLOAD = "moe"
 OTHER_WORKLOADS = ("math7b", "multiturn")
 PREFIX_WORKLOAD = "math7b"  # prefix rescoring and the backward are timed on the 7B math pool
-# DRAM bytes (read + written) per row in the loss of the LM-head kernel, by workload, from a
-# one-pass ncu capture (dram__bytes_read.sum + dram__bytes_write.sum) of one launch of the
-# current kernel; None until the current kernel has been captured.  The tag reduction's per
-# tag: 14.0656 GB read + 19.8 MB written for the 3.5023 G tags of the 1M sweep pool.
-LMHEAD_DRAM_BYTES_PER_ROW = {}
+# DRAM bytes (read + written) per row in the loss of the LM-head kernel, by (workload,
+# vocabulary splits), from one-pass ncu captures (dram__bytes_read.sum + dram__bytes_write.sum)
+# of one 400,000-row launch of the current kernel on the MoE-shaped head: 76.23 GB + 44.1 MB
+# with 4 splits, 35.38 GB + 18.3 MB with 2 (the vocabulary is read 1.4-1.5 times per round of
+# items, so the traffic grows with the rows).  Emptied whenever the kernel changes, until it is
+# captured again.  The tag reduction's per tag: 14.0656 GB read + 19.8 MB written for the
+# 3.5023 G tags of the 1M sweep pool.
+LMHEAD_DRAM_BYTES_PER_ROW = {("moe", 4): (76225025024 + 44133120) / 400000,
+                             ("moe", 2): (35377250048 + 18313216) / 400000}
 TAG_REDUCE_DRAM_BYTES_PER_TAG = (14065824512 + 19798528) / 3502330341
 SWEEP_N = 1048576
 SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)
@@ -731,7 +735,8 @@ def run_gpu(args):
         cpu = _cpu_baseline(args.cpu_rows)
 
     if rank == 0:
-        traffic = LMHEAD_DRAM_BYTES_PER_ROW.get(WORKLOAD)
+        chosen = splits or 4  # the automatic choice at this size is 4 (pick_splits)
+        traffic = LMHEAD_DRAM_BYTES_PER_ROW.get((WORKLOAD, chosen))
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": K,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,

@@ -132,4 +132,4 @@ extern "C" const char* pace_status_string(pace_status status) {
   return "PACE_ERR_UNKNOWN";
 }
 
-extern "C" int32_t pace_version(void) { return 200; }
+extern "C" int32_t pace_version(void) { return 300; }

@@ -53,7 +53,7 @@ def test_host_entry_points_from_c99(tmp_path):
     stdin = "".join(f"{n} {nt} {b!r} {m!r} {p!r} {u}\n" for n, nt, b, m, p, u in cases)
     r = subprocess.run([exe], input=stdin, capture_output=True, text=True, check=True)
     lines = r.stdout.strip().splitlines()
-    assert lines[0] == "version 200"
+    assert lines[0] == "version 300"
     assert lines[1] == "status PACE_OK PACE_ERR_TIMEOUT PACE_ERR_UNKNOWN"
     assert lines[2].split()[1:5] == ["0", "4", "32", "8"]
     assert float.fromhex(lines[3].split()[3]) == 0.9

@@ -45,7 +45,7 @@ def test_status_strings_and_defaults(pace):
     assert pace.status_string(0) == "PACE_OK"
     assert pace.status_string(2) == "PACE_ERR_VERSION_ORDER"
     assert pace.status_string(99) == "PACE_ERR_UNKNOWN"
-    assert pace.lib().pace_version() == 200  # 0.2.0: pace_set_lmhead_splits added
+    assert pace.lib().pace_version() == 300  # 0.3.0: sharded selection, PaceLossArgs.partial
     sp = pace.PaceScoreParams()
     pace.lib().pace_score_params_default(ctypes.byref(sp))
     assert (sp.mode, sp.gamma, sp.min_obs, sp.group_size, sp.f_missing) == (0, 4, 32, 8, 1.0)
