@@ -112,8 +112,31 @@ struct LmArgs {
   float* part_m;                // [rows_cap * kMaxSplits], row r's splits at r * S
   float* part_s;
   float* tgt_logit;             // [rows_cap]
+  unsigned* round_ctr;          // pacing counter, zero at launch (or null: no pacing)
   int32_t* status;
 };
+
+// Longest a cluster waits at a round boundary for the others (a soft barrier:
+// it proceeds after this even if some cluster is late, so it can never hang).
+constexpr uint64_t kRoundWaitNs = 250000;  // 250 us
+
+// Pacing of the persistent clusters.  The clusters sweeping one vocabulary
+// split share its tiles through L2 only while they stay close; left alone, their
+// small speed differences add up over the hundreds of rounds of a long launch,
+// the leaders fetch tiles from DRAM that the laggards fetch again later, and the
+// extra DRAM traffic costs the power-capped SMs their clock (a 1.01M-row launch
+// of the 7B head read the vocabulary 8.7 times per round).  So before starting
+// its k-th item a cluster waits until every cluster has issued the loads of its
+// (k-1)-th (the counter holds the number of items whose loads were issued), for
+// at most kRoundWaitNs.
+__device__ __forceinline__ void wait_round(const unsigned* ctr, unsigned target) {
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    if (*reinterpret_cast<const volatile unsigned*>(ctr) >= target) return;
+    if (global_timer_ns() - t0 > kRoundWaitNs) return;
+    __nanosleep(128);
+  }
+}
 
 __device__ __forceinline__ uint64_t make_policy_evict_normal() {
   uint64_t pol;
@@ -206,10 +229,15 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
       const uint64_t pol = make_policy_evict_normal();
       uint32_t it = 0;
       bool ok = true;
-      for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next()) {
+      unsigned round = 0;  // this cluster's items so far (the round of the current one)
+      for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next(), ++round) {
         const int64_t rp = c.item / n_splits;
         const int split = static_cast<int>(c.item % n_splits);
         const int32_t row0 = static_cast<int32_t>((rp * CLUSTER + crank) * BM);
+        // every round before the last is full, so round k starts once all
+        // clusters issued their round k-1 loads (the even CTA paces the pair)
+        if (leader && round > 0 && p.round_ctr)
+          wait_round(p.round_ctr, round * static_cast<unsigned>(n_clusters));
         const int tile0 = split * tiles_per_split;
         const int tile1 = min(tile0 + tiles_per_split, p.n_vtiles);
         for (int t = tile0; t < tile1 && ok; ++t) {
@@ -229,6 +257,7 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
             tma_load_2d_pair(sb, &tm_b, bar, kb * BK, nb, pol);
           }
         }
+        if (leader && ok && p.round_ctr) atomicAdd(p.round_ctr, 1u);
       }
       if (!ok) give_up();
       // Drain: every copy issued must have landed before the CTA exits.  The
@@ -469,6 +498,7 @@ void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, bool compact,
   w->part_m = cv.take<float>(static_cast<size_t>(rows_cap) * kMaxSplits);
   w->part_s = cv.take<float>(static_cast<size_t>(rows_cap) * kMaxSplits);
   w->tgt = cv.take<float>(static_cast<size_t>(rows_cap));
+  w->round_ctr = cv.take<unsigned>(1);
 }
 
 bool lm_needs_compaction(const PaceBatch* b) {
@@ -531,12 +561,14 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   a.part_m = ws.part_m;
   a.part_s = ws.part_s;
   a.tgt_logit = ws.tgt;
+  a.round_ctr = ws.round_ctr;
   a.status = status_dev;
   // persistent: at most one wave of 2-CTA clusters, never more clusters than the
   // most items the rows could make (the split count is chosen on the device)
   const int64_t items = (rows_cap + 2 * BM - 1) / (2 * BM) * kMaxSplits;
   const int64_t clusters = items < li.max_clusters ? items : li.max_clusters;
   const int64_t grid = clusters * CLUSTER;
+  PACE_TRY_CUDA(cudaMemsetAsync(ws.round_ctr, 0, sizeof(unsigned), st));
   const ProfileEvents& pe = profile_events(PACE_PROFILE_LMHEAD);
   if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
   lmhead_lse_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tm_a, tm_b, a);

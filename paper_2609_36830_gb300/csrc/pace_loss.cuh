@@ -27,6 +27,7 @@ struct LmWs {
   float* part_m;
   float* part_s;
   float* tgt;
+  unsigned* round_ctr;  // the LM head's pacing counter (items whose loads were issued)
 };
 
 void carve_surrogate_ws(Carver& cv, int64_t n_seq, SurrogateWs* w);
