@@ -46,13 +46,12 @@ OTHER_WORKLOADS = ("math7b", "multiturn")
 PREFIX_WORKLOAD = "math7b"  # prefix rescoring and the backward are timed on the 7B math pool
 # DRAM bytes (read + written) per row in the loss of the LM-head kernel, by (workload,
 # vocabulary splits), from one-pass ncu captures (dram__bytes_read.sum + dram__bytes_write.sum)
-# of one 400,000-row launch of the current kernel on the MoE-shaped head: 76.23 GB + 44.1 MB
-# with 4 splits, 35.38 GB + 18.3 MB with 2 (the vocabulary is read 1.4-1.5 times per round of
-# items, so the traffic grows with the rows).  Emptied whenever the kernel changes, until it is
-# captured again.  The tag reduction's per tag: 14.0656 GB read + 19.8 MB written for the
-# 3.5023 G tags of the 1M sweep pool.
-LMHEAD_DRAM_BYTES_PER_ROW = {("moe", 4): (76225025024 + 44133120) / 400000,
-                             ("moe", 2): (35377250048 + 18313216) / 400000}
+# of one launch of the current kernel at this bench's size (3,958,414 rows of the MoE-shaped
+# head): 526.726 GB + 191.1 MB with 4 splits, 296.312 GB + 126.1 MB with 2.  Emptied whenever
+# the kernel changes, until it is captured again.  The tag reduction's per tag: 14.0656 GB
+# read + 19.8 MB written for the 3.5023 G tags of the 1M sweep pool.
+LMHEAD_DRAM_BYTES_PER_ROW = {("moe", 4): (526726449920 + 191105792) / 3958414,
+                             ("moe", 2): (296312474368 + 126139136) / 3958414}
 TAG_REDUCE_DRAM_BYTES_PER_TAG = (14065824512 + 19798528) / 3502330341
 SWEEP_N = 1048576
 SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)

@@ -79,6 +79,7 @@ struct GemmArgs {
   int64_t ldo;
   // EPI_ACC
   float* acc_out;               // fp32 [M][ldo]
+  unsigned* round_ctr;          // pacing counter, zeroed before the launch (or null)
   int32_t* status;
 };
 
@@ -213,11 +214,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
       asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
       uint32_t it = 0;
       bool ok = true;
-      for (int64_t t = cid; t < n_items && ok; t += n_clusters) {
+      unsigned round = 0;  // this cluster's items so far
+      for (int64_t t = cid; t < n_items && ok; t += n_clusters, ++round) {
         int64_t mp, nt;
         item_of(p, m_tiles, t, &mp, &nt);
         const int32_t m0 = static_cast<int32_t>((2 * mp + crank) * GBM);
         const int32_t n0 = static_cast<int32_t>(nt * GBN);
+        // the clusters start each round together (every round but the last is full)
+        if (leader && round > 0 && p.round_ctr)
+          wait_round(p.round_ctr, round * static_cast<unsigned>(n_clusters));
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const uint32_t s = it % GSTAGES, ph = (it / GSTAGES) & 1u;
           if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
@@ -254,6 +259,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             tma_load_2d_pair(sb, &tm_b, bar, k0, nh, pol);
           }
         }
+        if (leader && ok && p.round_ctr) atomicAdd(p.round_ctr, 1u);
       }
       if (!ok) give_up();
       // every copy issued has landed before the CTA exits: the even CTA sees
@@ -495,7 +501,7 @@ __global__ void count_used_seqs_kernel(const long long* __restrict__ seq_in, int
 
 template <bool A_MN, bool B_MN, int EPI>
 pace_status launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmArgs a,
-                        cudaStream_t st) {
+                        unsigned* round_ctr, cudaStream_t st) {
   constexpr int kMaxDevices = 64;
   static bool done[kMaxDevices] = {};  // shared-memory opt-in made on that device
   static std::mutex mu;
@@ -517,6 +523,8 @@ pace_status launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, GemmArgs a
   if (items == 0) return PACE_OK;
   const int64_t max_clusters = sm_count() / 2;
   const int64_t grid = 2 * (items < max_clusters ? items : max_clusters);
+  PACE_TRY_CUDA(cudaMemsetAsync(round_ctr, 0, sizeof(unsigned), st));
+  a.round_ctr = round_ctr;
   gemm_kernel<A_MN, B_MN, EPI><<<static_cast<unsigned>(grid), kGemmThreads, kGSmemBytes, st>>>(
       ta, tb, a);
   return last_launch_status();
@@ -526,6 +534,7 @@ struct BwWs {
   LmWs lm;            // compaction + gathered rows (hidden_c)
   uint16_t* g;        // bf16 G of one chunk, 64-column blocks [ceil(V / 64)][chunk][64]
   int* n_seq_used;
+  unsigned* round_ctr;  // the GEMMs' pacing counter
 };
 
 int64_t chunk_rows(int64_t n_rows) {
@@ -538,6 +547,7 @@ void carve_bw_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, int V, BwWs* 
   const int64_t g_cols = (static_cast<int64_t>(V) + 63) / 64 * 64;
   w->g = cv.take<uint16_t>(static_cast<size_t>(chunk_rows(n_rows > 0 ? n_rows : 1)) * g_cols);
   w->n_seq_used = cv.take<int>(1);
+  w->round_ctr = cv.take<unsigned>(1);
 }
 
 }  // namespace
@@ -664,7 +674,7 @@ extern "C" pace_status pace_token_logprob_backward(
       a.g_pitch = rows_c_pad;
       a.V = V;
       a.status = status_dev;
-      PACE_TRY((launch_gemm<false, false, EPI_G>(ta, tb, a, st)));
+      PACE_TRY((launch_gemm<false, false, EPI_G>(ta, tb, a, ws.round_ctr, st)));
     }
     // 2. dH rows = G W   (W read MN-major: [K = V][N = H])
     {
@@ -684,7 +694,7 @@ extern "C" pace_status pace_token_logprob_backward(
       a.rows_out = grad_hidden;
       a.ldo = H;
       a.status = status_dev;
-      PACE_TRY((launch_gemm<false, true, EPI_ROWS>(ta, tb, a, st)));
+      PACE_TRY((launch_gemm<false, true, EPI_ROWS>(ta, tb, a, ws.round_ctr, st)));
     }
     // 3. dW += G^T H_c   (G read MN-major: [K = rows][M = V]; H_c MN-major: [K = rows][N = H])
     {
@@ -703,7 +713,7 @@ extern "C" pace_status pace_token_logprob_backward(
       a.acc_out = grad_w;
       a.ldo = H;
       a.status = status_dev;
-      PACE_TRY((launch_gemm<true, true, EPI_ACC>(ta, tb, a, st)));
+      PACE_TRY((launch_gemm<true, true, EPI_ACC>(ta, tb, a, ws.round_ctr, st)));
     }
   }
   return PACE_OK;

@@ -26,7 +26,14 @@
 // of S contiguous vocabulary splits; each CTA writes one (max, sum) pair per row
 // and split.  Consecutive items share a row pair, so the hidden tiles re-read
 // for every vocabulary tile stay in L2 while the vocabulary streams.  S is
-// chosen on the device from the rows actually present (pick_splits).
+// chosen on the device from the rows actually present (pick_splits).  A soft
+// barrier at item boundaries (wait_round) keeps the clusters of a split
+// together, so each vocabulary tile is fetched from DRAM about once per round:
+// left alone, the clusters' small speed differences add up over the hundreds
+// of rounds of a long launch, the leaders fetch tiles from DRAM that the
+// laggards fetch again later, and the extra DRAM traffic costs the
+// power-capped SMs their clock (a 1.01M-row launch of the 7B head read the
+// vocabulary 8.7 times per round; paced, 1.02 times).
 //
 // lse_merge_kernel: per row, merges the S partial pairs into the log-sum-exp
 //   and writes lp = z_y / tau - lse.
@@ -115,28 +122,6 @@ struct LmArgs {
   unsigned* round_ctr;          // pacing counter, zero at launch (or null: no pacing)
   int32_t* status;
 };
-
-// Longest a cluster waits at a round boundary for the others (a soft barrier:
-// it proceeds after this even if some cluster is late, so it can never hang).
-constexpr uint64_t kRoundWaitNs = 250000;  // 250 us
-
-// Pacing of the persistent clusters.  The clusters sweeping one vocabulary
-// split share its tiles through L2 only while they stay close; left alone, their
-// small speed differences add up over the hundreds of rounds of a long launch,
-// the leaders fetch tiles from DRAM that the laggards fetch again later, and the
-// extra DRAM traffic costs the power-capped SMs their clock (a 1.01M-row launch
-// of the 7B head read the vocabulary 8.7 times per round).  So before starting
-// its k-th item a cluster waits until every cluster has issued the loads of its
-// (k-1)-th (the counter holds the number of items whose loads were issued), for
-// at most kRoundWaitNs.
-__device__ __forceinline__ void wait_round(const unsigned* ctr, unsigned target) {
-  const uint64_t t0 = global_timer_ns();
-  for (;;) {
-    if (*reinterpret_cast<const volatile unsigned*>(ctr) >= target) return;
-    if (global_timer_ns() - t0 > kRoundWaitNs) return;
-    __nanosleep(128);
-  }
-}
 
 __device__ __forceinline__ uint64_t make_policy_evict_normal() {
   uint64_t pol;

@@ -205,6 +205,27 @@ __device__ __forceinline__ bool mbar_wait_bounded_cluster(uint64_t* bar, uint32_
   }
 }
 
+// ---- pacing of persistent clusters
+
+// Longest a cluster waits at a round boundary for the others (a soft barrier:
+// it proceeds after this even if some cluster is late, so it can never hang).
+constexpr uint64_t kRoundWaitNs = 250000;  // 250 us
+
+// Persistent clusters that take items c, c + n_clusters, ... share the operand
+// tiles of a round through L2 only while they stay in step.  Before its k-th
+// item a cluster waits until the counter (items whose loads were issued,
+// zeroed before the launch, incremented once per item by each cluster) reaches
+// k * n_clusters, for at most kRoundWaitNs.  A timing signal only: no data is
+// passed through the counter.
+__device__ __forceinline__ void wait_round(const unsigned* ctr, unsigned target) {
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    if (*reinterpret_cast<const volatile unsigned*>(ctr) >= target) return;
+    if (global_timer_ns() - t0 > kRoundWaitNs) return;
+    __nanosleep(128);
+  }
+}
+
 // ---- TMA (bulk tensor copies, global -> shared)
 
 __device__ __forceinline__ void tma_prefetch_desc(const void* desc) {
