@@ -164,65 +164,6 @@ __global__ void __launch_bounds__(kSmallThreads)
     write_unit(u, rejected, rej_before, u - rej_before, G, 0, accepted_ids, rejected_ids, flags);
 }
 
-// 512 < U <= kRankMax: the same ranks, spread over many blocks.  Every block
-// loads all U order keys into shared memory; each warp ranks one unit (its 32
-// lanes split the U comparisons) and stores whether it is rejected (rank < k)
-// in decision[u].  The second kernel (one block) turns the decisions into the
-// id lists.  decision is the caller's accepted_ids buffer, whose final
-// contents the second kernel writes only after it has read every decision.
-constexpr int kRankMax = 4096;
-constexpr int kRankThreads = 256;  // 8 warps: 8 units per block
-
-__global__ void __launch_bounds__(kRankThreads)
-    select_rank_kernel(const double* __restrict__ score, int n_units, int64_t k,
-                       int32_t* __restrict__ decision, int32_t* status) {
-  __shared__ uint64_t s[kRankMax];
-  for (int u = threadIdx.x; u < n_units; u += blockDim.x) {
-    const double x = score[u];
-    if (blockIdx.x == 0 && isnan(x)) report(status, PACE_ERR_NAN_INPUT);
-    s[u] = order_key(x);
-  }
-  __syncthreads();
-  const int lane = threadIdx.x & 31;
-  const int u = static_cast<int>(blockIdx.x) * (kRankThreads / 32) + (threadIdx.x >> 5);
-  if (u >= n_units) return;  // whole warps leave together
-  const uint64_t x = s[u];
-  unsigned rank = 0;
-  for (int w = lane; w < n_units; w += 32) {
-    const uint64_t y = s[w];
-    rank += (y > x) || (y == x && w < u);
-  }
-  rank = __reduce_add_sync(0xffffffffu, rank);
-  if (lane == 0) decision[u] = static_cast<int64_t>(rank) < k ? 1 : 0;
-}
-
-// One block: decisions (in accepted_ids) -> positions -> id lists and flags.
-__global__ void __launch_bounds__(1024)
-    select_rank_write_kernel(int n_units, int G, int32_t* accepted_ids, int32_t* rejected_ids,
-                             uint8_t* flags) {
-  constexpr int kPer = kRankMax / 1024;
-  int rej[kPer];
-  int mine = 0;
-  const int base = static_cast<int>(threadIdx.x) * kPer;  // contiguous units per thread
-#pragma unroll
-  for (int i = 0; i < kPer; ++i) {
-    const int u = base + i;
-    rej[i] = u < n_units ? accepted_ids[u] : 0;
-    mine += rej[i];
-  }
-  // every decision is read (the scan's barriers) before any list is written
-  int rpos = block_exclusive_scan<int>(mine, nullptr);
-  __syncthreads();
-#pragma unroll
-  for (int i = 0; i < kPer; ++i) {
-    const int u = base + i;
-    if (u < n_units) {
-      write_unit(u, rej[i] != 0, rpos, u - rpos, G, 0, accepted_ids, rejected_ids, flags);
-      rpos += rej[i];
-    }
-  }
-}
-
 // 512 < U <= 131,072: one launch of one thread-block cluster of C CTAs (1, 2,
 // 4 or 8; 1024 threads each).  CTA r owns the contiguous units
 // [r * B, r * B + B) with B = ceil(U / C) <= 16,384; its thread t owns the
@@ -970,15 +911,6 @@ extern "C" pace_status pace_select_k(const double* unit_score, int64_t n_units, 
     select_small_kernel<<<1, kSmallThreads, 0, st>>>(unit_score, static_cast<int>(n_units), G, k,
                                                      accepted_ids, rejected_ids, traj_accepted,
                                                      status_dev);
-    return last_launch_status();
-  }
-  if (n_units <= kRankMax) {
-    const int blocks = static_cast<int>((n_units + kRankThreads / 32 - 1) / (kRankThreads / 32));
-    select_rank_kernel<<<blocks, kRankThreads, 0, st>>>(unit_score, static_cast<int>(n_units), k,
-                                                        accepted_ids, status_dev);
-    PACE_TRY(last_launch_status());
-    select_rank_write_kernel<<<1, 1024, 0, st>>>(static_cast<int>(n_units), G, accepted_ids,
-                                                 rejected_ids, traj_accepted);
     return last_launch_status();
   }
   if (n_units <= kSelMaxUnits) {
