@@ -548,6 +548,19 @@ PACE_API pace_status pace_set_lmhead_splits(int32_t splits);
  * the caller.  Returns PACE_ERR_INVALID_ARG for an unknown kernel. */
 PACE_API pace_status pace_set_profile_events(int32_t kernel, void* begin, void* end);
 
+/* Not part of the method: checks the integer construction of the doubles the
+ * scoring writes.  For every i, with T[i] >= 1:
+ *   q_int[i]  = S[i] / T[i] as the scoring kernels build it on the integer pipe,
+ *   q_fp64[i] = the same quotient from the fp64 pipe, __ll2double_rn(S[i]) then
+ *               a correctly rounded division (the rounding the oracle's
+ *               (double)S / (double)T performs),
+ *   c_int[i], c_fp64[i] = (double)S[i] both ways.
+ * The two must agree bit for bit.  All arrays are device arrays of n entries.
+ * Returns PACE_ERR_INVALID_ARG for n < 0 or a NULL array when n > 0. */
+PACE_API pace_status pace_div_selftest(const int64_t* S, const uint32_t* T, int64_t n,
+                                       double* q_int, double* q_fp64, double* c_int,
+                                       double* c_fp64, void* stream);
+
 /* Not part of the method: exercises the failure path every tensor-core
  * kernel relies on.  One GPU thread waits, with the same bounded wait the
  * kernels use, on an mbarrier that nothing ever completes; after limit_ns

@@ -54,6 +54,111 @@ __device__ __forceinline__ void l2_prefetch_bulk(const void* p, uint32_t bytes) 
                : "memory");
 }
 
+// ---- exact integer quotients without the fp64 pipe
+//
+// GB300's fp64 pipe is narrow, and the finalisation is bound by it (one int64
+// to double conversion and one correctly rounded division per trajectory).  The
+// functions below build the same doubles from integer arithmetic: the result
+// of __ddiv_rn(__ll2double_rn(S), T) for 64-bit S and 32-bit T > 0, and of
+// __ll2double_rn(x), bit for bit.
+
+// (double)x rounded to nearest even, from its bits (every int64 is in range).
+__device__ __forceinline__ double i64_to_double_rn(long long x) {
+  if (x == 0) return 0.0;
+  const unsigned long long sign = x < 0 ? (1ull << 63) : 0ull;
+  unsigned long long a = x < 0 ? 0ull - static_cast<unsigned long long>(x)
+                               : static_cast<unsigned long long>(x);
+  int top = 63 - __clzll(static_cast<long long>(a));  // leading bit position
+  unsigned long long mant;
+  if (top <= 52) {
+    mant = a << (52 - top);
+  } else {
+    const int sh = top - 52;  // bits dropped, 1..11
+    mant = a >> sh;
+    const unsigned long long rem = a & ((1ull << sh) - 1);
+    const unsigned long long half = 1ull << (sh - 1);
+    if (rem > half || (rem == half && (mant & 1ull))) ++mant;
+    if (mant >> 53) {  // carried into a new bit: 2^53 -> 2^52 one binade up
+      mant >>= 1;
+      ++top;
+    }
+  }
+  const unsigned long long bits = sign | (static_cast<unsigned long long>(top + 1023) << 52) |
+                                  (mant & ((1ull << 52) - 1));
+  return __longlong_as_double(static_cast<long long>(bits));
+}
+
+// RN(RN53(S) / T): exactly __ddiv_rn(__ll2double_rn(S), (double)T), T >= 1.
+// |S| is first rounded to 53 significant bits (a * 2^e, a < 2^53) as the
+// conversion does; then q = a / T, r = a % T and the fraction r / T is
+// developed in 32-bit digits by integer division, giving a 64-bit quotient
+// with its leading bit set plus a sticky bit, which is rounded to 53 bits
+// (nearest, ties to even).  The quotient lies in [2^-32, 2^63], always normal.
+__device__ __forceinline__ double i64_div_u32_rn(long long S, unsigned T) {
+  if (S == 0) return 0.0;
+  const unsigned long long sign = S < 0 ? (1ull << 63) : 0ull;
+  unsigned long long a = S < 0 ? 0ull - static_cast<unsigned long long>(S)
+                               : static_cast<unsigned long long>(S);
+  int e = 0;  // the dividend is a * 2^e
+  {
+    const int top = 63 - __clzll(static_cast<long long>(a));
+    if (top > 52) {
+      const int sh = top - 52;
+      unsigned long long m = a >> sh;
+      const unsigned long long rem = a & ((1ull << sh) - 1);
+      const unsigned long long half = 1ull << (sh - 1);
+      if (rem > half || (rem == half && (m & 1ull))) ++m;
+      e = sh;
+      if (m >> 53) {  // 2^53 = 2^52 * 2: keep a below 2^53
+        m >>= 1;
+        ++e;
+      }
+      a = m;
+    }
+  }
+  const unsigned long long t = T;
+  const unsigned long long q = a / t;
+  const unsigned long long r = a - q * t;
+  // fraction digits of r / T (r < T < 2^32, so each digit fits 32 bits)
+  const unsigned long long n1 = r << 32;
+  const unsigned long long d1 = n1 / t;
+  const unsigned long long r1 = n1 - d1 * t;
+  const unsigned long long n2 = r1 << 32;
+  const unsigned long long d2 = n2 / t;
+  const unsigned long long r2 = n2 - d2 * t;
+  const unsigned long long frac = (d1 << 32) | d2;  // r / T = frac * 2^-64 + ...
+  unsigned long long x;  // 64 significant bits, leading bit at 63
+  bool sticky;
+  int exp2;              // exponent of the leading bit
+  if (q != 0) {
+    const int lq = 64 - __clzll(static_cast<long long>(q));  // bits of q, 1..53
+    const int f = 64 - lq;                                   // fraction bits kept, 11..63
+    x = (q << f) | (frac >> lq);
+    sticky = r2 != 0 || (frac & ((1ull << lq) - 1)) != 0;
+    exp2 = lq - 1 + e;
+  } else {
+    // r / T >= 2^-32: frac has at most 31 leading zeros; a third digit refills them
+    const unsigned long long n3 = r2 << 32;
+    const unsigned long long d3 = n3 / t;
+    const unsigned long long r3 = n3 - d3 * t;
+    const int lz = __clzll(static_cast<long long>(frac));  // 0..31
+    x = lz ? (frac << lz) | (d3 >> (32 - lz)) : frac;
+    sticky = r3 != 0 || (lz ? ((d3 << (32 + lz)) != 0) : (d3 != 0));
+    exp2 = -1 - lz + e;
+  }
+  unsigned long long mant = x >> 11;  // 53 bits
+  const bool round_bit = (x >> 10) & 1ull;
+  const bool rest = sticky || (x & 0x3FFull) != 0;
+  if (round_bit && (rest || (mant & 1ull))) ++mant;
+  if (mant >> 53) {
+    mant >>= 1;
+    ++exp2;
+  }
+  const unsigned long long bits = sign | (static_cast<unsigned long long>(exp2 + 1023) << 52) |
+                                  (mant & ((1ull << 52) - 1));
+  return __longlong_as_double(static_cast<long long>(bits));
+}
+
 struct LaneAcc {
   long long sum;   // sum of policy tags seen by this lane for the current trajectory
   unsigned cnt;    // number of policy tokens
@@ -426,9 +531,9 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
       report(p.status, PACE_ERR_VERSION_ORDER);
     // Lemma 1: K_gen = (1/T) sum (c - v_t) = (c T - sum v_t) / T, exact integers
     const long long gen_sum = static_cast<long long>(c) * static_cast<long long>(t_count) - tag_sum;
-    const double kgen =
-        t_count > 0u ? __ddiv_rn(__ll2double_rn(gen_sum), __ull2double_rn(t_count)) : 0.0;
-    const double kwait = __ll2double_rn(static_cast<long long>(p.j) - c);
+    // the correctly rounded K_gen and K_wait, built on the integer pipe
+    const double kgen = t_count > 0u ? i64_div_u32_rn(gen_sum, t_count) : 0.0;
+    const double kwait = i64_to_double_rn(static_cast<long long>(p.j) - c);
     double f;
     if (!p.window_ready) {
       f = 1.0;
@@ -491,8 +596,7 @@ __global__ void stale_k_kernel(const int64_t* __restrict__ offsets,
   if (mp1 != 0u && static_cast<int64_t>(mp1) - 1 > j) report(status, PACE_ERR_VERSION_ORDER);
   const long long lag_sum = static_cast<long long>(j) * static_cast<long long>(t_count) -
                             static_cast<long long>(sumv[i]);
-  const double kb =
-      t_count > 0u ? __ddiv_rn(__ll2double_rn(lag_sum), __ull2double_rn(t_count)) : 0.0;
+  const double kb = t_count > 0u ? i64_div_u32_rn(lag_sum, t_count) : 0.0;
   if (kbar) kbar[i] = kb;
   admitted[i] = kb <= k_max ? 1 : 0;
 }
@@ -698,4 +802,37 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
                       static_cast<size_t>(threads) * sizeof(int);
   score_finalize_kernel<<<static_cast<unsigned>(blocks), threads, smem, st>>>(a);
   return last_launch_status();
+}
+
+namespace pace {
+namespace {
+
+// Both constructions of the same doubles, side by side (the self-test below).
+__global__ void div_selftest_kernel(const long long* __restrict__ S,
+                                    const unsigned* __restrict__ T, int64_t n,
+                                    double* __restrict__ q_int, double* __restrict__ q_fp64,
+                                    double* __restrict__ c_int, double* __restrict__ c_fp64) {
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    q_int[i] = i64_div_u32_rn(S[i], T[i]);
+    q_fp64[i] = __ddiv_rn(__ll2double_rn(S[i]), __ull2double_rn(T[i]));
+    c_int[i] = i64_to_double_rn(S[i]);
+    c_fp64[i] = __ll2double_rn(S[i]);
+  }
+}
+
+}  // namespace
+}  // namespace pace
+
+extern "C" pace_status pace_div_selftest(const int64_t* S, const uint32_t* T, int64_t n,
+                                         double* q_int, double* q_fp64, double* c_int,
+                                         double* c_fp64, void* stream) {
+  if (n < 0 || (n > 0 && (!S || !T || !q_int || !q_fp64 || !c_int || !c_fp64)))
+    return PACE_ERR_INVALID_ARG;
+  if (n == 0) return PACE_OK;
+  pace::div_selftest_kernel<<<static_cast<unsigned>(n < 4096 ? (n + 255) / 256 : 16 * pace::sm_count()),
+                              256, 0, pace::as_stream(stream)>>>(
+      reinterpret_cast<const long long*>(S), reinterpret_cast<const unsigned*>(T), n, q_int,
+      q_fp64, c_int, c_fp64);
+  return pace::last_launch_status();
 }

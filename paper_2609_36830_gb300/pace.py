@@ -106,6 +106,7 @@ SIGNATURES = {
     "pace_set_lmhead_splits": ([_I32], _I32),
     "pace_kernel_launches": ([], ctypes.c_uint64),
     "pace_wait_timeout_selftest": ([ctypes.c_uint64, _P, _P], _I32),
+    "pace_div_selftest": ([_P, _P, _I64, _P, _P, _P, _P, _P], _I32),
 }
 
 

@@ -252,3 +252,31 @@ def test_large_logits(scale):
     assert np.isfinite(lp).all() and np.isfinite(lse).all()
     assert np.abs(lp - olp).max() <= TOL, np.abs(lp - olp).max()
     assert np.abs(lse - olse).max() <= TOL, np.abs(lse - olse).max()
+
+
+def test_concurrent_launches_on_two_streams():
+    """Two LM-head calls at once on two streams, each sized to fill the GPU: the second
+    launch's clusters are not all resident until the first's retire, so its round barrier
+    (a bounded wait on the other clusters' progress) times out and proceeds on the resident
+    ones.  Both results must equal the same calls run one after the other, with no
+    timeout reported."""
+    rows, H, V = 100000, 1024, 8192  # ~20 rounds of items per launch
+    hb = workloads.bf16_normal_host((rows, H), 1.0, 31)
+    wb = workloads.bf16_normal_host((V, H), 2.0 / math.sqrt(H), 32)
+    y = np.random.default_rng(33).integers(0, V, size=rows).astype(np.int32)
+    hidden, w, tg = bf16_dev(hb), bf16_dev(wb), to_dev(y)
+    b = pace.make_batch(torch.tensor([0, rows], dtype=torch.int64, device=DEV), rows)
+    ref = [_run(hidden, w, tg)[0] for _ in range(2)]
+    outs, statuses = [], []
+    streams = [torch.cuda.Stream(device=DEV) for _ in range(2)]
+    ws = [pace.workspace(pace.token_logprob_workspace_size(rows, 1, H, V), DEV) for _ in range(2)]
+    torch.cuda.synchronize()
+    for s, w_s in zip(streams, ws):
+        with torch.cuda.stream(s):
+            st = pace.new_status(DEV)
+            outs.append(pace.token_logprob(b, hidden, w, tg, 1.0, ws=w_s, status=st))
+            statuses.append(st)
+    torch.cuda.synchronize()
+    assert all(int(st.item()) == 0 for st in statuses)
+    for lp, r in zip(outs, ref):
+        np.testing.assert_array_equal(as_np(lp), r)

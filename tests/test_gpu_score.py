@@ -1,5 +1,6 @@
 """Pool scoring on the GPU vs the oracle: fp64 bits must be identical
 (K_gen, K_wait, F, score, unit score) on every workload, mode and edge case."""
+import ctypes
 import json
 import os
 
@@ -235,3 +236,44 @@ def test_device_side_errors(what, code):
     else:
         off[10] = off[11] + 1  # not non-decreasing
     gpu_score(tags, off, c, pool.s_pre, j, w, expect_status=code)
+
+
+def _div_selftest(S, T):
+    L = pace.lib()
+    n = S.size
+    dS, dT = to_dev(S.astype(np.int64)), to_dev(T.astype(np.uint32).view(np.int32))
+    outs = [torch.empty(n, dtype=torch.float64, device=DEV) for _ in range(4)]
+    st = L.pace_div_selftest(ctypes.c_void_p(dS.data_ptr()), ctypes.c_void_p(dT.data_ptr()), n,
+                             *[ctypes.c_void_p(o.data_ptr()) for o in outs], None)
+    assert st == pace.OK
+    torch.cuda.synchronize()
+    return [as_np(o) for o in outs]
+
+
+def test_integer_quotient_matches_the_fp64_pipe_bit_for_bit():
+    """K_gen = S / T and K_wait = (double)x are built on the integer pipe (GB300's
+    fp64 pipe bounds the finalisation).  They must equal __ddiv_rn(__ll2double_rn(S), T)
+    and __ll2double_rn(x) bit for bit - and numpy's float64(S) / float64(T) on the
+    host, the oracle's arithmetic - over all magnitudes and the rounding edge cases."""
+    rng = np.random.default_rng(99)
+    n = 1 << 20
+    bits_s = rng.integers(0, 64, size=n)
+    S = (rng.integers(0, 1 << 62, size=n, dtype=np.int64) >> (62 - np.minimum(bits_s, 62)))
+    S = np.where(bits_s == 63, rng.integers(-(1 << 62), 1 << 62, size=n, dtype=np.int64) * 2 + 1,
+                 S)
+    S = np.where(rng.random(n) < 0.5, -S, S)
+    bits_t = rng.integers(0, 33, size=n)
+    T = (rng.integers(1, 1 << 32, size=n, dtype=np.int64) >> (32 - bits_t)).clip(1, (1 << 32) - 1)
+    edge_s = [0, 1, -1, 7, (1 << 53) - 1, 1 << 53, (1 << 53) + 1, (1 << 53) + 3, (1 << 54) + 2,
+              (1 << 54) + 6, -(1 << 53) - 1, (1 << 62) + (1 << 9), (1 << 63) - 1, -(1 << 63),
+              -((1 << 63) - 1), 3 * 5 * 7 * 11 * 13 * (1 << 20), 123456789012345]
+    edge_t = [1, 2, 3, 7, (1 << 31), (1 << 32) - 1, 65535, 3 * 5 * 7]
+    es, et = np.meshgrid(np.array(edge_s, dtype=np.int64), np.array(edge_t, dtype=np.int64))
+    S = np.concatenate([S, es.ravel(), np.arange(-5000, 5000, dtype=np.int64) * 37])
+    T = np.concatenate([T, et.ravel(), np.full(10000, 37, np.int64)])
+    q_int, q_fp64, c_int, c_fp64 = _div_selftest(S, T)
+    np.testing.assert_array_equal(q_int.view(np.uint64), q_fp64.view(np.uint64))
+    np.testing.assert_array_equal(c_int.view(np.uint64), c_fp64.view(np.uint64))
+    host = S.astype(np.float64) / T.astype(np.float64)
+    np.testing.assert_array_equal(q_int.view(np.uint64), host.view(np.uint64))
+    np.testing.assert_array_equal(c_int.view(np.uint64), S.astype(np.float64).view(np.uint64))
