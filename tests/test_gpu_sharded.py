@@ -112,3 +112,23 @@ def test_sharded_step_matches_single_gpu_step_and_oracle(name, n_traj, n_shards)
     in_loss = np.repeat(oflag, np.diff(rw.row_offsets)).astype(bool) & rw.mask.astype(bool)
     scale = max(abs(oloss), float(np.abs(oterm[in_loss]).mean()))
     assert abs(losses[0] - oloss) <= 1e-3 * scale
+
+
+def test_sharded_selection_reports_nan_scores():
+    """A NaN unit score on any shard is reported through that shard's status word
+    (first pass), as the single-GPU selection does."""
+    us = np.linspace(0.0, 5.0, 600)
+    us[450] = np.nan
+    bounds = [0, 300, 600]
+    statuses, gens, bufs = [], [], []
+    for u0, u1 in zip(bounds[:-1], bounds[1:]):
+        buf = sharded.ShardSelectBuffers(u1 - u0, 2, DEV)
+        st = pace.new_status(DEV)
+        gens.append(sharded.select_protocol(to_dev(np.ascontiguousarray(us[u0:u1])), 2, 100,
+                                            u0 * 2, buf, status=st))
+        statuses.append(st)
+        bufs.append(buf)
+    sharded.run_lockstep(gens)
+    torch.cuda.synchronize()
+    assert int(statuses[0].item()) == 0
+    assert int(statuses[1].item()) == pace.ERR_NAN_INPUT

@@ -117,3 +117,41 @@ def test_lmhead_split_control_range(pace):
     for good in (0, 1, 2, 4, 8):
         assert L.pace_set_lmhead_splits(good) == pace.OK
     assert L.pace_set_lmhead_splits(0) == pace.OK  # back to the automatic choice
+
+
+def test_shard_selection_argument_checks_return_before_launch(pace):
+    """The sharded rejection's calls refuse bad arguments on the host, before any launch."""
+    L = pace.lib()
+    fake = ctypes.c_void_p(0x1000)
+    ws = ctypes.c_void_p(0x100000)  # 256-byte aligned, never dereferenced here
+    n = 1 << 20
+    assert L.pace_select_shard_workspace_size(100) > 0
+    assert L.pace_select_shard_workspace_size(-1) == 0
+    # pass out of range, a negative k, a missing histogram, no previous histogram after pass 0
+    assert L.pace_select_shard_pass(fake, 100, 6, 3, fake, fake, ws, n, None, None) == \
+        pace.ERR_INVALID_ARG
+    assert L.pace_select_shard_pass(fake, 100, 0, -1, None, fake, ws, n, None, None) == \
+        pace.ERR_INVALID_ARG
+    assert L.pace_select_shard_pass(fake, 100, 0, 3, None, None, ws, n, None, None) == \
+        pace.ERR_INVALID_ARG
+    assert L.pace_select_shard_pass(fake, 100, 2, 3, None, fake, ws, n, None, None) == \
+        pace.ERR_INVALID_ARG
+    # workspace missing, unaligned or too small
+    assert L.pace_select_shard_pass(fake, 100, 0, 3, None, fake, None, n, None, None) == \
+        pace.ERR_WORKSPACE
+    assert L.pace_select_shard_pass(fake, 100, 0, 3, None, fake, ctypes.c_void_p(0x100008), n,
+                                    None, None) == pace.ERR_WORKSPACE
+    assert L.pace_select_shard_pass(fake, 100, 0, 3, None, fake, ws, 8, None, None) == \
+        pace.ERR_WORKSPACE
+    # ties: missing output; write: ids past int32, missing tie count, bad group size
+    assert L.pace_select_shard_ties(fake, 100, fake, None, ws, n, None, None) == \
+        pace.ERR_INVALID_ARG
+    assert L.pace_select_shard_write(fake, 100, 8, 3, fake, (1 << 31) - 100, fake, fake, fake,
+                                     None, ws, n, None, None) == pace.ERR_INVALID_ARG
+    assert L.pace_select_shard_write(fake, 100, 8, 3, None, 0, fake, fake, fake, None, ws, n,
+                                     None, None) == pace.ERR_INVALID_ARG
+    assert L.pace_select_shard_write(fake, 100, 0, 3, fake, 0, fake, fake, fake, None, ws, n,
+                                     None, None) == pace.ERR_INVALID_ARG
+    assert L.pace_loss_from_partial(None, fake, None) == pace.ERR_INVALID_ARG
+    assert L.pace_div_selftest(None, None, -1, None, None, None, None, None) == \
+        pace.ERR_INVALID_ARG
