@@ -5,10 +5,12 @@
 //                       bound): per trajectory the count T of policy tokens,
 //                       the exact integer sum of their tags and the largest
 //                       tag (+1, for the Lemma 1 premise check).
-//   window_prep_kernel  (pools of 32k trajectories and more) block 0 sorts the
-//                       prefix-score window W; the other blocks tabulate
-//                       F = phi(count / |W|) (Eqs. 9-10) for every possible count
-//                       0..|W| (F depends on s only through the count).
+//                       On pools of 32k trajectories and more the same launch
+//                       also prepares the prefix-score window (extra blocks
+//                       after the streaming ones, run in its tail): one sorts W,
+//                       the others tabulate F = phi(count / |W|) (Eqs. 9-10)
+//                       for every possible count 0..|W| (F depends on s only
+//                       through the count).
 //   score_finalize_kernel  one thread per trajectory: K_gen, K_wait, the ECDF
 //                       count of s against the window (binary search in the
 //                       sorted window, or a direct count on small pools), F
@@ -246,15 +248,101 @@ __device__ __forceinline__ void acc_group(LaneAcc& a, const int4& q) {
 // any length mix are balanced across warps.  The walk never leaves
 // [0, n_traj) and loads only tags[0, n_tokens), whatever the offsets hold;
 // inconsistent offsets are reported by the finalize kernel.
+// phi_gamma(q) of Eq. 10 with integer gamma, powers by repeated
+// multiplication, every operation rounded once (no FMA).
+__device__ __forceinline__ double sharpen(double q, int gamma) {
+  const double omq = __dsub_rn(1.0, q);
+  double a = q, b = omq;
+  for (int g = 1; g < gamma; ++g) {
+    a = __dmul_rn(a, q);
+    b = __dmul_rn(b, omq);
+  }
+  return __ddiv_rn(a, __dadd_rn(a, b));
+}
+
+// The prefix-score window's preparation, done by extra blocks of the tag
+// reduction's launch (the blocks after its streaming blocks): they are
+// scheduled as the streaming blocks retire, so the preparation runs in the
+// reduction's ragged tail instead of as a launch of its own.  Prep block 0
+// sorts the window ascending (bitonic, in dynamic shared memory, padded to a
+// power of two with +inf, which sorts last and is never read back); the other
+// prep blocks tabulate F[c] = phi_gamma(c / n) for c = 0..n, kFPerBlock entries
+// each, so the table's fp64 divisions and products run on many SMs instead of
+// queueing on one SM's fp64 units.  NaN in the window is a data error.
+constexpr int kFPerBlock = 32;
+
+struct WindowPrep {
+  const float* window;  // null: no preparation blocks
+  int n;
+  int gamma;
+  float* sorted;        // [n]
+  double* f_table;      // [n + 1]
+  int32_t* status;
+};
+
+inline unsigned window_prep_blocks(int64_t n) {
+  return 1u + static_cast<unsigned>((n + 1 + kFPerBlock - 1) / kFPerBlock);
+}
+
+inline size_t window_prep_smem(int64_t n) {
+  size_t np2 = 1;
+  while (np2 < static_cast<size_t>(n)) np2 <<= 1;
+  return np2 * sizeof(float);
+}
+
+__device__ void window_prep_block(int b, const WindowPrep& w) {
+  const int n = w.n;
+  if (b > 0) {
+    const int c = (b - 1) * kFPerBlock + static_cast<int>(threadIdx.x);
+    if (threadIdx.x < kFPerBlock && c <= n)
+      w.f_table[c] = sharpen(__ddiv_rn(static_cast<double>(c), static_cast<double>(n)), w.gamma);
+    return;
+  }
+  extern __shared__ float sw[];
+  int np2 = 1;
+  while (np2 < n) np2 <<= 1;
+  for (int k = threadIdx.x; k < np2; k += blockDim.x) {
+    float v = k < n ? w.window[k] : __int_as_float(0x7f800000);
+    if (isnan(v)) {
+      report(w.status, PACE_ERR_NAN_INPUT);
+      v = __int_as_float(0x7f800000);
+    }
+    sw[k] = v;
+  }
+  // Each step compares the pairs (lo, lo + stride): pair i puts a zero bit at
+  // the stride's position of i, so every thread has work on every step.
+  for (int size = 2; size <= np2; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      __syncthreads();
+      for (int i = threadIdx.x; i < (np2 >> 1); i += blockDim.x) {
+        const int lo = ((i & ~(stride - 1)) << 1) | (i & (stride - 1));
+        const int hi = lo | stride;
+        const float a = sw[lo], c = sw[hi];
+        if ((a > c) == ((lo & size) == 0)) {
+          sw[lo] = c;
+          sw[hi] = a;
+        }
+      }
+    }
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < n; k += blockDim.x) w.sorted[k] = sw[k];
+}
+
 template <int kTilesPerBatch, int kMinBlocks>
 __global__ void __launch_bounds__(kReduceThreads, kMinBlocks)
     tag_reduce_kernel(const int32_t* __restrict__ tags, const int64_t* __restrict__ offsets,
                       int64_t n_traj, int64_t n_tokens, unsigned long long* __restrict__ sumv,
-                      unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1) {
+                      unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1,
+                      int n_stream_blocks, WindowPrep prep) {
+  if (static_cast<int>(blockIdx.x) >= n_stream_blocks) {  // the window's preparation
+    window_prep_block(static_cast<int>(blockIdx.x) - n_stream_blocks, prep);
+    return;
+  }
   constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const int64_t n_warps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  const int64_t n_warps = (static_cast<int64_t>(n_stream_blocks) * blockDim.x) >> 5;
   const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
   const int64_t b_begin = n_batches * warp / n_warps;
   const int64_t b_end = n_batches * (warp + 1) / n_warps;
@@ -403,65 +491,6 @@ struct FinalizeArgs {
   double* unit_score;
   int32_t* status;
 };
-
-// phi_gamma(q) of Eq. 10 with integer gamma, powers by repeated
-// multiplication, every operation rounded once (no FMA).
-__device__ __forceinline__ double sharpen(double q, int gamma) {
-  const double omq = __dsub_rn(1.0, q);
-  double a = q, b = omq;
-  for (int g = 1; g < gamma; ++g) {
-    a = __dmul_rn(a, q);
-    b = __dmul_rn(b, omq);
-  }
-  return __ddiv_rn(a, __dadd_rn(a, b));
-}
-
-// Block 0 sorts the window ascending (bitonic, in shared memory, padded to a
-// power of two with +inf, which sorts last and is never read back); the other
-// blocks tabulate F[c] = phi_gamma(c / n) for c = 0..n, kFPerBlock entries
-// each, so the table's fp64 divisions and products run on many SMs instead of
-// queueing on one SM's fp64 units.  NaN in the window is a data error.
-constexpr int kFPerBlock = 32;
-
-__global__ void __launch_bounds__(1024) window_prep_kernel(const float* __restrict__ window, int n,
-                                                           int gamma, float* __restrict__ sorted,
-                                                           double* __restrict__ f_table,
-                                                           int32_t* status) {
-  if (blockIdx.x > 0) {
-    const int c = (static_cast<int>(blockIdx.x) - 1) * kFPerBlock + static_cast<int>(threadIdx.x);
-    if (threadIdx.x < kFPerBlock && c <= n)
-      f_table[c] = sharpen(__ddiv_rn(static_cast<double>(c), static_cast<double>(n)), gamma);
-    return;
-  }
-  __shared__ float sw[kMaxWindow];
-  int np2 = 1;
-  while (np2 < n) np2 <<= 1;
-  for (int k = threadIdx.x; k < np2; k += blockDim.x) {
-    float w = k < n ? window[k] : __int_as_float(0x7f800000);
-    if (isnan(w)) {
-      report(status, PACE_ERR_NAN_INPUT);
-      w = __int_as_float(0x7f800000);
-    }
-    sw[k] = w;
-  }
-  for (int size = 2; size <= np2; size <<= 1) {
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      __syncthreads();
-      for (int k = threadIdx.x; k < np2; k += blockDim.x) {
-        const int partner = k ^ stride;
-        if (partner > k) {
-          const float a = sw[k], b = sw[partner];
-          if ((a > b) == ((k & size) == 0)) {
-            sw[k] = b;
-            sw[partner] = a;
-          }
-        }
-      }
-    }
-  }
-  __syncthreads();
-  for (int k = threadIdx.x; k < n; k += blockDim.x) sorted[k] = sw[k];
-}
 
 // blockDim.x = tpb * lanes: tpb trajectories per block (whole groups) and, on
 // the direct-count path, `lanes` threads per trajectory that each count one
@@ -628,11 +657,16 @@ ScoreWs carve_score_ws(Carver& cv, int64_t n_traj) {
   return w;
 }
 
-// Zero the accumulators and stream the tags once.
+// Zero the accumulators and stream the tags once; with prep.window set, the
+// same launch also sorts the window and tabulates F (extra blocks, run in the
+// stream's tail).
 pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t n_traj,
-                           int64_t n_tokens, const ScoreWs& ws, cudaStream_t st) {
+                           int64_t n_tokens, const ScoreWs& ws, const WindowPrep& prep,
+                           cudaStream_t st) {
   PACE_TRY_CUDA(cudaMemsetAsync(ws.sumv, 0, static_cast<size_t>(n_traj) * 16, st));
-  if (n_tokens == 0) return PACE_OK;
+  const unsigned prep_blocks = prep.window ? window_prep_blocks(prep.n) : 0u;
+  const size_t prep_smem = prep.window ? window_prep_smem(prep.n) : 0;
+  if (n_tokens == 0 && prep_blocks == 0) return PACE_OK;
   const bool small = n_tokens <= kSmallPoolTokens;
   const int tiles = small ? kTilesSmall : kTilesLarge;
   const int per_sm = small ? kBlocksSmall : kBlocksLarge;
@@ -642,16 +676,16 @@ pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t 
   int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
   const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;  // one wave
   if (blocks > cap) blocks = cap;
+  const unsigned grid = static_cast<unsigned>(blocks) + prep_blocks;
+  const int stream_blocks = static_cast<int>(blocks);
   const ProfileEvents& pe = profile_events(PACE_PROFILE_TAG_REDUCE);
   if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
   if (small)
-    tag_reduce_kernel<kTilesSmall, kBlocksSmall><<<static_cast<unsigned>(blocks), kReduceThreads,
-                                                   0, st>>>(tags, offsets, n_traj, n_tokens,
-                                                            ws.sumv, ws.cnt, ws.maxp1);
+    tag_reduce_kernel<kTilesSmall, kBlocksSmall><<<grid, kReduceThreads, prep_smem, st>>>(
+        tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1, stream_blocks, prep);
   else
-    tag_reduce_kernel<kTilesLarge, kBlocksLarge><<<static_cast<unsigned>(blocks), kReduceThreads,
-                                                   0, st>>>(tags, offsets, n_traj, n_tokens,
-                                                            ws.sumv, ws.cnt, ws.maxp1);
+    tag_reduce_kernel<kTilesLarge, kBlocksLarge><<<grid, kReduceThreads, prep_smem, st>>>(
+        tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1, stream_blocks, prep);
   PACE_TRY(last_launch_status());
   if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
   return PACE_OK;
@@ -681,7 +715,7 @@ extern "C" pace_status pace_stale_k(const int32_t* tags, const int64_t* offsets,
   ScoreWs ws = carve_score_ws(cv, n_traj);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
   cudaStream_t st = as_stream(stream);
-  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, st));
+  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, WindowPrep{}, st));
   const int threads = 256;
   stale_k_kernel<<<static_cast<unsigned>((n_traj + threads - 1) / threads), threads, 0, st>>>(
       offsets, ws.sumv, ws.cnt, ws.maxp1, n_traj, n_tokens, trainer_version, k_max, kbar,
@@ -736,19 +770,22 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
 
   cudaStream_t st = as_stream(stream);
-  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, st));
   const bool window_ready = window_len > 0 && window_len >= params->min_obs;
-  // Sorting W and tabulating F is one extra launch that pays off only on large
-  // pools; smaller ones count against the raw window (the same bits either way).
+  // With the sorted window and the F table the finalisation takes one binary
+  // search and one table read per trajectory; their preparation runs inside the
+  // tag reduction's launch.  Small pools count against the raw window instead
+  // (the same bits either way).
   const bool use_table = window_ready && n_traj >= kTableMinTraj;
+  WindowPrep prep{};
   if (use_table) {
-    const unsigned prep_blocks = 1u + static_cast<unsigned>((window_len + 1 + kFPerBlock - 1) /
-                                                            kFPerBlock);
-    window_prep_kernel<<<prep_blocks, 1024, 0, st>>>(window, static_cast<int>(window_len),
-                                                     params->gamma, wws.sorted, wws.f_table,
-                                                     status_dev);
-    PACE_TRY(last_launch_status());
+    prep.window = window;
+    prep.n = static_cast<int>(window_len);
+    prep.gamma = params->gamma;
+    prep.sorted = wws.sorted;
+    prep.f_table = wws.f_table;
+    prep.status = status_dev;
   }
+  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, prep, st));
   FinalizeArgs a;
   a.offsets = offsets;
   a.c_version = c_version;
