@@ -825,7 +825,11 @@ def run_case(args):
         gen = torch.Generator(device=device)
         gen.manual_seed(103)
         targets = torch.randint(0, V, (rows,), generator=gen, device=device, dtype=torch.int32)
-        b = pace.make_batch(torch.tensor([0, rows], dtype=torch.int64, device=device), rows)
+        # --case-mask: every row in the loss, but read through the compacted row
+        # index (the path masked and rejected rows take) instead of TMA boxes
+        mask = torch.ones(rows, dtype=torch.uint8, device=device) if args.case_mask else None
+        b = pace.make_batch(torch.tensor([0, rows], dtype=torch.int64, device=device), rows,
+                            mask=mask)
         lp = torch.empty(rows, dtype=torch.float32, device=device)
         ws = pace.workspace(pace.token_logprob_workspace_size(rows, 1, H, V), device)
         status = pace.new_status(device)
@@ -840,7 +844,7 @@ def run_case(args):
         ms = statistics.mean(a.elapsed_time(z) for a, z in evs)
         tf = 2.0 * rows * H * V / (ms / 1e3) / 1e12
         print(json.dumps({"case": "lmhead", "workload": args.case_workload, "rows": rows, "H": H,
-                          "V": V, "kernel_ms": ms,
+                          "V": V, "rows_by_index": bool(args.case_mask), "kernel_ms": ms,
                           "tflops": tf, "frac_burst": tf / peaks["bf16_tflops"]}), flush=True)
     elif args.case == "lmhead_bwd":
         spec = workloads.SPECS[WORKLOAD]
@@ -940,6 +944,8 @@ def main():
                     default=None,
                     help="time one kernel on a small case (profiler captures)")
     ap.add_argument("--case-rows", type=int, default=4864)
+    ap.add_argument("--case-mask", action="store_true",
+                    help="lmhead case: pass a mask of ones, so rows are read by index")
     ap.add_argument("--case-workload", default=WORKLOAD, choices=["math7b", "multiturn", "moe"])
     ap.add_argument("--case-traj", type=int, default=16384)
     ap.add_argument("--case-units", type=int, default=131072)

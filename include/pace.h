@@ -347,8 +347,11 @@ PACE_API pace_status pace_group_advantages(const float* reward, const uint8_t* s
  *              advantages (pace_group_advantages), the per-token clipped terms
  *              and the aggregated loss exactly as pace_surrogate_loss does,
  *              fused after the log-probs.
- * Rows in the loss are first compacted (their hidden states gathered into the
- * workspace) so the tensor cores only see rows that count. */
+ * Rows in the loss are first compacted into a list of row indices, and the LM
+ * head reads their hidden states through it, so the tensor cores only see rows
+ * that count; the hidden states are never copied (the workspace holds the
+ * index list and per-row partials, not rows: its size does not depend on
+ * hidden_size). */
 PACE_API pace_status pace_token_logprob(const PaceBatch* batch, const void* hidden, const void* w_vocab,
                                const int32_t* targets, int32_t hidden_size, int32_t vocab_size,
                                float temperature, float* logprob, float* lse,

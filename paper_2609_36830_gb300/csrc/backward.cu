@@ -20,8 +20,8 @@
 // even CTA's barrier; warp 1 of the even CTA issues tcgen05.mma.cta_group::2
 // (M 256 = 128 rows per CTA, N 256 = 128 columns from each CTA, K 16; the
 // instruction descriptor's major bits select K- or MN-major operand layouts);
-// warps 2-5 of each CTA drain its two TMEM accumulators.  No operand is
-// multicast.  Every wait is bounded.
+// warps 2-5 of each CTA drain its two TMEM accumulators.  Every CTA loads only
+// its own tiles.  Every wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>

@@ -4,11 +4,22 @@
 //
 // lmhead_lse_kernel (sm_103a, persistent CTA pairs, one CTA per SM, 192
 // threads, warp-specialised, tcgen05 on the pair):
-//   warp 0 / lane 0   TMA producer, in both CTAs: per K step the CTA's own
+//   warp 0            TMA producer, in both CTAs: per K step the CTA's own
 //                     128x64 hidden tile and its own half (128x64) of the pair's
 //                     256x64 vocabulary tile, into its own 4-stage shared-memory
 //                     ring (128-byte swizzle); the transaction bytes of both
-//                     CTAs complete on the even CTA's mbarrier.
+//                     CTAs complete on the even CTA's mbarrier.  Contiguous
+//                     rows: lane 0 loads both as boxes.  Rows in the loss a
+//                     subset (mask, rejected groups, fewer than 128 rows): the
+//                     hidden tile is read straight from the caller's
+//                     hidden-state tensor through the compact-row index.  Per
+//                     work item the warp splits the block's 128 rows into runs
+//                     of consecutive source rows (plan_block_loads) and each
+//                     run into boxes of 2^j rows; per K step one lane per box
+//                     issues its load (one box for a block inside a response).
+//                     A block of more than 32 boxes is fetched by four-row TMA
+//                     gathers (tile::gather4), one per lane.  No copy of the
+//                     rows is made.
 //   warp 1 / lane 0   MMA issuer, even CTA only: tcgen05.mma.cta_group::2
 //                     kind::f16 (bf16 x bf16 -> fp32), M=256 (128 rows from each
 //                     CTA), N=256 (128 vocabulary rows from each CTA), K=16 per
@@ -67,7 +78,16 @@ constexpr uint32_t kStageB = BN / CLUSTER * BK * 2;  // 16 KB: this CTA's half o
 constexpr uint32_t kStageBytes = kStageA + kStageB;
 constexpr uint32_t kTmemCols = 2 * BN;          // two fp32 accumulators of 256 columns
 constexpr uint32_t kIdesc = idesc_bf16_f32(CLUSTER * BM, BN);
-constexpr size_t kSmemBytes = 1024 /* alignment slack */ + STAGES * kStageBytes + 256;
+// after the stages: barriers and flags (256 bytes), then for rows read by
+// index the block's source rows (int32 [128]) and its planned loads (int2 [128])
+constexpr uint32_t kMiscBytes = 256 + BM * 4 + BM * 8;
+constexpr size_t kSmemBytes = 1024 /* alignment slack */ + STAGES * kStageBytes + kMiscBytes;
+// Tensor maps of the hidden states with boxes of 1, 2, 4, ..., 128 rows (64
+// columns, 128-byte swizzle): a contiguous run of rows loads as a few boxes.
+constexpr int kBoxLevels = 8;
+struct AMaps {
+  CUtensorMap box[kBoxLevels];  // box[j]: 2^j rows
+};
 constexpr int kMaxSplits = 8;
 
 // Number of vocabulary splits S for row_pairs row pairs on n_clusters persistent
@@ -116,6 +136,8 @@ struct LmArgs {
   float scale_log2;             // log2(e) / temperature
   const int32_t* targets;
   const int32_t* rowidx;        // compact row -> original row, or null (identity)
+  int32_t gather;               // 1: rows read by index (rowidx), in planned boxes
+  int32_t max_level;            // largest box level no taller than the hidden-state tensor
   float* part_m;                // [rows_cap * kMaxSplits], row r's splits at r * S
   float* part_s;
   float* tgt_logit;             // [rows_cap]
@@ -142,9 +164,70 @@ struct ItemCursor {
   __device__ void next() { item += n_clusters; }
 };
 
+// The loads of one 128-row block whose rows are read by index.  Block row r is
+// compact row row0 + r; its source row is rowidx[row0 + r] while that is below
+// n_valid, and the rows past the end (loaded, never written back) take source
+// rows 0, 1, 2, ... so they form one run.  A run is a maximal stretch of block
+// rows with consecutive source rows; a run of L rows is loaded as one box per
+// set bit of L (2^j rows, largest first, j at most max_level).  Writes the
+// source rows to row_src[BM], the boxes to piece[] as (first source row, first
+// block row | level << 8) and their number to *n_pieces.  All 32 lanes call it.
+__device__ void plan_block_loads(const int32_t* __restrict__ rowidx, int64_t row0,
+                                 int64_t n_valid, int max_level, int lane, int32_t* row_src,
+                                 int2* piece, volatile int* n_pieces) {
+  const int64_t left = n_valid - row0;
+  const int r_inv = left <= 0 ? 0 : (left >= BM ? BM : static_cast<int>(left));
+  int32_t v[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int r = 32 * j + lane;
+    v[j] = r < r_inv ? rowidx[row0 + r] : r - r_inv;
+  }
+  uint32_t starts[4];
+  uint32_t carry = 0;  // source row of the previous word's last row
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    uint32_t prev = __shfl_up_sync(0xffffffffu, static_cast<uint32_t>(v[j]), 1);
+    if (lane == 0) prev = carry;
+    const bool st = (j == 0 && lane == 0) || static_cast<uint32_t>(v[j]) != prev + 1u;
+    starts[j] = __ballot_sync(0xffffffffu, st);
+    carry = __shfl_sync(0xffffffffu, static_cast<uint32_t>(v[j]), 31);
+    row_src[32 * j + lane] = v[j];
+  }
+  __syncwarp();
+  if (lane == 0) {
+    const uint64_t lo = starts[0] | (static_cast<uint64_t>(starts[1]) << 32);
+    const uint64_t hi = starts[2] | (static_cast<uint64_t>(starts[3]) << 32);
+    int n = 0, r = 0;
+    while (r < BM) {
+      const int q = r + 1;  // the run ends at the next start at or after q (BM: none)
+      const uint64_t m = q < 64 ? (lo & (~0ull << q)) : 0ull;
+      int e;
+      if (m) {
+        e = __ffsll(static_cast<long long>(m)) - 1;
+      } else {
+        const uint64_t m2 = q < 64 ? hi : (q < BM ? (hi & (~0ull << (q - 64))) : 0ull);
+        e = m2 ? 64 + __ffsll(static_cast<long long>(m2)) - 1 : BM;
+      }
+      int32_t s0 = row_src[r];
+      int len = e - r;
+      while (len > 0) {
+        int lev = 31 - __clz(len);
+        if (lev > max_level) lev = max_level;
+        piece[n++] = make_int2(s0, r | (lev << 8));
+        r += 1 << lev;
+        s0 += 1 << lev;
+        len -= 1 << lev;
+      }
+    }
+    *n_pieces = n;
+  }
+  __syncwarp();
+}
+
 __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
-    lmhead_lse_kernel(const __grid_constant__ CUtensorMap tm_a,
-                      const __grid_constant__ CUtensorMap tm_b, LmArgs p) {
+    lmhead_lse_kernel(const __grid_constant__ AMaps am, const __grid_constant__ CUtensorMap tm_b,
+                      LmArgs p) {
   extern __shared__ unsigned char smem_raw[];
   // the same offsets in both CTAs: the pair's MMA reads each CTA's operand
   // tiles at the addresses the even CTA's descriptors name
@@ -159,6 +242,9 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
   uint64_t* mma_done = tmem_empty + 2;       // [1]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* n_pieces = reinterpret_cast<volatile int*>(tmem_slot + 2);
+  int32_t* row_src = reinterpret_cast<int32_t*>(smem + STAGES * kStageBytes + 256);  // [BM]
+  int2* piece = reinterpret_cast<int2*>(row_src + BM);                            // [BM]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -207,10 +293,13 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
   };
 
   if (warp == 0) {
-    if (lane == 0) {
+    // rows by index (rows in the loss a subset, listed in rowidx): the whole
+    // warp produces; else lane 0 alone loads 128-row boxes
+    const bool gather = p.gather != 0;
+    if (lane == 0 || gather) {
       // ------------------------------------------------ TMA producer (both CTAs)
-      tma_prefetch_desc(&tm_a);
-      tma_prefetch_desc(&tm_b);
+      if (lane < kBoxLevels) tma_prefetch_desc(&am.box[lane]);
+      if (lane == 0) tma_prefetch_desc(&tm_b);
       const uint64_t pol = make_policy_evict_normal();
       uint32_t it = 0;
       bool ok = true;
@@ -218,11 +307,35 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
       for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next(), ++round) {
         const int64_t rp = c.item / n_splits;
         const int split = static_cast<int>(c.item % n_splits);
-        const int32_t row0 = static_cast<int32_t>((rp * CLUSTER + crank) * BM);
+        const int64_t row0 = (rp * CLUSTER + crank) * BM;
+        // rows by index: this lane's box (first source row, first block row,
+        // level), or on a scattered block its four rows for a gather
+        int32_t psrc = 0, g4[4] = {0, 0, 0, 0};
+        int pdst = 0, plev = -1;
+        bool scattered = false;
+        if (gather) {
+          plan_block_loads(p.rowidx, row0, n_valid, p.max_level, lane, row_src, piece, n_pieces);
+          const int n = *n_pieces;
+          scattered = n > 32;
+          if (!scattered) {
+            if (lane < n) {
+              const int2 pc = piece[lane];
+              psrc = pc.x;
+              pdst = pc.y & 0xff;
+              plev = pc.y >> 8;
+            }
+          } else {
+            // rows past the end gather row 0 (every gathered row exists)
+            const int64_t left = n_valid - row0;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) g4[j] = 4 * lane + j < left ? row_src[4 * lane + j] : 0;
+          }
+        }
         // every round before the last is full, so round k starts once all
         // clusters issued their round k-1 loads (the even CTA paces the pair)
-        if (leader && round > 0 && p.round_ctr)
+        if (leader && lane == 0 && round > 0 && p.round_ctr)
           wait_round(p.round_ctr, round * static_cast<unsigned>(n_clusters));
+        if (gather) __syncwarp();
         const int tile0 = split * tiles_per_split;
         const int tile1 = min(tile0 + tiles_per_split, p.n_vtiles);
         for (int t = tile0; t < tile1 && ok; ++t) {
@@ -230,32 +343,51 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
           for (int kb = 0; kb < nkb; ++kb, ++it) {
             const uint32_t s = it % STAGES;
             const uint32_t ph = (it / STAGES) & 1u;
-            if (!mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag)) {
+            bool got = mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag);
+            if (gather) got = __all_sync(0xffffffffu, got);  // one outcome for the warp
+            if (!got) {
               ok = false;
               break;
             }
             unsigned char* sa = stage_base + s * kStageBytes;
             unsigned char* sb = sa + kStageA;
             const uint32_t bar = cluster_addr(&full[s], 0);
-            if (leader) mbar_arrive_expect_tx(&full[s], CLUSTER * kStageBytes);
-            tma_load_2d_pair(sa, &tm_a, bar, kb * BK, row0, pol);
-            tma_load_2d_pair(sb, &tm_b, bar, kb * BK, nb, pol);
+            if (lane == 0) {
+              if (leader) mbar_arrive_expect_tx(&full[s], CLUSTER * kStageBytes);
+              if (!gather)
+                tma_load_2d_pair(sa, &am.box[kBoxLevels - 1], bar, kb * BK,
+                                 static_cast<int32_t>(row0), pol);
+              tma_load_2d_pair(sb, &tm_b, bar, kb * BK, nb, pol);
+            }
+            if (gather) {
+              if (!scattered) {
+                if (plev >= 0)
+                  tma_load_2d_pair(sa + pdst * (BK * 2), &am.box[plev], bar, kb * BK, psrc, pol);
+              } else {
+                tma_gather4_pair(sa + lane * 4 * (BK * 2), &am.box[0], bar, kb * BK, g4[0],
+                                 g4[1], g4[2], g4[3], pol);
+              }
+            }
           }
         }
-        if (leader && ok && p.round_ctr) atomicAdd(p.round_ctr, 1u);
+        if (leader && lane == 0 && ok && p.round_ctr) atomicAdd(p.round_ctr, 1u);
+        if (gather) __syncwarp();  // row_src and piece are rewritten for the next item
       }
-      if (!ok) give_up();
-      // Drain: every copy issued must have landed before the CTA exits.  The
-      // even CTA sees both CTAs' bytes on its full barriers; the odd CTA sees
-      // its stages consumed on its empty barriers.  After a timeout anywhere
-      // the waits are short: copies land in microseconds.
-      const uint64_t lim = *abort_flag ? 1000000ull : kWaitLimitNs;
-      for (uint32_t s = 0; s < STAGES && s < it; ++s) {
-        const uint32_t last = it - 1 - ((it - 1 - s) % STAGES);  // last index with stage s
-        if (leader)
-          mbar_wait_bounded(&full[s], (last / STAGES) & 1u, nullptr, lim);
-        else
-          mbar_wait_bounded(&empty[s], (last / STAGES) & 1u, nullptr, lim);
+      if (lane == 0) {
+        if (!ok) give_up();
+        // Drain: every copy issued must have landed before the CTA exits.  The
+        // even CTA sees both CTAs' bytes (all lanes' gathers included) on its
+        // full barriers; the odd CTA sees its stages consumed on its empty
+        // barriers.  After a timeout anywhere the waits are short: copies land
+        // in microseconds.
+        const uint64_t lim = *abort_flag ? 1000000ull : kWaitLimitNs;
+        for (uint32_t s = 0; s < STAGES && s < it; ++s) {
+          const uint32_t last = it - 1 - ((it - 1 - s) % STAGES);  // last index with stage s
+          if (leader)
+            mbar_wait_bounded(&full[s], (last / STAGES) & 1u, nullptr, lim);
+          else
+            mbar_wait_bounded(&empty[s], (last / STAGES) & 1u, nullptr, lim);
+        }
       }
     }
   } else if (warp == 1) {
@@ -473,13 +605,14 @@ pace_status lm_launch_info(LmLaunchInfo* out) {
 
 }  // namespace
 
-void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, bool compact,
+void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, bool dense_rows,
                  LmWs* w) {
   const int64_t rows_cap = n_rows > BM ? n_rows : BM;
   carve_compact_ws(cv, n_seq, n_rows, &w->cw);
   carve_surrogate_ws(cv, n_seq, &w->sw);
-  w->hidden_c = compact ? static_cast<void*>(cv.take<uint16_t>(static_cast<size_t>(rows_cap) * H))
-                        : nullptr;
+  w->hidden_c =
+      dense_rows ? static_cast<void*>(cv.take<uint16_t>(static_cast<size_t>(rows_cap) * H))
+                 : nullptr;
   w->part_m = cv.take<float>(static_cast<size_t>(rows_cap) * kMaxSplits);
   w->part_s = cv.take<float>(static_cast<size_t>(rows_cap) * kMaxSplits);
   w->tgt = cv.take<float>(static_cast<size_t>(rows_cap));
@@ -503,7 +636,7 @@ pace_status check_lm_args(const PaceBatch* batch, const void* hidden, const void
   return PACE_OK;
 }
 
-// Compaction, gather, fused LM head and merge: lp (and lse) for every row in
+// Compaction, fused LM head and merge: lp (and lse) for every row in
 // the batch's loss, 0 elsewhere.
 pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* w_vocab,
                         const int32_t* targets, int H, int V, float temperature, float* logprob,
@@ -514,22 +647,29 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
     PACE_TRY_CUDA(cudaMemsetAsync(logprob, 0, static_cast<size_t>(n_rows) * sizeof(float), st));
     if (lse) PACE_TRY_CUDA(cudaMemsetAsync(lse, 0, static_cast<size_t>(n_rows) * sizeof(float), st));
   }
-  const void* a_ptr = hidden;
   const long long* n_valid_dev = nullptr;
   const int32_t* rowidx = nullptr;
   int64_t rows_cap = n_rows;
   if (compact) {
+    // the LM head reads the rows in the loss through rowidx (no dense copy)
     PACE_TRY(run_compaction(batch, ws.cw, status_dev, st));
-    PACE_TRY(run_gather(hidden, H, n_rows, ws.cw, ws.hidden_c, st));
-    a_ptr = ws.hidden_c;
     n_valid_dev = ws.cw.total;
     rowidx = ws.cw.rowidx;
     rows_cap = n_rows > BM ? n_rows : BM;
   }
   if (n_rows == 0) return PACE_OK;
   const int n_vtiles = (V + BN - 1) / BN;
-  CUtensorMap tm_a, tm_b;
-  PACE_TRY(encode_bf16_2d(&tm_a, a_ptr, rows_cap, H, H, BK, BM));
+  AMaps am;
+  CUtensorMap tm_b;
+  // boxes of 2^j hidden rows for j up to the tensor's height (at most 128);
+  // taller levels repeat the tallest valid map and are never used
+  int max_level = 0;
+  while (max_level + 1 < kBoxLevels && (int64_t{1} << (max_level + 1)) <= n_rows) ++max_level;
+  if (!compact && max_level != kBoxLevels - 1) return PACE_ERR_INVALID_ARG;  // n_rows >= 128
+  for (int j = 0; j < kBoxLevels; ++j) {
+    if (j <= max_level) PACE_TRY(encode_bf16_2d(&am.box[j], hidden, n_rows, H, H, BK, 1 << j));
+    else am.box[j] = am.box[max_level];
+  }
   PACE_TRY(encode_bf16_2d(&tm_b, w_vocab, V, H, H, BK, BN / CLUSTER));  // one CTA's half tile
   LmLaunchInfo li;
   PACE_TRY(lm_launch_info(&li));
@@ -543,6 +683,8 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   a.scale_log2 = 1.4426950408889634f / temperature;
   a.targets = targets;
   a.rowidx = rowidx;
+  a.gather = compact ? 1 : 0;
+  a.max_level = max_level;
   a.part_m = ws.part_m;
   a.part_s = ws.part_s;
   a.tgt_logit = ws.tgt;
@@ -556,7 +698,7 @@ pace_status run_logprob(const PaceBatch* batch, const void* hidden, const void* 
   PACE_TRY_CUDA(cudaMemsetAsync(ws.round_ctr, 0, sizeof(unsigned), st));
   const ProfileEvents& pe = profile_events(PACE_PROFILE_LMHEAD);
   if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
-  lmhead_lse_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tm_a, tm_b, a);
+  lmhead_lse_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(am, tm_b, a);
   PACE_TRY(last_launch_status());
   if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
   int64_t mblocks = (rows_cap + 255) / 256;
@@ -579,7 +721,7 @@ extern "C" size_t pace_token_logprob_workspace_size(int64_t n_rows, int64_t n_se
   if (n_rows < 0 || n_seq < 0 || hidden_size <= 0 || vocab_size <= 0) return 0;
   Carver cv;
   LmWs w;
-  carve_lm_ws(cv, n_rows, n_seq, hidden_size, true, &w);
+  carve_lm_ws(cv, n_rows, n_seq, hidden_size, false, &w);
   return cv.used;
 }
 
@@ -596,8 +738,7 @@ extern "C" pace_status pace_token_logprob(const PaceBatch* batch, const void* hi
   if (!workspace || !aligned(workspace, 256)) return PACE_ERR_WORKSPACE;
   Carver cv(workspace, workspace_bytes);
   LmWs ws;
-  carve_lm_ws(cv, batch->n_rows, batch->n_seq, hidden_size,
-              lm_needs_compaction(batch), &ws);
+  carve_lm_ws(cv, batch->n_rows, batch->n_seq, hidden_size, false, &ws);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
   cudaStream_t st = as_stream(stream);
   PACE_TRY(run_logprob(batch, hidden, w_vocab, targets, hidden_size, vocab_size, temperature,

@@ -245,6 +245,26 @@ __device__ __forceinline__ void tma_load_2d_pair(void* smem_dst, const void* des
       : "memory");
 }
 
+// Four whole rows (r0..r3) of a 2-D tensor map whose box is one row high,
+// starting at column x, into this CTA's shared memory at smem_dst, one row
+// after the other; the transaction bytes (4 box rows) complete on the mbarrier
+// at cluster address bar_caddr, as tma_load_2d_pair's do.  With the 128-byte
+// swizzle, each row's 16-byte chunks land at the positions their shared-memory
+// address selects, so four gathers into consecutive 512-byte slices build the
+// same tile as one box of 4 n rows.
+__device__ __forceinline__ void tma_gather4_pair(void* smem_dst, const void* desc,
+                                                 uint32_t bar_caddr, int32_t x, int32_t r0,
+                                                 int32_t r1, int32_t r2, int32_t r3,
+                                                 uint64_t cache_hint) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+      ".cta_group::2.L2::cache_hint [%0], [%1, {%3, %4, %5, %6, %7}], [%2], %8;" ::"r"(
+          smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(desc)), "r"(bar_caddr), "r"(x), "r"(r0), "r"(r1), "r"(r2),
+      "r"(r3), "l"(cache_hint)
+      : "memory");
+}
+
 // ---- tcgen05 on CTA pairs (5th-generation tensor cores, accumulators in
 // tensor memory).  Every tcgen05 instruction of a kernel names the same CTA
 // group; the kernels here all run on pairs (cta_group::2): one MMA of

@@ -23,7 +23,8 @@ struct CompactWs {
 struct LmWs {
   CompactWs cw;
   SurrogateWs sw;
-  void* hidden_c;  // gathered rows [max(n_rows, 128)][H] (null when no compaction)
+  void* hidden_c;  // dense copy of the rows in the loss [max(n_rows, 128)][H] (backward
+                   // only; null for the forward, whose LM head reads rows by index)
   float* part_m;
   float* part_s;
   float* tgt;
@@ -33,7 +34,7 @@ struct LmWs {
 void carve_surrogate_ws(Carver& cv, int64_t n_seq, SurrogateWs* w);
 pace_status launch_group_adv(const float* reward, const uint8_t* accepted, int64_t n_seq, int G,
                              float eps, int unbiased, float* adv, cudaStream_t st);
-void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, bool compact,
+void carve_lm_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, bool dense_rows,
                  LmWs* w);
 bool lm_needs_compaction(const PaceBatch* b);
 pace_status check_lm_args(const PaceBatch* batch, const void* hidden, const void* w_vocab,

@@ -88,7 +88,7 @@ struct PrefixWs {
 };
 
 void carve_prefix_ws(Carver& cv, int64_t n_rows, int64_t n_seq, int H, PrefixWs* w) {
-  carve_lm_ws(cv, n_rows, n_seq, H, true, &w->lm);
+  carve_lm_ws(cv, n_rows, n_seq, H, false, &w->lm);
   w->mask_c = cv.take<uint8_t>(n_rows > 0 ? n_rows : 1);
   w->n_elig = cv.take<long long>(n_seq > 0 ? n_seq : 1);
   w->logprob = cv.take<float>(n_rows > 0 ? n_rows : 1);

@@ -62,6 +62,32 @@ def test_small_shapes_all_rows(rows, H, V, masked):
     assert (lp[~sel] == 0).all() and (lse[~sel] == 0).all()
 
 
+@pytest.mark.parametrize("rows,H,V,max_run", [(3000, 256, 2048, 300), (2500, 128, 1000, 9),
+                                              (100, 64, 700, 40), (7, 64, 256, 3)])
+def test_masks_of_runs(rows, H, V, max_run):
+    """Rows in the loss as runs of random length (the shape prompt masks and
+    rejected groups give): the LM head loads each run of consecutive rows as
+    boxes of 2^j rows, or gathers a block of scattered rows, and every row in
+    the loss must still match the oracle."""
+    rng = np.random.default_rng(rows + max_run)
+    m = np.zeros(rows, np.uint8)
+    pos = 0
+    while pos < rows:
+        n = int(rng.integers(1, max_run + 1))
+        m[pos:pos + n] = rng.random() < 0.7
+        pos += n
+    hb = workloads.bf16_normal_host((rows, H), 1.0, rows + 5 * H)
+    wb = workloads.bf16_normal_host((V, H), 1.0 / math.sqrt(H) * 2.0, V + 3 * H)
+    y = rng.integers(0, V, size=rows).astype(np.int32)
+    lp, lse = _run(bf16_dev(hb), bf16_dev(wb), to_dev(y), mask=to_dev(m))
+    st, olp, olse = oracle.token_logprob(hb, wb, y)
+    assert st == 0
+    sel = m.astype(bool)
+    assert np.abs(lp[sel] - olp[sel]).max(initial=0) <= TOL
+    assert np.abs(lse[sel] - olse[sel]).max(initial=0) <= TOL
+    assert (lp[~sel] == 0).all() and (lse[~sel] == 0).all()
+
+
 def test_vocab_smaller_than_one_tile():
     rng = np.random.default_rng(1)
     rows, H, V = 200, 64, 100
