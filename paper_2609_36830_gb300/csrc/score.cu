@@ -5,7 +5,7 @@
 //                       bound): per trajectory the count T of policy tokens,
 //                       the exact integer sum of their tags and the largest
 //                       tag (+1, for the Lemma 1 premise check).
-//                       On pools of 32k trajectories and more the same launch
+//                       On pools of 8k trajectories and more the same launch
 //                       also prepares the prefix-score window (extra blocks
 //                       after the streaming ones, run in its tail): one sorts W,
 //                       the others tabulate F = phi(count / |W|) (Eqs. 9-10)
@@ -37,7 +37,7 @@ constexpr int kTilesLarge = 8, kBlocksLarge = 2;
 constexpr int kTilesSmall = 4, kBlocksSmall = 3;
 constexpr int64_t kSmallPoolTokens = int64_t(1) << 27;
 constexpr int kMaxWindow = 4096;
-constexpr int64_t kTableMinTraj = 32768;  // pools from this size sort W and tabulate F
+constexpr int64_t kTableMinTraj = 8192;  // pools from this size sort W and tabulate F
 
 __device__ __forceinline__ int4 ld_stream_v4(const int32_t* p) {
   int4 v;
