@@ -45,13 +45,15 @@ WORKLOAD = "moe"
 OTHER_WORKLOADS = ("math7b", "multiturn")
 PREFIX_WORKLOAD = "math7b"  # prefix rescoring and the backward are timed on the 7B math pool
 # DRAM bytes (read + written) per row in the loss of the LM-head kernel, by (workload,
-# vocabulary splits), from one-pass ncu captures (dram__bytes_read.sum + dram__bytes_write.sum)
-# of one launch of the current kernel at this bench's size (3,958,414 rows of the MoE-shaped
-# head): 526.726 GB + 191.1 MB with 4 splits, 296.312 GB + 126.1 MB with 2.  Emptied whenever
-# the kernel changes, until it is captured again.  The tag reduction's per tag: 14.0656 GB
-# read + 19.8 MB written for the 3.5023 G tags of the 1M sweep pool.
-LMHEAD_DRAM_BYTES_PER_ROW = {("moe", 4): (526726449920 + 191105792) / 3958414,
-                             ("moe", 2): (296312474368 + 126139136) / 3958414}
+# vocabulary splits), from a one-pass ncu capture (dram__bytes_read.sum +
+# dram__bytes_write.sum) of one wave of the current kernel reading rows by index: 19,456 rows
+# of the MoE-shaped head with 4 splits, 2.575841 GB read + 4.0 MB written.  With 4 splits
+# every round of items reads the vocabulary once, so the bytes grow with the rows (a full
+# 3,958,414-row launch of the previous kernel read 133.1 KB per row, this wave 132.6 KB).
+# With 2 splits a single wave is not proportional to a long launch, so no figure is given.
+# Emptied whenever the kernel changes, until it is captured again.  The tag reduction's per
+# tag: 14.0656 GB read + 19.8 MB written for the 3.5023 G tags of the 1M sweep pool.
+LMHEAD_DRAM_BYTES_PER_ROW = {("moe", 4): (2575841024 + 4003584) / 19456}
 TAG_REDUCE_DRAM_BYTES_PER_TAG = (14065824512 + 19798528) / 3502330341
 SWEEP_N = 1048576
 SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)
@@ -755,8 +757,9 @@ def run_gpu(args):
                          "flops_per_launch": flops,
                          "traffic": traffic * M if traffic else None,
                          "traffic_note": "dram read+write bytes per launch: bytes per row in the "
-                                         "loss from a one-pass ncu capture of the current kernel, "
-                                         "times the rows of this launch"},
+                                         "loss from a one-pass ncu capture of one wave (19,456 "
+                                         "rows, 4 splits) of the current kernel, times the rows "
+                                         "of this launch (null unless 4 splits were used)"},
             "cpu_baseline": cpu,
             "e2e": {"value": job_rows / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e_ms},
