@@ -75,15 +75,25 @@ constexpr int CLUSTER = 2;                      // the CTA pair of one 2-CTA MMA
 constexpr int kThreads = 192;
 constexpr uint32_t kStageA = BM * BK * 2;       // 16 KB: this CTA's 128 hidden rows
 constexpr uint32_t kStageB = BN / CLUSTER * BK * 2;  // 16 KB: this CTA's half of the vocabulary tile
-constexpr uint32_t kStageBytes = kStageA + kStageB;
 constexpr uint32_t kTmemCols = 2 * BN;          // two fp32 accumulators of 256 columns
 constexpr uint32_t kIdesc = idesc_bf16_f32(CLUSTER * BM, BN);
-// after the stages: barriers and flags (256 bytes), then for rows read by
-// index the block's source rows (int32 [128]) and its planned loads (int2 [128])
+// Shared memory: the hidden tiles, each with a 16 KB spill region before and
+// after it (shared by neighbours: spill | A0 | spill | A1 | ... | A3 | spill),
+// so a 128-row box may start up to 127 rows before or after its tile's first
+// row; then the vocabulary tiles; then barriers and flags (256 bytes) and, for
+// rows read by index, the block's source rows (int32 [128]) and its planned
+// loads (int2 [128]).
+constexpr uint32_t kSpill = kStageA;
+constexpr uint32_t kARegion = kSpill + STAGES * (kStageA + kSpill);
 constexpr uint32_t kMiscBytes = 256 + BM * 4 + BM * 8;
-constexpr size_t kSmemBytes = 1024 /* alignment slack */ + STAGES * kStageBytes + kMiscBytes;
+constexpr size_t kSmemBytes =
+    1024 /* alignment slack */ + kARegion + STAGES * kStageB + kMiscBytes;
+__host__ __device__ constexpr uint32_t a_tile_off(uint32_t s) {
+  return kSpill + s * (kStageA + kSpill);
+}
+__host__ __device__ constexpr uint32_t b_tile_off(uint32_t s) { return kARegion + s * kStageB; }
 // Tensor maps of the hidden states with boxes of 1, 2, 4, ..., 128 rows (64
-// columns, 128-byte swizzle): a contiguous run of rows loads as a few boxes.
+// columns, 128-byte swizzle).
 constexpr int kBoxLevels = 8;
 struct AMaps {
   CUtensorMap box[kBoxLevels];  // box[j]: 2^j rows
@@ -166,61 +176,86 @@ struct ItemCursor {
 
 // The loads of one 128-row block whose rows are read by index.  Block row r is
 // compact row row0 + r; its source row is rowidx[row0 + r] while that is below
-// n_valid, and the rows past the end (loaded, never written back) take source
-// rows 0, 1, 2, ... so they form one run.  A run is a maximal stretch of block
-// rows with consecutive source rows; a run of L rows is loaded as one box per
-// set bit of L (2^j rows, largest first, j at most max_level).  Writes the
-// source rows to row_src[BM], the boxes to piece[] as (first source row, first
-// block row | level << 8) and their number to *n_pieces.  All 32 lanes call it.
+// n_valid.  A run is a maximal stretch of block rows with consecutive source
+// rows; the rows past n_valid (loaded, never written back) belong to the last
+// run.  With 128-row boxes available (max_level 7), a block of one run is one
+// box; of several runs, the first run is one box that ends at the run's end
+// (its earlier rows land in the spill region before the tile), the last run one
+// box that starts at the run's start (its later rows land in the spill region
+// after the tile), and a run in between one box per set bit of its length,
+// largest first.  Boxes never overlap inside the tile.  Without 128-row boxes
+// (a hidden-state tensor of fewer than 128 rows) every run is split by the set
+// bits of its length.  Writes the source rows to row_src[BM], the boxes to
+// piece[] as (first source row, (first block row + 128) | level << 9), their
+// number to plan[0] and their bytes per K step to plan[1].  All 32 lanes call
+// it.
 __device__ void plan_block_loads(const int32_t* __restrict__ rowidx, int64_t row0,
                                  int64_t n_valid, int max_level, int lane, int32_t* row_src,
-                                 int2* piece, volatile int* n_pieces) {
+                                 int2* piece, volatile int* plan) {
   const int64_t left = n_valid - row0;
   const int r_inv = left <= 0 ? 0 : (left >= BM ? BM : static_cast<int>(left));
   int32_t v[4];
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
     const int r = 32 * j + lane;
-    v[j] = r < r_inv ? rowidx[row0 + r] : r - r_inv;
+    v[j] = r < r_inv ? rowidx[row0 + r] : 0;
   }
   uint32_t starts[4];
   uint32_t carry = 0;  // source row of the previous word's last row
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
+    const int r = 32 * j + lane;
     uint32_t prev = __shfl_up_sync(0xffffffffu, static_cast<uint32_t>(v[j]), 1);
     if (lane == 0) prev = carry;
-    const bool st = (j == 0 && lane == 0) || static_cast<uint32_t>(v[j]) != prev + 1u;
+    const bool st = r == 0 || (r < r_inv && static_cast<uint32_t>(v[j]) != prev + 1u);
     starts[j] = __ballot_sync(0xffffffffu, st);
     carry = __shfl_sync(0xffffffffu, static_cast<uint32_t>(v[j]), 31);
-    row_src[32 * j + lane] = v[j];
+    row_src[r] = v[j];
   }
   __syncwarp();
   if (lane == 0) {
     const uint64_t lo = starts[0] | (static_cast<uint64_t>(starts[1]) << 32);
     const uint64_t hi = starts[2] | (static_cast<uint64_t>(starts[3]) << 32);
-    int n = 0, r = 0;
+    const int m = __popcll(lo) + __popcll(hi);  // runs in the block
+    const bool full_boxes = max_level == kBoxLevels - 1;
+    int n = 0, k = 0, r = 0;
+    uint32_t rows = 0;
     while (r < BM) {
       const int q = r + 1;  // the run ends at the next start at or after q (BM: none)
-      const uint64_t m = q < 64 ? (lo & (~0ull << q)) : 0ull;
+      const uint64_t mlo = q < 64 ? (lo & (~0ull << q)) : 0ull;
       int e;
-      if (m) {
-        e = __ffsll(static_cast<long long>(m)) - 1;
+      if (mlo) {
+        e = __ffsll(static_cast<long long>(mlo)) - 1;
       } else {
-        const uint64_t m2 = q < 64 ? hi : (q < BM ? (hi & (~0ull << (q - 64))) : 0ull);
-        e = m2 ? 64 + __ffsll(static_cast<long long>(m2)) - 1 : BM;
+        const uint64_t mhi = q < 64 ? hi : (q < BM ? (hi & (~0ull << (q - 64))) : 0ull);
+        e = mhi ? 64 + __ffsll(static_cast<long long>(mhi)) - 1 : BM;
       }
-      int32_t s0 = row_src[r];
-      int len = e - r;
-      while (len > 0) {
-        int lev = 31 - __clz(len);
-        if (lev > max_level) lev = max_level;
-        piece[n++] = make_int2(s0, r | (lev << 8));
-        r += 1 << lev;
-        s0 += 1 << lev;
-        len -= 1 << lev;
+      const int32_t s0 = row_src[r];
+      const int len = e - r;
+      if (full_boxes && k == 0 && m > 1) {  // first of several: ends at the run's end
+        piece[n++] = make_int2(s0 + len - BM, (len - BM + BM) | ((kBoxLevels - 1) << 9));
+        rows += BM;
+      } else if (full_boxes && k == m - 1) {  // last (or only): starts at the run's start
+        piece[n++] = make_int2(s0, (r + BM) | ((kBoxLevels - 1) << 9));
+        rows += BM;
+      } else {
+        int at = r, rem = len;
+        int32_t src = s0;
+        while (rem > 0) {
+          int lev = 31 - __clz(rem);
+          if (lev > max_level) lev = max_level;
+          piece[n++] = make_int2(src, (at + BM) | (lev << 9));
+          rows += 1u << lev;
+          at += 1 << lev;
+          src += 1 << lev;
+          rem -= 1 << lev;
+        }
       }
+      r = e;
+      ++k;
     }
-    *n_pieces = n;
+    plan[0] = n;
+    plan[1] = static_cast<int>(rows * (BK * 2));
   }
   __syncwarp();
 }
@@ -233,8 +268,7 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
   // tiles at the addresses the even CTA's descriptors name
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  unsigned char* stage_base = smem;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kARegion + STAGES * kStageB);
   uint64_t* full = bars;                     // [STAGES] even CTA: both CTAs' tiles landed
   uint64_t* empty = bars + STAGES;           // [STAGES] the pair's MMAs are done with the stage
   uint64_t* tmem_full = bars + 2 * STAGES;   // [2] this CTA's accumulator is ready
@@ -242,8 +276,8 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
   uint64_t* mma_done = tmem_empty + 2;       // [1]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  volatile int* n_pieces = reinterpret_cast<volatile int*>(tmem_slot + 2);
-  int32_t* row_src = reinterpret_cast<int32_t*>(smem + STAGES * kStageBytes + 256);  // [BM]
+  volatile int* plan = reinterpret_cast<volatile int*>(tmem_slot + 2);  // [2] boxes, A bytes
+  int32_t* row_src = reinterpret_cast<int32_t*>(reinterpret_cast<unsigned char*>(bars) + 256);
   int2* piece = reinterpret_cast<int2*>(row_src + BM);                            // [BM]
 
   const int warp = threadIdx.x >> 5;
@@ -264,7 +298,7 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&full[s], 1);
+      mbar_init(&full[s], CLUSTER);  // each CTA's producer arrives with its bytes
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -313,16 +347,18 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
         int32_t psrc = 0, g4[4] = {0, 0, 0, 0};
         int pdst = 0, plev = -1;
         bool scattered = false;
+        uint32_t a_bytes = kStageA;  // this CTA's hidden-tile bytes per K step
         if (gather) {
-          plan_block_loads(p.rowidx, row0, n_valid, p.max_level, lane, row_src, piece, n_pieces);
-          const int n = *n_pieces;
+          plan_block_loads(p.rowidx, row0, n_valid, p.max_level, lane, row_src, piece, plan);
+          const int n = plan[0];
           scattered = n > 32;
           if (!scattered) {
+            a_bytes = static_cast<uint32_t>(plan[1]);
             if (lane < n) {
               const int2 pc = piece[lane];
               psrc = pc.x;
-              pdst = pc.y & 0xff;
-              plev = pc.y >> 8;
+              pdst = (pc.y & 0x1ff) - BM;  // first block row, -127..127
+              plev = pc.y >> 9;
             }
           } else {
             // rows past the end gather row 0 (every gathered row exists)
@@ -349,11 +385,16 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
               ok = false;
               break;
             }
-            unsigned char* sa = stage_base + s * kStageBytes;
-            unsigned char* sb = sa + kStageA;
+            unsigned char* sa = smem + a_tile_off(s);
+            unsigned char* sb = smem + b_tile_off(s);
             const uint32_t bar = cluster_addr(&full[s], 0);
             if (lane == 0) {
-              if (leader) mbar_arrive_expect_tx(&full[s], CLUSTER * kStageBytes);
+              // this CTA's bytes of the stage, announced with its arrival on the
+              // even CTA's barrier (which completes once both CTAs' bytes land)
+              if (leader)
+                mbar_arrive_expect_tx(&full[s], a_bytes + kStageB);
+              else
+                mbar_arrive_expect_tx_cluster(bar, a_bytes + kStageB);
               if (!gather)
                 tma_load_2d_pair(sa, &am.box[kBoxLevels - 1], bar, kb * BK,
                                  static_cast<int32_t>(row0), pol);
@@ -416,8 +457,8 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
-            const uint32_t sa = smem_u32(stage_base + s * kStageBytes);
-            const uint32_t sb = sa + kStageA;
+            const uint32_t sa = smem_u32(smem + a_tile_off(s));
+            const uint32_t sb = smem_u32(smem + b_tile_off(s));
 #pragma unroll
             for (int k = 0; k < BK / 16; ++k) {
               tc_mma_f16_pair(d_tmem, smem_desc_k128(sa + k * 32), smem_desc_k128(sb + k * 32),

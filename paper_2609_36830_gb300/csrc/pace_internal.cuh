@@ -174,6 +174,15 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_caddr) {
                : "memory");
 }
 
+// Arrive on the mbarrier at cluster address bar_caddr (this CTA's or a peer's)
+// and raise its expected transaction bytes by `bytes`, in one step.
+__device__ __forceinline__ void mbar_arrive_expect_tx_cluster(uint32_t bar_caddr, uint32_t bytes) {
+  asm volatile(
+      "mbarrier.arrive.expect_tx.shared::cluster.b64 _, [%0], %1;" ::"r"(bar_caddr),
+      "r"(bytes)
+      : "memory");
+}
+
 __device__ __forceinline__ void st_cluster_u32(uint32_t caddr, uint32_t v) {
   asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(caddr), "r"(v) : "memory");
 }
