@@ -178,17 +178,17 @@ struct ItemCursor {
 // compact row row0 + r; its source row is rowidx[row0 + r] while that is below
 // n_valid.  A run is a maximal stretch of block rows with consecutive source
 // rows; the rows past n_valid (loaded, never written back) belong to the last
-// run.  With 128-row boxes available (max_level 7), a block of one run is one
-// box; of several runs, the first run is one box that ends at the run's end
-// (its earlier rows land in the spill region before the tile), the last run one
-// box that starts at the run's start (its later rows land in the spill region
-// after the tile), and a run in between one box per set bit of its length,
-// largest first.  Boxes never overlap inside the tile.  Without 128-row boxes
-// (a hidden-state tensor of fewer than 128 rows) every run is split by the set
-// bits of its length.  Writes the source rows to row_src[BM], the boxes to
-// piece[] as (first source row, (first block row + 128) | level << 9), their
-// number to plan[0] and their bytes per K step to plan[1].  All 32 lanes call
-// it.
+// run.  A block of one run is loaded as one box per set bit of its length (one
+// 128-row box when the tensor has 128 rows or more).  Of several runs, the
+// first is one box of the smallest power of two rows that covers it, ending at
+// the run's end (its earlier rows land in the spill region before the tile),
+// the last one such box starting at the run's start (its later rows land in the
+// spill region after the tile), and a run in between one box per set bit of
+// its length, largest first.  Boxes never overlap inside the tile, and no box
+// is taller than 2^max_level rows (the tallest map the hidden-state tensor
+// allows).  Writes the source rows to row_src[BM], the boxes to piece[] as
+// (first source row, (first block row + 128) | level << 9), their number to
+// plan[0] and their bytes per K step to plan[1].  All 32 lanes call it.
 __device__ void plan_block_loads(const int32_t* __restrict__ rowidx, int64_t row0,
                                  int64_t n_valid, int max_level, int lane, int32_t* row_src,
                                  int2* piece, volatile int* plan) {
@@ -217,7 +217,6 @@ __device__ void plan_block_loads(const int32_t* __restrict__ rowidx, int64_t row
     const uint64_t lo = starts[0] | (static_cast<uint64_t>(starts[1]) << 32);
     const uint64_t hi = starts[2] | (static_cast<uint64_t>(starts[3]) << 32);
     const int m = __popcll(lo) + __popcll(hi);  // runs in the block
-    const bool full_boxes = max_level == kBoxLevels - 1;
     int n = 0, k = 0, r = 0;
     uint32_t rows = 0;
     while (r < BM) {
@@ -232,23 +231,25 @@ __device__ void plan_block_loads(const int32_t* __restrict__ rowidx, int64_t row
       }
       const int32_t s0 = row_src[r];
       const int len = e - r;
-      if (full_boxes && k == 0 && m > 1) {  // first of several: ends at the run's end
-        piece[n++] = make_int2(s0 + len - BM, (len - BM + BM) | ((kBoxLevels - 1) << 9));
-        rows += BM;
-      } else if (full_boxes && k == m - 1) {  // last (or only): starts at the run's start
-        piece[n++] = make_int2(s0, (r + BM) | ((kBoxLevels - 1) << 9));
-        rows += BM;
-      } else {
-        int at = r, rem = len;
+      const int cl = len <= 1 ? 0 : 32 - __clz(len - 1);  // smallest level that covers the run
+      if (m > 1 && (k == 0 || k == m - 1) && cl <= max_level) {
+        // first or last of several runs: one box of 2^cl rows, ending at the
+        // first run's end (spilling before the tile) or starting at the last
+        // run's start (spilling after it)
+        const int at = k == 0 ? len - (1 << cl) : r;
+        piece[n++] = make_int2(s0 + (at - r), (at + BM) | (cl << 9));
+        rows += 1u << cl;
+      } else {  // the only run, or one in between: one box per set bit of its length
+        int at = r, left_rows = len;
         int32_t src = s0;
-        while (rem > 0) {
-          int lev = 31 - __clz(rem);
+        while (left_rows > 0) {
+          int lev = 31 - __clz(left_rows);
           if (lev > max_level) lev = max_level;
           piece[n++] = make_int2(src, (at + BM) | (lev << 9));
           rows += 1u << lev;
           at += 1 << lev;
           src += 1 << lev;
-          rem -= 1 << lev;
+          left_rows -= 1 << lev;
         }
       }
       r = e;
