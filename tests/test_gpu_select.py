@@ -52,6 +52,24 @@ def test_select_k_matches_oracle(U, dist):
             _check_k(s, G, k)
 
 
+@pytest.mark.parametrize("U", [513, 1000, 2047, 4095, 4096, 4097])
+@pytest.mark.parametrize("dist", ["ties", "continuous", "ulps", "signed_wide"])
+def test_one_cta_pools(U, dist):
+    """One CTA holds the pool (G = 1) around the sizes where a cluster of one
+    CTA gives way to larger clusters: ids exact."""
+    rng = np.random.default_rng(7 * U + len(dist))
+    if dist == "ties":
+        s = rng.integers(0, 5, size=U).astype(np.float64)
+    elif dist == "continuous":
+        s = rng.random(U) * 40.0
+    elif dist == "ulps":
+        s = 1.0 + rng.integers(0, 4, size=U) * np.finfo(np.float64).eps
+    else:
+        s = np.where(rng.random(U) < 0.5, -1.0, 1.0) * 10.0 ** rng.uniform(-300, 300, size=U)
+    for k in (1, 2, U // 3, U // 2, U - 1, U):
+        _check_k(s, 1, k)
+
+
 @pytest.mark.parametrize("reps", [50, 100, 1000])  # 400, 800 and 8000 units
 def test_select_handles_negative_zero_and_subnormals(reps):
     s = np.array([0.0, -0.0, 5e-324, 1e-310, 0.0, 3.0, -0.0, 5e-324] * reps, np.float64)
