@@ -7,19 +7,21 @@
 //   warp 0            TMA producer, in both CTAs: per K step the CTA's own
 //                     128x64 hidden tile and its own half (128x64) of the pair's
 //                     256x64 vocabulary tile, into its own 4-stage shared-memory
-//                     ring (128-byte swizzle); the transaction bytes of both
-//                     CTAs complete on the even CTA's mbarrier.  Contiguous
-//                     rows: lane 0 loads both as boxes.  Rows in the loss a
-//                     subset (mask, rejected groups, fewer than 128 rows): the
-//                     hidden tile is read straight from the caller's
-//                     hidden-state tensor through the compact-row index.  Per
-//                     work item the warp splits the block's 128 rows into runs
-//                     of consecutive source rows (plan_block_loads) and each
-//                     run into boxes of 2^j rows; per K step one lane per box
-//                     issues its load (one box for a block inside a response).
-//                     A block of more than 32 boxes is fetched by four-row TMA
-//                     gathers (tile::gather4), one per lane.  No copy of the
-//                     rows is made.
+//                     ring (128-byte swizzle), as one TMA instruction of lanes
+//                     0..n (lane 0 the vocabulary half-tile, lanes 1..n the n
+//                     boxes of the hidden tile); each CTA arrives on the even
+//                     CTA's full barrier with its own bytes.  Contiguous rows:
+//                     one 128-row box.  Rows in the loss a subset (mask,
+//                     rejected groups, fewer than 128 rows): the hidden tile is
+//                     read straight from the caller's hidden-state tensor
+//                     through the compact-row index.  Per work item the warp
+//                     splits the block's 128 rows into runs of consecutive
+//                     source rows (plan_block_loads) and the runs into boxes of
+//                     2^j rows (one box for a block inside a response; the
+//                     first and last of several runs spill into 16 KB regions
+//                     around the tile).  A block of more than 31 boxes is
+//                     fetched by four-row TMA gathers (tile::gather4), one per
+//                     lane.  No copy of the rows is made.
 //   warp 1 / lane 0   MMA issuer, even CTA only: tcgen05.mma.cta_group::2
 //                     kind::f16 (bf16 x bf16 -> fp32), M=256 (128 rows from each
 //                     CTA), N=256 (128 vocabulary rows from each CTA), K=16 per
@@ -95,6 +97,7 @@ __host__ __device__ constexpr uint32_t b_tile_off(uint32_t s) { return kARegion 
 // Tensor maps of the hidden states with boxes of 1, 2, 4, ..., 128 rows (64
 // columns, 128-byte swizzle).
 constexpr int kBoxLevels = 8;
+constexpr int kMaxBoxes = 31;  // more boxes in a block: four-row gathers instead
 struct AMaps {
   CUtensorMap box[kBoxLevels];  // box[j]: 2^j rows
 };
@@ -328,108 +331,105 @@ __global__ void __cluster_dims__(CLUSTER, 1, 1) __launch_bounds__(kThreads, 1)
   };
 
   if (warp == 0) {
-    // rows by index (rows in the loss a subset, listed in rowidx): the whole
-    // warp produces; else lane 0 alone loads 128-row boxes
+    // ------------------------------------------------ TMA producer (both CTAs)
+    // The whole warp produces.  Per K step one TMA instruction, issued by
+    // lanes 0..n: lane 0 loads the CTA's half of the vocabulary tile, lanes
+    // 1..n the n boxes of its hidden tile (one 128-row box for contiguous rows;
+    // for rows read by index, the boxes plan_block_loads gives).  A block of
+    // more than kMaxBoxes boxes is gathered four rows a lane instead.
     const bool gather = p.gather != 0;
-    if (lane == 0 || gather) {
-      // ------------------------------------------------ TMA producer (both CTAs)
-      if (lane < kBoxLevels) tma_prefetch_desc(&am.box[lane]);
-      if (lane == 0) tma_prefetch_desc(&tm_b);
-      const uint64_t pol = make_policy_evict_normal();
-      uint32_t it = 0;
-      bool ok = true;
-      unsigned round = 0;  // this cluster's items so far (the round of the current one)
-      for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next(), ++round) {
-        const int64_t rp = c.item / n_splits;
-        const int split = static_cast<int>(c.item % n_splits);
-        const int64_t row0 = (rp * CLUSTER + crank) * BM;
-        // rows by index: this lane's box (first source row, first block row,
-        // level), or on a scattered block its four rows for a gather
-        int32_t psrc = 0, g4[4] = {0, 0, 0, 0};
-        int pdst = 0, plev = -1;
-        bool scattered = false;
-        uint32_t a_bytes = kStageA;  // this CTA's hidden-tile bytes per K step
-        if (gather) {
-          plan_block_loads(p.rowidx, row0, n_valid, p.max_level, lane, row_src, piece, plan);
-          const int n = plan[0];
-          scattered = n > 32;
-          if (!scattered) {
-            a_bytes = static_cast<uint32_t>(plan[1]);
-            if (lane < n) {
-              const int2 pc = piece[lane];
-              psrc = pc.x;
-              pdst = (pc.y & 0x1ff) - BM;  // first block row, -127..127
-              plev = pc.y >> 9;
-            }
-          } else {
-            // rows past the end gather row 0 (every gathered row exists)
-            const int64_t left = n_valid - row0;
+    if (lane == 0) tma_prefetch_desc(&tm_b);
+    if (lane < kBoxLevels) tma_prefetch_desc(&am.box[lane]);
+    const uint64_t pol = make_policy_evict_normal();
+    uint32_t it = 0;
+    bool ok = true;
+    unsigned round = 0;  // this cluster's items so far (the round of the current one)
+    for (ItemCursor c(cid, n_clusters, n_items); c.valid() && ok; c.next(), ++round) {
+      const int64_t rp = c.item / n_splits;
+      const int split = static_cast<int>(c.item % n_splits);
+      const int64_t row0 = (rp * CLUSTER + crank) * BM;
+      // this lane's load: lane 0 the vocabulary half-tile (its coordinates are
+      // set per tile below), lane 1 + q the hidden tile's box q
+      int n = 1;
+      uint32_t a_bytes = kStageA;  // this CTA's hidden-tile bytes per K step
+      int32_t psrc = static_cast<int32_t>(row0);
+      int pdst = 0, plev = kBoxLevels - 1;
+      int32_t g4[4] = {0, 0, 0, 0};
+      bool scattered = false;
+      if (gather) {
+        plan_block_loads(p.rowidx, row0, n_valid, p.max_level, lane, row_src, piece, plan);
+        n = plan[0];
+        scattered = n > kMaxBoxes;
+        if (!scattered) {
+          a_bytes = static_cast<uint32_t>(plan[1]);
+          if (lane >= 1 && lane <= n) {
+            const int2 pc = piece[lane - 1];
+            psrc = pc.x;
+            pdst = (pc.y & 0x1ff) - BM;  // first block row, -127..127
+            plev = pc.y >> 9;
+          }
+        } else {
 #pragma unroll
-            for (int j = 0; j < 4; ++j) g4[j] = 4 * lane + j < left ? row_src[4 * lane + j] : 0;
-          }
+          for (int j = 0; j < 4; ++j) g4[j] = row_src[4 * lane + j];  // row 0 past the end
         }
-        // every round before the last is full, so round k starts once all
-        // clusters issued their round k-1 loads (the even CTA paces the pair)
-        if (leader && lane == 0 && round > 0 && p.round_ctr)
-          wait_round(p.round_ctr, round * static_cast<unsigned>(n_clusters));
-        if (gather) __syncwarp();
-        const int tile0 = split * tiles_per_split;
-        const int tile1 = min(tile0 + tiles_per_split, p.n_vtiles);
-        for (int t = tile0; t < tile1 && ok; ++t) {
-          const int32_t nb = t * BN + static_cast<int32_t>(crank) * (BN / CLUSTER);
-          for (int kb = 0; kb < nkb; ++kb, ++it) {
-            const uint32_t s = it % STAGES;
-            const uint32_t ph = (it / STAGES) & 1u;
-            bool got = mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag);
-            if (gather) got = __all_sync(0xffffffffu, got);  // one outcome for the warp
-            if (!got) {
-              ok = false;
-              break;
-            }
-            unsigned char* sa = smem + a_tile_off(s);
-            unsigned char* sb = smem + b_tile_off(s);
-            const uint32_t bar = cluster_addr(&full[s], 0);
-            if (lane == 0) {
-              // this CTA's bytes of the stage, announced with its arrival on the
-              // even CTA's barrier (which completes once both CTAs' bytes land)
-              if (leader)
-                mbar_arrive_expect_tx(&full[s], a_bytes + kStageB);
-              else
-                mbar_arrive_expect_tx_cluster(bar, a_bytes + kStageB);
-              if (!gather)
-                tma_load_2d_pair(sa, &am.box[kBoxLevels - 1], bar, kb * BK,
-                                 static_cast<int32_t>(row0), pol);
-              tma_load_2d_pair(sb, &tm_b, bar, kb * BK, nb, pol);
-            }
-            if (gather) {
-              if (!scattered) {
-                if (plev >= 0)
-                  tma_load_2d_pair(sa + pdst * (BK * 2), &am.box[plev], bar, kb * BK, psrc, pol);
-              } else {
-                tma_gather4_pair(sa + lane * 4 * (BK * 2), &am.box[0], bar, kb * BK, g4[0],
-                                 g4[1], g4[2], g4[3], pol);
-              }
-            }
-          }
-        }
-        if (leader && lane == 0 && ok && p.round_ctr) atomicAdd(p.round_ctr, 1u);
-        if (gather) __syncwarp();  // row_src and piece are rewritten for the next item
       }
-      if (lane == 0) {
-        if (!ok) give_up();
-        // Drain: every copy issued must have landed before the CTA exits.  The
-        // even CTA sees both CTAs' bytes (all lanes' gathers included) on its
-        // full barriers; the odd CTA sees its stages consumed on its empty
-        // barriers.  After a timeout anywhere the waits are short: copies land
-        // in microseconds.
-        const uint64_t lim = *abort_flag ? 1000000ull : kWaitLimitNs;
-        for (uint32_t s = 0; s < STAGES && s < it; ++s) {
-          const uint32_t last = it - 1 - ((it - 1 - s) % STAGES);  // last index with stage s
-          if (leader)
-            mbar_wait_bounded(&full[s], (last / STAGES) & 1u, nullptr, lim);
-          else
-            mbar_wait_bounded(&empty[s], (last / STAGES) & 1u, nullptr, lim);
+      // every round before the last is full, so round k starts once all
+      // clusters issued their round k-1 loads (the even CTA paces the pair)
+      if (leader && lane == 0 && round > 0 && p.round_ctr)
+        wait_round(p.round_ctr, round * static_cast<unsigned>(n_clusters));
+      __syncwarp();
+      const int tile0 = split * tiles_per_split;
+      const int tile1 = min(tile0 + tiles_per_split, p.n_vtiles);
+      const int issuers = scattered ? 1 : n + 1;
+      for (int t = tile0; t < tile1 && ok; ++t) {
+        const int32_t nb = t * BN + static_cast<int32_t>(crank) * (BN / CLUSTER);
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const uint32_t s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1u;
+          // one outcome for the warp
+          if (!__all_sync(0xffffffffu, mbar_wait_bounded(&empty[s], ph ^ 1u, abort_flag))) {
+            ok = false;
+            break;
+          }
+          unsigned char* sa = smem + a_tile_off(s);
+          unsigned char* sb = smem + b_tile_off(s);
+          const uint32_t bar = cluster_addr(&full[s], 0);
+          if (lane == 0) {
+            // this CTA's bytes of the stage, announced with its arrival on the
+            // even CTA's barrier (which completes once both CTAs' bytes land)
+            if (leader)
+              mbar_arrive_expect_tx(&full[s], a_bytes + kStageB);
+            else
+              mbar_arrive_expect_tx_cluster(bar, a_bytes + kStageB);
+          }
+          if (lane < issuers) {
+            const void* desc = lane == 0 ? static_cast<const void*>(&tm_b)
+                                         : static_cast<const void*>(&am.box[plev]);
+            unsigned char* dst = lane == 0 ? sb : sa + pdst * (BK * 2);
+            tma_load_2d_pair(dst, desc, bar, kb * BK, lane == 0 ? nb : psrc, pol);
+          }
+          if (scattered)
+            tma_gather4_pair(sa + lane * 4 * (BK * 2), &am.box[0], bar, kb * BK, g4[0], g4[1],
+                             g4[2], g4[3], pol);
         }
+      }
+      if (leader && lane == 0 && ok && p.round_ctr) atomicAdd(p.round_ctr, 1u);
+      __syncwarp();  // row_src and piece are rewritten for the next item
+    }
+    if (lane == 0) {
+      if (!ok) give_up();
+      // Drain: every copy issued must have landed before the CTA exits.  The
+      // even CTA sees both CTAs' bytes (every lane's loads included) on its
+      // full barriers; the odd CTA sees its stages consumed on its empty
+      // barriers.  After a timeout anywhere the waits are short: copies land
+      // in microseconds.
+      const uint64_t lim = *abort_flag ? 1000000ull : kWaitLimitNs;
+      for (uint32_t s = 0; s < STAGES && s < it; ++s) {
+        const uint32_t last = it - 1 - ((it - 1 - s) % STAGES);  // last index with stage s
+        if (leader)
+          mbar_wait_bounded(&full[s], (last / STAGES) & 1u, nullptr, lim);
+        else
+          mbar_wait_bounded(&empty[s], (last / STAGES) & 1u, nullptr, lim);
       }
     }
   } else if (warp == 1) {
