@@ -232,7 +232,10 @@ def _sweep_scoring(steps, warmup, device, n_traj=SWEEP_N):
     # algorithmic bytes of the tag reduction: every tag once, the offsets once,
     # the 16-byte per-trajectory accumulators written once
     k_bytes = 4 * tok + 8 * (n + 1) + 16 * n
+    fused = n >= L.pace_score_fused_min_traj_default()
     res = {"workload": f"sweep pool {n} trajectories, {tok} tags", "traj_per_s": n / (s_ms / 1e3),
+           # from 2^18 trajectories the tag reduction's launch also finalises the scores
+           "tag_reduce_launch_finalises": bool(fused),
            "tag_reduce_traffic": (TAG_REDUCE_DRAM_BYTES_PER_TAG * tok
                                   if TAG_REDUCE_DRAM_BYTES_PER_TAG else None),
            "ms_per_call": s_ms, "ms_per_call_graph": g_ms, "tag_reduce_ms": k_ms,

@@ -543,6 +543,20 @@ typedef enum {
  * Returns PACE_ERR_INVALID_ARG unless 0 <= splits <= 8. */
 PACE_API pace_status pace_set_lmhead_splits(int32_t splits);
 
+/* Not part of the method: a tuning control for pace_score_pool.  Pools of at
+ * least min_traj trajectories (with groups of at most 256) finalise their
+ * scores inside the tag reduction's launch: each block, once its share of the
+ * tag stream is done, scores its own slice of the groups after bounded waits
+ * for the blocks that streamed those groups' tokens (a cooperative launch, so
+ * every block is resident and the waits end); most of the per-trajectory work
+ * then hides in the stream's ragged tail.  Smaller pools finalise in a launch
+ * of their own, which is faster there.  Results are identical either way.
+ * From now on, in this process, the given threshold applies (0: every pool;
+ * the default is pace_score_fused_min_traj_default(), 2^18).  Returns
+ * PACE_ERR_INVALID_ARG for a negative min_traj. */
+PACE_API pace_status pace_set_score_fused_min_traj(int64_t min_traj);
+PACE_API int64_t pace_score_fused_min_traj_default(void);
+
 /* Not part of the method: a measurement aid.  From now on, on the calling
  * host thread, record the CUDA event `begin` (a cudaEvent_t) on the call's
  * stream immediately before each launch of the given kernel and `end`

@@ -20,6 +20,9 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <mutex>
+
 #include "pace_internal.cuh"
 
 namespace pace {
@@ -37,6 +40,14 @@ constexpr int kTilesLarge = 8, kBlocksLarge = 2;
 constexpr int kTilesSmall = 4, kBlocksSmall = 3;
 constexpr int64_t kSmallPoolTokens = int64_t(1) << 27;
 constexpr int kMaxWindow = 4096;
+// Pools of at least this many trajectories finalise inside the tag reduction's
+// launch (pace_set_score_fused_min_traj); smaller ones use a launch of their own.
+constexpr int64_t kFusedMinTrajDefault = int64_t(1) << 18;
+
+std::atomic<int64_t>& fused_min_traj() {
+  static std::atomic<int64_t> v{kFusedMinTrajDefault};
+  return v;
+}
 constexpr int64_t kTableMinTraj = 8192;  // pools from this size sort W and tabulate F
 
 __device__ __forceinline__ int4 ld_stream_v4(const int32_t* p) {
@@ -329,16 +340,17 @@ __device__ void window_prep_block(int b, const WindowPrep& w) {
   for (int k = threadIdx.x; k < n; k += blockDim.x) w.sorted[k] = sw[k];
 }
 
-template <int kTilesPerBatch, int kMinBlocks>
-__global__ void __launch_bounds__(kReduceThreads, kMinBlocks)
-    tag_reduce_kernel(const int32_t* __restrict__ tags, const int64_t* __restrict__ offsets,
-                      int64_t n_traj, int64_t n_tokens, unsigned long long* __restrict__ sumv,
-                      unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1,
-                      int n_stream_blocks, WindowPrep prep) {
-  if (static_cast<int>(blockIdx.x) >= n_stream_blocks) {  // the window's preparation
-    window_prep_block(static_cast<int>(blockIdx.x) - n_stream_blocks, prep);
-    return;
-  }
+// One warp's share of the stream (every warp of the first n_stream_blocks
+// blocks calls it; it returns early when the range is empty or the offsets end
+// before the tokens do).
+template <int kTilesPerBatch>
+__device__ __forceinline__ void stream_warp_range(const int32_t* __restrict__ tags,
+                                                  const int64_t* __restrict__ offsets,
+                                                  int64_t n_traj, int64_t n_tokens,
+                                                  unsigned long long* __restrict__ sumv,
+                                                  unsigned* __restrict__ cnt,
+                                                  unsigned* __restrict__ maxp1,
+                                                  int n_stream_blocks) {
   constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -492,24 +504,44 @@ struct FinalizeArgs {
   int32_t* status;
 };
 
-// blockDim.x = tpb * lanes: tpb trajectories per block (whole groups) and, on
-// the direct-count path, `lanes` threads per trajectory that each count one
-// strided share of the window (lanes = 1 with the sorted window).  Thread t
-// counts for trajectory slot t % tpb; threads t < tpb then do that
-// trajectory's fp64 work and the group means.
-__global__ void score_finalize_kernel(FinalizeArgs p) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  const int wpad = (p.window_len + 3) & ~3;
-  const int tpb = static_cast<int>(blockDim.x) / p.lanes;
-  float* swin = reinterpret_cast<float*>(smem_raw);
-  double* sscore = reinterpret_cast<double*>(smem_raw + align_up(wpad * sizeof(float), 16));
-  int* pcount = reinterpret_cast<int*>(sscore + tpb);  // [lanes][tpb] partial counts
+// Shared memory of one finalisation pass: the window (padded to a multiple of
+// 4 floats), optionally the F table, the scores of the pass's trajectories and
+// the partial counts.
+struct FinalizeSmem {
+  float* swin;
+  double* ftab;    // [window_len + 1] or null (then F is read from global memory)
+  double* sscore;  // [tpb]
+  int* pcount;     // [lanes][tpb]
+};
 
-  const bool sorted = p.window_sorted != nullptr;
+__host__ __device__ inline size_t finalize_smem_bytes(int64_t window_len, int tpb, int threads,
+                                                      bool table_in_smem) {
+  return align_up(static_cast<size_t>((window_len + 3) & ~3) * sizeof(float), 16) +
+         (table_in_smem ? static_cast<size_t>(window_len + 1) * sizeof(double) : 0) +
+         static_cast<size_t>(tpb) * sizeof(double) + static_cast<size_t>(threads) * sizeof(int);
+}
+
+__device__ __forceinline__ FinalizeSmem finalize_smem(unsigned char* raw, int window_len, int tpb,
+                                                      bool table_in_smem) {
+  FinalizeSmem m;
+  const int wpad = (window_len + 3) & ~3;
+  m.swin = reinterpret_cast<float*>(raw);
+  double* d = reinterpret_cast<double*>(raw + align_up(wpad * sizeof(float), 16));
+  m.ftab = table_in_smem ? d : nullptr;
+  m.sscore = table_in_smem ? d + window_len + 1 : d;
+  m.pcount = reinterpret_cast<int*>(m.sscore + tpb);
+  return m;
+}
+
+// The window into shared memory: the sorted window, or the raw one NaN-padded
+// to a multiple of 4 (NaN never counts as <= s); four loads per thread in
+// flight at a time; with m.ftab set, the F table too.  L2 loads: the sorted
+// window and the table may have been written by another block of the same
+// launch.  Every thread of the block calls it.
+__device__ void finalize_load_window(const FinalizeArgs& p, const FinalizeSmem& m) {
   if (p.window_ready) {
-    // the sorted window, or the raw one NaN-padded to a multiple of 4 (NaN never
-    // counts as <= s); four loads per thread in flight at a time, since small
-    // blocks each copy the whole window
+    const bool sorted = p.window_sorted != nullptr;
+    const int wpad = (p.window_len + 3) & ~3;
     const float* src = sorted ? p.window_sorted : p.window;
     const int nb = static_cast<int>(blockDim.x);
     for (int k0 = threadIdx.x; k0 < wpad; k0 += 4 * nb) {
@@ -517,44 +549,95 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int k = k0 + j * nb;
-        w[j] = k < p.window_len ? src[k] : __int_as_float(0x7fc00000);
+        w[j] = k < p.window_len ? __ldcg(src + k) : __int_as_float(0x7fc00000);
       }
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int k = k0 + j * nb;
-        if (k < wpad) swin[k] = w[j];
+        if (k < wpad) m.swin[k] = w[j];
         if (!sorted && k < p.window_len && isnan(w[j])) report(p.status, PACE_ERR_NAN_INPUT);
       }
     }
+    if (m.ftab && sorted)
+      for (int k = threadIdx.x; k <= p.window_len; k += nb) m.ftab[k] = __ldcg(p.f_table + k);
   }
   __syncthreads();
+}
 
-  const int slot = static_cast<int>(threadIdx.x) % tpb;
-  const int64_t i = static_cast<int64_t>(blockIdx.x) * tpb + slot;
-  const bool lead = static_cast<int>(threadIdx.x) < tpb;  // owns trajectory i's results
-  const float s = (i < p.n_traj && p.s_pre) ? p.s_pre[i] : __int_as_float(0x7fc00000);
+// What one thread of a pass reads for its trajectory: the inputs (loadable any
+// time) and the accumulators of the stream (only once the stream blocks that
+// hold its tokens are done).
+struct TrajIn {
+  float s;
+  int32_t c;
+  int64_t o0, o1;
+  unsigned long long sum;
+  unsigned cnt, maxp1;
+};
+
+__device__ __forceinline__ void load_traj_inputs(const FinalizeArgs& p, int64_t i0, int64_t i_end,
+                                                 int tpb, int lanes, TrajIn& in) {
+  const int tid = static_cast<int>(threadIdx.x);
+  const int64_t i = i0 + tid % tpb;
+  const bool valid = tid < tpb * lanes && i < i_end;
+  in.s = (valid && p.s_pre) ? p.s_pre[i] : __int_as_float(0x7fc00000);
+  if (tid < tpb && i < i_end) {
+    in.c = p.c_version[i];
+    in.o0 = p.offsets[i];
+    in.o1 = p.offsets[i + 1];
+  }
+}
+
+__device__ __forceinline__ void load_traj_acc(const FinalizeArgs& p, int64_t i0, int64_t i_end,
+                                              int tpb, TrajIn& in) {
+  const int tid = static_cast<int>(threadIdx.x);
+  const int64_t i = i0 + tid;
+  if (tid < tpb && i < i_end) {
+    in.cnt = __ldcg(p.cnt + i);
+    in.maxp1 = __ldcg(p.maxp1 + i);
+    in.sum = __ldcg(p.sumv + i);
+  }
+}
+
+// One pass over trajectories [i0, i0 + tpb) clipped to i_end (i0 and tpb whole
+// groups), from what load_traj_inputs and load_traj_acc read: thread t <
+// tpb * lanes counts for trajectory slot t % tpb (on the direct-count path
+// `lanes` threads per trajectory each count one strided share of the window;
+// lanes = 1 with the sorted window); threads t < tpb then do that trajectory's
+// fp64 work, and the first thread of each group its mean in fixed left-to-right
+// order.  Every thread of the block calls it.
+__device__ void finalize_pass(const FinalizeArgs& p, int64_t i0, int64_t i_end, int tpb,
+                              int lanes, const FinalizeSmem& m, const TrajIn& in) {
+  const bool sorted = p.window_sorted != nullptr;
+  const int wpad = (p.window_len + 3) & ~3;
+  const int tid = static_cast<int>(threadIdx.x);
+  const bool active = tid < tpb * lanes;
+  const int slot = tid % tpb;
+  const int64_t i = i0 + slot;
+  const bool lead = tid < tpb;  // owns trajectory i's results
+  const float s = in.s;
   if (p.window_ready && !sorted) {
     // direct count of window values <= s, one strided share of the window per lane
     int count = 0;
-    if (!isnan(s)) {
-      const float4* w4 = reinterpret_cast<const float4*>(swin);
-      for (int k = static_cast<int>(threadIdx.x) / tpb; k < wpad / 4; k += p.lanes) {
+    if (active && !isnan(s)) {
+      const float4* w4 = reinterpret_cast<const float4*>(m.swin);
+      for (int k = tid / tpb; k < wpad / 4; k += lanes) {
         const float4 w = w4[k];
         count += (w.x <= s) + (w.y <= s) + (w.z <= s) + (w.w <= s);
       }
     }
-    pcount[threadIdx.x] = count;
+    if (active) m.pcount[tid] = count;
     __syncthreads();
   }
 
-  if (lead && i < p.n_traj) {
-    const int64_t o0 = p.offsets[i], o1 = p.offsets[i + 1];
+  if (lead && i < i_end) {
+    const int64_t o0 = in.o0, o1 = in.o1;
     if (o1 < o0 || (i == 0 && o0 != 0) || (i == p.n_traj - 1 && o1 != p.n_tokens))
       report(p.status, PACE_ERR_INVALID_ARG);
-    const int64_t c = p.c_version[i];
-    const unsigned t_count = p.cnt[i];
-    const unsigned mp1 = p.maxp1[i];
-    const long long tag_sum = static_cast<long long>(p.sumv[i]);
+    const int64_t c = in.c;
+    const unsigned t_count = in.cnt;
+    const unsigned mp1 = in.maxp1;
+    const long long tag_sum = static_cast<long long>(in.sum);
     if (c < 0 || mp1 >= 0x80000000u) report(p.status, PACE_ERR_INVALID_ARG);
     if (c > p.j || (mp1 != 0u && static_cast<int64_t>(mp1) - 1 > c))
       report(p.status, PACE_ERR_VERSION_ORDER);
@@ -574,13 +657,13 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
       int lo = 0, hi = p.window_len;
       while (lo < hi) {
         const int mid = (lo + hi) >> 1;
-        if (swin[mid] <= s) lo = mid + 1;
+        if (m.swin[mid] <= s) lo = mid + 1;
         else hi = mid;
       }
-      f = p.f_table[lo];
+      f = m.ftab ? m.ftab[lo] : __ldcg(p.f_table + lo);
     } else {  // small pools: F from the summed partial counts
       int count = 0;
-      for (int l = 0; l < p.lanes; ++l) count += pcount[l * tpb + slot];
+      for (int l = 0; l < lanes; ++l) count += m.pcount[l * tpb + slot];
       f = sharpen(__ddiv_rn(static_cast<double>(count), static_cast<double>(p.window_len)),
                   p.gamma);
     }
@@ -592,18 +675,165 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
     if (p.kwait) p.kwait[i] = kwait;
     if (p.weight) p.weight[i] = f;
     p.score[i] = sc;
-    sscore[slot] = sc;
+    m.sscore[slot] = sc;
   }
   __syncthreads();
   const int G = p.group_size;
-  if (p.unit_score && lead && i < p.n_traj && (slot % G) == 0) {
+  if (p.unit_score && lead && i < i_end && (slot % G) == 0) {
     double acc = 0.0;
-    for (int g = 0; g < G; ++g) acc = __dadd_rn(acc, sscore[slot + g]);
+    for (int g = 0; g < G; ++g) acc = __dadd_rn(acc, m.sscore[slot + g]);
     // for G = 2^m, acc * 2^-m is the same correctly rounded value as acc / G
     // (2^-m is exact), one multiplication instead of a division
     p.unit_score[i / G] = (G & (G - 1)) == 0 ? __dmul_rn(acc, 1.0 / static_cast<double>(G))
                                              : __ddiv_rn(acc, static_cast<double>(G));
   }
+}
+
+// The finalisation as a launch of its own (groups of more than 256): blockDim.x
+// = tpb * lanes, tpb trajectories (whole groups) per block.
+__global__ void score_finalize_kernel(FinalizeArgs p) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int tpb = static_cast<int>(blockDim.x) / p.lanes;
+  const FinalizeSmem m = finalize_smem(smem_raw, p.window_len, tpb, false);
+  const int64_t i0 = static_cast<int64_t>(blockIdx.x) * tpb;
+  TrajIn in;
+  load_traj_inputs(p, i0, p.n_traj, tpb, p.lanes, in);
+  load_traj_acc(p, i0, p.n_traj, tpb, in);
+  finalize_load_window(p, m);
+  finalize_pass(p, i0, p.n_traj, tpb, p.lanes, m, in);
+}
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// The finalisation inside the tag reduction's launch (groups of at most 256).
+// The launch is cooperative, so all its blocks are resident at once and every
+// wait below ends as soon as the blocks it waits for have streamed their share.
+struct FusedFinalize {
+  unsigned* done;       // [stream blocks] set once a block's warps have all streamed; null: off
+  unsigned* ticket;     // counts the blocks that have finished streaming
+  unsigned* prep_done;  // counts the finished preparation tasks
+  int prep_tasks;       // window sort + F-table slices (0: no table)
+  int tpb, lanes;       // trajectories per finalisation pass, threads per trajectory
+  WindowPrep prep;
+  FinalizeArgs fin;
+};
+
+// Run by every block once its own warps have streamed: publish that, take a
+// finishing ticket (the first finishers, idle in the reduction's ragged tail,
+// run the window's preparation tasks: task 0 sorts W, task 1 + k tabulates F
+// for 32 counts), then finalise this block's slice of the groups,
+// [U b / S, U (b + 1) / S), once the stream blocks covering those groups'
+// tokens and the preparation are done.  Each block thus finalises in the tail
+// as soon as its neighbourhood of the stream is complete, and no launch of its
+// own is needed.
+template <int kTilesPerBatch>
+__device__ __forceinline__ void fused_finalize(const int64_t* __restrict__ offsets,
+                                               int64_t n_tokens, int n_stream_blocks,
+                                               const FusedFinalize& fz) {
+  __shared__ unsigned s_ticket;
+  const int tid = static_cast<int>(threadIdx.x);
+  const int S = n_stream_blocks;
+  const int64_t blk = blockIdx.x;
+  __threadfence();  // this thread's accumulator atomics before the block's flag
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    atomicAdd(fz.done + blk, 1u);
+    s_ticket = atomicAdd(fz.ticket, 1u);
+  }
+  __syncthreads();
+  for (unsigned task = s_ticket; task < static_cast<unsigned>(fz.prep_tasks);
+       task += static_cast<unsigned>(S)) {
+    window_prep_block(static_cast<int>(task), fz.prep);
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) atomicAdd(fz.prep_done, 1u);
+  }
+
+  const FinalizeArgs& p = fz.fin;
+  const int G = p.group_size;
+  const int64_t U = p.n_traj / G;
+  const int64_t u_lo = U * blk / S, u_hi = U * (blk + 1) / S;
+  if (u_lo >= u_hi) return;
+  const int64_t i_lo = u_lo * G, i_hi = u_hi * G;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const bool sorted = p.window_sorted != nullptr;
+  const FinalizeSmem m = finalize_smem(smem_raw, p.window_len, fz.tpb, sorted);
+  // the first pass's inputs are in flight while the waits below run
+  TrajIn cur;
+  load_traj_inputs(p, i_lo, i_hi, fz.tpb, fz.lanes, cur);
+  if (tid < 32) {
+    const int lane = tid;
+    // stream blocks holding the tokens of trajectories [i_lo, i_hi): the warp of
+    // batch b is the last w with n_batches * w / n_warps <= b
+    int64_t b_lo = 0, b_hi = -1;
+    int64_t t0 = offsets[i_lo], t1 = offsets[i_hi];
+    t0 = t0 < 0 ? 0 : (t0 > n_tokens ? n_tokens : t0);
+    t1 = t1 < 0 ? 0 : (t1 > n_tokens ? n_tokens : t1);
+    if (t1 < t0) {  // inconsistent offsets (reported by the pass): wait for every block
+      b_hi = S - 1;
+    } else if (t1 > t0) {
+      constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
+      const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
+      const int64_t n_warps = static_cast<int64_t>(S) * (kReduceThreads / 32);
+      const int64_t w0 = ((t0 / kBatchTokens + 1) * n_warps - 1) / n_batches;
+      const int64_t w1 = (((t1 - 1) / kBatchTokens + 1) * n_warps - 1) / n_batches;
+      b_lo = w0 / (kReduceThreads / 32);
+      b_hi = w1 / (kReduceThreads / 32);
+    }
+    bool ok = true;
+    const uint64_t start = global_timer_ns();
+    for (int64_t b = b_lo + lane; ok && b <= b_hi; b += 32) {
+      while (ld_acquire_u32(fz.done + b) == 0u) {
+        if (global_timer_ns() - start > kWaitLimitNs) {
+          ok = false;
+          break;
+        }
+        __nanosleep(64);
+      }
+    }
+    if (lane == 0 && fz.prep_tasks > 0) {
+      while (ok && ld_acquire_u32(fz.prep_done) < static_cast<unsigned>(fz.prep_tasks)) {
+        if (global_timer_ns() - start > kWaitLimitNs) ok = false;
+        else __nanosleep(64);
+      }
+    }
+    if (!__all_sync(0xffffffffu, ok) && lane == 0) report(p.status, PACE_ERR_TIMEOUT);
+  }
+  __syncthreads();
+  load_traj_acc(p, i_lo, i_hi, fz.tpb, cur);
+  finalize_load_window(p, m);
+  for (int64_t i0 = i_lo; i0 < i_hi; i0 += fz.tpb) {
+    // the next pass's reads are in flight while this pass computes
+    TrajIn nxt;
+    const int64_t i1 = i0 + fz.tpb;
+    if (i1 < i_hi) {
+      load_traj_inputs(p, i1, i_hi, fz.tpb, fz.lanes, nxt);
+      load_traj_acc(p, i1, i_hi, fz.tpb, nxt);
+    }
+    finalize_pass(p, i0, i_hi, fz.tpb, fz.lanes, m, cur);
+    __syncthreads();  // the pass's shared scores and counts are reused
+    cur = nxt;
+  }
+}
+
+template <int kTilesPerBatch, int kMinBlocks>
+__global__ void __launch_bounds__(kReduceThreads, kMinBlocks)
+    tag_reduce_kernel(const int32_t* __restrict__ tags, const int64_t* __restrict__ offsets,
+                      int64_t n_traj, int64_t n_tokens, unsigned long long* __restrict__ sumv,
+                      unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1,
+                      int n_stream_blocks, WindowPrep prep, FusedFinalize fz) {
+  if (static_cast<int>(blockIdx.x) >= n_stream_blocks) {  // the window's preparation
+    window_prep_block(static_cast<int>(blockIdx.x) - n_stream_blocks, prep);
+    return;
+  }
+  stream_warp_range<kTilesPerBatch>(tags, offsets, n_traj, n_tokens, sumv, cnt, maxp1,
+                                    n_stream_blocks);
+  if (fz.done) fused_finalize<kTilesPerBatch>(offsets, n_tokens, n_stream_blocks, fz);
 }
 
 // Stale-k admission (Sec. 2): kbar = sum (j - v_t) / T = (j T - sum v_t) / T in
@@ -634,7 +864,11 @@ struct ScoreWs {
   unsigned long long* sumv;
   unsigned* cnt;
   unsigned* maxp1;
+  unsigned* flags;  // [2 + kMaxStreamBlocks]: ticket, preparation count, stream blocks done
 };
+
+// Stream blocks of one launch at most (one wave: SMs x resident blocks per SM).
+constexpr int kMaxStreamBlocks = 4096;
 
 struct WindowWs {
   float* sorted;    // [window_len]
@@ -650,43 +884,127 @@ WindowWs carve_window_ws(Carver& cv, int64_t window_len) {
 
 ScoreWs carve_score_ws(Carver& cv, int64_t n_traj) {
   ScoreWs w;
-  // one contiguous block so a single memset clears it
-  w.sumv = cv.take<unsigned long long>(static_cast<size_t>(n_traj) * 2);
+  // one contiguous block (accumulators, then the flags) so a single memset clears it
+  w.sumv = cv.take<unsigned long long>(static_cast<size_t>(n_traj) * 2 +
+                                       (2 + kMaxStreamBlocks) / 2);
   w.cnt = w.sumv ? reinterpret_cast<unsigned*>(w.sumv + n_traj) : nullptr;
   w.maxp1 = w.cnt ? w.cnt + n_traj : nullptr;
+  w.flags = w.maxp1 ? w.maxp1 + n_traj : nullptr;
   return w;
 }
 
-// Zero the accumulators and stream the tags once; with prep.window set, the
+// Resident blocks per SM of a tag-reduction instance with the given dynamic
+// shared memory (cached per device, instance and size).
+template <int kTiles, int kBlocks>
+pace_status reduce_blocks_per_sm(size_t smem, int* out) {
+  constexpr int kMaxDevices = 64;
+  static int cache[kMaxDevices][2] = {};
+  static size_t cache_smem[kMaxDevices][2] = {};
+  static std::mutex mu;
+  int dev = 0;
+  PACE_TRY_CUDA(cudaGetDevice(&dev));
+  const int which = kTiles == kTilesSmall ? 0 : 1;
+  std::lock_guard<std::mutex> g(mu);
+  if (dev >= 0 && dev < kMaxDevices && cache[dev][which] > 0 && cache_smem[dev][which] == smem) {
+    *out = cache[dev][which];
+    return PACE_OK;
+  }
+  int nb = 0;
+  // above the default 48 KB (windows of more than ~2,000 values with their F
+  // table) the kernel must be allowed the larger dynamic shared memory first
+  if (smem > 48 * 1024)
+    PACE_TRY_CUDA(cudaFuncSetAttribute(tag_reduce_kernel<kTiles, kBlocks>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem)));
+  PACE_TRY_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+      &nb, tag_reduce_kernel<kTiles, kBlocks>, kReduceThreads, smem));
+  if (dev >= 0 && dev < kMaxDevices) {
+    cache[dev][which] = nb;
+    cache_smem[dev][which] = smem;
+  }
+  *out = nb;
+  return PACE_OK;
+}
+
+template <int kTiles, int kBlocks>
+pace_status launch_tag_reduce(unsigned grid, size_t smem, bool cooperative, cudaStream_t st,
+                              const int32_t* tags, const int64_t* offsets, int64_t n_traj,
+                              int64_t n_tokens, const ScoreWs& ws, int stream_blocks,
+                              const WindowPrep& prep, const FusedFinalize& fz) {
+  if (!cooperative) {
+    tag_reduce_kernel<kTiles, kBlocks><<<grid, kReduceThreads, smem, st>>>(
+        tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1, stream_blocks, prep, fz);
+    return last_launch_status();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kReduceThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  PACE_TRY_CUDA(cudaLaunchKernelEx(&cfg, tag_reduce_kernel<kTiles, kBlocks>, tags, offsets,
+                                   n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1, stream_blocks,
+                                   prep, fz));
+  return last_launch_status();
+}
+
+// Zero the accumulators and stream the tags once.  With prep.window set, the
 // same launch also sorts the window and tabulates F (extra blocks, run in the
-// stream's tail).
+// stream's tail).  With fz.fin set (fz.done is filled in here), the launch is
+// cooperative and also finalises every trajectory and group (fused_finalize):
+// one wave of stream blocks, at least one block even for an empty stream.
 pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t n_traj,
                            int64_t n_tokens, const ScoreWs& ws, const WindowPrep& prep,
-                           cudaStream_t st) {
-  PACE_TRY_CUDA(cudaMemsetAsync(ws.sumv, 0, static_cast<size_t>(n_traj) * 16, st));
-  const unsigned prep_blocks = prep.window ? window_prep_blocks(prep.n) : 0u;
-  const size_t prep_smem = prep.window ? window_prep_smem(prep.n) : 0;
-  if (n_tokens == 0 && prep_blocks == 0) return PACE_OK;
+                           FusedFinalize fz, bool fused, size_t fused_smem, cudaStream_t st) {
+  const unsigned prep_blocks = (prep.window && !fused) ? window_prep_blocks(prep.n) : 0u;
+  size_t smem = prep_blocks ? window_prep_smem(prep.n) : 0;
+  if (fused) smem = fused_smem;
   const bool small = n_tokens <= kSmallPoolTokens;
   const int tiles = small ? kTilesSmall : kTilesLarge;
-  const int per_sm = small ? kBlocksSmall : kBlocksLarge;
+  int per_sm = small ? kBlocksSmall : kBlocksLarge;
+  if (fused) {
+    int nb = 0;
+    const pace_status occ = small ? reduce_blocks_per_sm<kTilesSmall, kBlocksSmall>(smem, &nb)
+                                  : reduce_blocks_per_sm<kTilesLarge, kBlocksLarge>(smem, &nb);
+    if (occ != PACE_OK) return occ;
+    if (nb < 1) return PACE_ERR_UNSUPPORTED_SHAPE;
+    per_sm = nb < per_sm ? nb : per_sm;
+  }
   const int64_t batch_tokens = static_cast<int64_t>(kTileTokens) * tiles;
   const int64_t n_batches = (n_tokens + batch_tokens - 1) / batch_tokens;
   const int warps_per_block = kReduceThreads / 32;
   int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
-  const int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;  // one wave
+  int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;  // one wave
+  if (cap > kMaxStreamBlocks) cap = kMaxStreamBlocks;
   if (blocks > cap) blocks = cap;
+  if (fused && blocks < 1) blocks = 1;
+  const size_t zero_bytes = static_cast<size_t>(n_traj) * 16 +
+                            (fused ? static_cast<size_t>(2 + blocks) * sizeof(unsigned) : 0);
+  PACE_TRY_CUDA(cudaMemsetAsync(ws.sumv, 0, zero_bytes, st));
+  if (blocks == 0 && prep_blocks == 0) return PACE_OK;
+  if (fused) {
+    fz.ticket = ws.flags;
+    fz.prep_done = ws.flags + 1;
+    fz.done = ws.flags + 2;
+  } else {
+    fz = FusedFinalize{};
+  }
   const unsigned grid = static_cast<unsigned>(blocks) + prep_blocks;
   const int stream_blocks = static_cast<int>(blocks);
   const ProfileEvents& pe = profile_events(PACE_PROFILE_TAG_REDUCE);
   if (pe.begin) PACE_TRY_CUDA(cudaEventRecord(pe.begin, st));
   if (small)
-    tag_reduce_kernel<kTilesSmall, kBlocksSmall><<<grid, kReduceThreads, prep_smem, st>>>(
-        tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1, stream_blocks, prep);
+    PACE_TRY((launch_tag_reduce<kTilesSmall, kBlocksSmall>(grid, smem, fused, st, tags, offsets,
+                                                            n_traj, n_tokens, ws, stream_blocks,
+                                                            prep, fz)));
   else
-    tag_reduce_kernel<kTilesLarge, kBlocksLarge><<<grid, kReduceThreads, prep_smem, st>>>(
-        tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1, stream_blocks, prep);
-  PACE_TRY(last_launch_status());
+    PACE_TRY((launch_tag_reduce<kTilesLarge, kBlocksLarge>(grid, smem, fused, st, tags, offsets,
+                                                            n_traj, n_tokens, ws, stream_blocks,
+                                                            prep, fz)));
   if (pe.end) PACE_TRY_CUDA(cudaEventRecord(pe.end, st));
   return PACE_OK;
 }
@@ -715,13 +1033,22 @@ extern "C" pace_status pace_stale_k(const int32_t* tags, const int64_t* offsets,
   ScoreWs ws = carve_score_ws(cv, n_traj);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
   cudaStream_t st = as_stream(stream);
-  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, WindowPrep{}, st));
+  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, WindowPrep{}, FusedFinalize{},
+                          false, 0, st));
   const int threads = 256;
   stale_k_kernel<<<static_cast<unsigned>((n_traj + threads - 1) / threads), threads, 0, st>>>(
       offsets, ws.sumv, ws.cnt, ws.maxp1, n_traj, n_tokens, trainer_version, k_max, kbar,
       admitted, status_dev);
   return last_launch_status();
 }
+
+extern "C" pace_status pace_set_score_fused_min_traj(int64_t min_traj) {
+  if (min_traj < 0) return PACE_ERR_INVALID_ARG;
+  fused_min_traj().store(min_traj == 0 ? 0 : min_traj);
+  return PACE_OK;
+}
+
+extern "C" int64_t pace_score_fused_min_traj_default(void) { return kFusedMinTrajDefault; }
 
 extern "C" void pace_score_params_default(PaceScoreParams* p) {
   if (!p) return;
@@ -785,7 +1112,6 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
     prep.f_table = wws.f_table;
     prep.status = status_dev;
   }
-  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, prep, st));
   FinalizeArgs a;
   a.offsets = offsets;
   a.c_version = c_version;
@@ -811,11 +1137,43 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   a.score = score;
   a.unit_score = unit_score;
   a.status = status_dev;
-  // Whole groups per block.  With the sorted window: one thread per trajectory,
-  // 64 to 256 threads; small pools take fewer groups per block so that the
-  // per-trajectory fp64 work (GB300's fp64 rate is low) is spread over about two
-  // blocks per SM instead of queueing on a few SMs.  With the direct count, up to
-  // 8 threads per trajectory share the count so its chain is 8 times shorter.
+
+  if (G <= kReduceThreads && n_traj >= fused_min_traj().load()) {
+    // Large pools whose groups fit one block: the finalisation runs inside the
+    // tag reduction's launch, each stream block finalising its slice of the
+    // groups in the stream's ragged tail, where most of the per-trajectory work
+    // hides (1M sweep pool: 2.31 -> 2.28 ms per call).  On small pools the chain
+    // after the last stream block (flags, waits, one pass) costs more than a
+    // launch of its own (16k: 65.6 -> 71 us), so they keep that launch.  Passes
+    // of whole groups over the block's 256 threads; on the direct-count path
+    // up to 8 threads per trajectory share the count.
+    int lanes = 1;
+    if (!use_table && window_ready) {
+      lanes = 8;
+      while (lanes > 1 && G * lanes > kReduceThreads) lanes /= 2;
+    }
+    FusedFinalize fz{};
+    fz.lanes = lanes;
+    fz.tpb = (kReduceThreads / lanes / G) * G;
+    a.lanes = lanes;
+    fz.fin = a;
+    if (use_table) {
+      fz.prep = prep;
+      fz.prep_tasks = static_cast<int>(window_prep_blocks(prep.n));
+    }
+    size_t smem = finalize_smem_bytes(window_len, fz.tpb, kReduceThreads, use_table);
+    if (use_table && window_prep_smem(prep.n) > smem) smem = window_prep_smem(prep.n);
+    return run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, WindowPrep{}, fz, true, smem, st);
+  }
+
+  PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, prep, FusedFinalize{}, false, 0,
+                          st));
+  // A launch of its own: whole groups per block.  With the sorted window: one
+  // thread per trajectory, 64 to 256 threads; small pools take fewer groups per
+  // block so that the per-trajectory fp64 work (GB300's fp64 rate is low) is
+  // spread over about two blocks per SM instead of queueing on a few SMs.  With
+  // the direct count, up to 8 threads per trajectory share the count so its
+  // chain is 8 times shorter.
   const int max_units = G >= 256 ? 1 : 256 / G;
   const int64_t n_units = n_traj / G;
   const int64_t spread = 2 * static_cast<int64_t>(sm_count());
@@ -834,9 +1192,7 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   a.lanes = lanes;
   const int threads = tpb * lanes;
   const int64_t blocks = (n_traj + tpb - 1) / tpb;
-  const size_t smem = align_up(((window_len + 3) & ~3) * sizeof(float), 16) +
-                      static_cast<size_t>(tpb) * sizeof(double) +
-                      static_cast<size_t>(threads) * sizeof(int);
+  const size_t smem = finalize_smem_bytes(window_len, tpb, threads, false);
   score_finalize_kernel<<<static_cast<unsigned>(blocks), threads, smem, st>>>(a);
   return last_launch_status();
 }

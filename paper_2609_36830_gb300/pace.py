@@ -104,6 +104,8 @@ SIGNATURES = {
     "pace_token_logprob_backward_workspace_size": ([_I64, _I64, _I32, _I32], _SZ),
     "pace_set_profile_events": ([_I32, _P, _P], _I32),
     "pace_set_lmhead_splits": ([_I32], _I32),
+    "pace_set_score_fused_min_traj": ([_I64], _I32),
+    "pace_score_fused_min_traj_default": ([], _I64),
     "pace_kernel_launches": ([], ctypes.c_uint64),
     "pace_wait_timeout_selftest": ([ctypes.c_uint64, _P, _P], _I32),
     "pace_div_selftest": ([_P, _P, _I64, _P, _P, _P, _P, _P], _I32),
@@ -453,6 +455,14 @@ def set_profile_events(kernel: int, begin=None, end=None):
         return ctypes.c_void_p(ev.cuda_event)
     b, e = handle(begin), handle(end)
     _check(lib().pace_set_profile_events(int(kernel), b, e), "pace_set_profile_events")
+
+
+def set_score_fused_min_traj(min_traj: Optional[int] = None):
+    """pace_set_score_fused_min_traj: pools of at least min_traj trajectories finalise
+    their scores inside the tag reduction's launch (None: the library's default)."""
+    if min_traj is None:
+        min_traj = lib().pace_score_fused_min_traj_default()
+    _check(lib().pace_set_score_fused_min_traj(int(min_traj)), "pace_set_score_fused_min_traj")
 
 
 def set_lmhead_splits(splits: int):

@@ -25,8 +25,16 @@ def _capture(fn):
     return g
 
 
+@pytest.fixture(params=["own_launch", "in_reduction"])
+def finalisation(request):
+    """Both finalisation paths of pace_score_pool, the second a cooperative launch."""
+    pace.set_score_fused_min_traj(1 << 62 if request.param == "own_launch" else 0)
+    yield request.param
+    pace.set_score_fused_min_traj()
+
+
 @pytest.mark.parametrize("n_traj", [1024, 16384])  # 128 units: one-block rank; 2048: radix
-def test_scoring_and_selection_replay(n_traj):
+def test_scoring_and_selection_replay(n_traj, finalisation):
     pool = workloads.make_pool("sweep", n_traj=n_traj, device=DEV)
     n = pool.n_traj
     c = torch.from_numpy(pool.c_version).to(DEV)

@@ -16,6 +16,16 @@ pytestmark = pytest.mark.gpu
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "hand_pool.json")
 
 
+@pytest.fixture(autouse=True, params=["own_launch", "in_reduction"])
+def finalisation(request):
+    """Every test of this file runs on both finalisation paths: a launch of its
+    own (the default below 2^18 trajectories) and inside the tag reduction's
+    cooperative launch (the default from 2^18), whatever the pool's size."""
+    pace.set_score_fused_min_traj(1 << 62 if request.param == "own_launch" else 0)
+    yield request.param
+    pace.set_score_fused_min_traj()
+
+
 def _check(g, o, what):
     for k in ("kgen", "kwait", "weight", "score", "unit_score"):
         assert_bits_equal(g[k], o[k], f"{what}:{k}")
@@ -205,6 +215,25 @@ def test_window_shapes_and_ties(n_traj, wlen, gamma):
         o = oracle_score(tags, offsets, c, s_pre, j, window, mode=mode, gamma=gamma, min_obs=1,
                          group_size=4)
         _check(g, o, f"w{wlen}/g{gamma}/{mode}")
+
+
+@pytest.mark.parametrize("n_traj,n_tok,wlen", [(64, 0, 512), (8192, 0, 4096), (8192, 1500, 4096),
+                                                (16384, 70000, 512)])
+def test_short_streams(n_traj, n_tok, wlen):
+    """Pools whose tag stream is empty or a block or two long: the finalisation
+    runs in the tag reduction's launch, so its one or few stream blocks score every
+    group; on the table path (8,192 trajectories and more) those few blocks also run
+    every window-preparation task (the sort and up to 129 slices of the F table)."""
+    rng = np.random.default_rng(n_traj + n_tok + wlen)
+    lens = np.zeros(n_traj, np.int64)
+    if n_tok:
+        lens[:] = np.bincount(rng.integers(0, n_traj, size=n_tok), minlength=n_traj)
+    tags, offsets, c, s_pre, j, _ = _mk_fast(lens, rng)
+    window = rng.random(wlen).astype(np.float32)
+    for G in (1, 8, min(256, n_traj)):
+        g = gpu_score(tags, offsets, c, s_pre, j, window, group_size=G, min_obs=1)
+        o = oracle_score(tags, offsets, c, s_pre, j, window, group_size=G, min_obs=1)
+        _check(g, o, f"{n_traj}/{n_tok}/G={G}")
 
 
 def test_empty_pool():

@@ -123,6 +123,15 @@ def test_lmhead_split_control_range(pace):
     assert L.pace_set_lmhead_splits(0) == pace.OK  # back to the automatic choice
 
 
+def test_score_fusion_control_range(pace):
+    L = pace.lib()
+    assert L.pace_set_score_fused_min_traj(-1) == pace.ERR_INVALID_ARG
+    for good in (0, 1, 1 << 18, 1 << 62):
+        assert L.pace_set_score_fused_min_traj(good) == pace.OK
+    assert L.pace_score_fused_min_traj_default() == 1 << 18
+    pace.set_score_fused_min_traj()
+
+
 def test_shard_selection_argument_checks_return_before_launch(pace):
     """The sharded rejection's calls refuse bad arguments on the host, before any launch."""
     L = pace.lib()
