@@ -186,28 +186,115 @@ __device__ __forceinline__ void acc_elem(LaneAcc& a, int32_t v, bool in_range) {
   a.maxp1 = (in && vp1 > a.maxp1) ? vp1 : a.maxp1;
 }
 
-// Warp-reduce the lane partials and add them to trajectory `traj`'s totals.
-// Integer adds and max are order-independent, so the totals are exact and
-// deterministic however trajectories are split across warps.
-__device__ __forceinline__ void flush(LaneAcc& a, int64_t traj, unsigned long long* sumv,
-                                      unsigned* cnt, unsigned* maxp1) {
+// The stream's per-trajectory totals, written without atomics (so nothing has
+// to be zeroed before a call).  The warp holding a trajectory's first token
+// writes its slot with one 16-byte store: x = the sum of its part's policy tags
+// with bit 63 set when the trajectory continues past that warp's range (the sum
+// of valid tags is below 2^63), y = count | (max tag + 1) << 32.  Every warp
+// writes one head slot: its part of the trajectory that began before its range
+// (traj = -1 if none).  A continuing trajectory's totals are its slot plus the
+// head slots of the following warps up to the one holding its last token.
+constexpr unsigned long long kContinues = 1ull << 63;
+
+struct HeadSlot {
+  long long traj;
+  unsigned long long sum;
+  unsigned cnt, maxp1;
+  long long pad;
+};
+
+struct TagTotals {
+  ulonglong2* slot;  // [n_traj]
+  HeadSlot* head;    // [stream warps]
+};
+
+// Geometry of one tag-reduction launch: warp w streams batches
+// [n_batches w / n_warps, n_batches (w + 1) / n_warps).
+struct StreamGeom {
+  int64_t batch_tokens;
+  int64_t n_batches;
+  int64_t n_warps;
+};
+
+// The last warp whose range starts at or before batch b (the one that streams it).
+__host__ __device__ __forceinline__ int64_t warp_of_batch(const StreamGeom& g, int64_t b) {
+  return ((b + 1) * g.n_warps - 1) / g.n_batches;
+}
+
+// Warp-reduce the lane partials and write them: the head slot of this warp, or
+// trajectory traj's slot.  Integer adds and max are order-independent, so the
+// totals are exact and deterministic however trajectories are split.
+__device__ __forceinline__ void emit(LaneAcc& a, int64_t traj, bool continues, bool head,
+                                     int64_t warp, const TagTotals& tt) {
   const unsigned full = 0xffffffffu;
-  const bool any = __any_sync(full, a.cnt != 0u);
-  if (any) {
-    long long s = a.sum;
+  long long s = a.sum;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(full, s, o);
-    const unsigned c = __reduce_add_sync(full, a.cnt);
-    const unsigned m = __reduce_max_sync(full, a.maxp1);
-    if ((threadIdx.x & 31) == 0) {
-      atomicAdd(&sumv[traj], static_cast<unsigned long long>(s));
-      atomicAdd(&cnt[traj], c);
-      atomicMax(&maxp1[traj], m);
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(full, s, o);
+  const unsigned c = __reduce_add_sync(full, a.cnt);
+  const unsigned m = __reduce_max_sync(full, a.maxp1);
+  if ((threadIdx.x & 31) == 0) {
+    if (head) {
+      HeadSlot h;
+      h.traj = traj;
+      h.sum = static_cast<unsigned long long>(s);
+      h.cnt = c;
+      h.maxp1 = m;
+      h.pad = 0;
+      tt.head[warp] = h;
+    } else {
+      ulonglong2 v;
+      v.x = static_cast<unsigned long long>(s) | (continues ? kContinues : 0ull);
+      v.y = static_cast<unsigned long long>(c) | (static_cast<unsigned long long>(m) << 32);
+      tt.slot[traj] = v;
     }
   }
   a.sum = 0;
   a.cnt = 0;
   a.maxp1 = 0;
+}
+
+// Trajectory i's totals (T, the exact sum of its policy tags, the largest tag
+// + 1) from the slots, given its offsets o0, o1.  Empty (or inconsistent)
+// ranges have zero totals (their slot, loaded regardless so that the load
+// need not wait for the offsets, is not used).  The head slots of a continuing
+// trajectory are loaded two at a time before either is used.  L2 loads: other
+// blocks of the same launch may have written the slots.
+__device__ __forceinline__ void traj_totals(const TagTotals& tt, const StreamGeom& g,
+                                            int64_t n_tokens, int64_t i, int64_t o0, int64_t o1,
+                                            long long& sum, unsigned& cnt, unsigned& maxp1) {
+  const ulonglong2 v = __ldcg(tt.slot + i);
+  sum = 0;
+  cnt = 0u;
+  maxp1 = 0u;
+  if (o0 < 0 || o1 <= o0 || o0 >= n_tokens) return;
+  sum = static_cast<long long>(v.x & ~kContinues);
+  cnt = static_cast<unsigned>(v.y);
+  maxp1 = static_cast<unsigned>(v.y >> 32);
+  if (v.x & kContinues) {
+    const int64_t last = (o1 < n_tokens ? o1 : n_tokens) - 1;
+    const int64_t w0 = warp_of_batch(g, o0 / g.batch_tokens);
+    const int64_t w1 = warp_of_batch(g, last / g.batch_tokens);
+    for (int64_t w = w0 + 1; w <= w1; w += 2) {
+      longlong2 h0[2], h1[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        if (w + u <= w1) {
+          const longlong2* hp = reinterpret_cast<const longlong2*>(tt.head + w + u);
+          h0[u] = __ldcg(hp);
+          h1[u] = __ldcg(hp + 1);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        if (w + u <= w1 && h0[u].x == i) {
+          sum += h0[u].y;
+          cnt += static_cast<unsigned>(h1[u].x);
+          const unsigned m = static_cast<unsigned>(static_cast<unsigned long long>(h1[u].x) >> 32);
+          maxp1 = m > maxp1 ? m : maxp1;
+        }
+      }
+    }
+  }
 }
 
 // The stream is integer-ALU heavy (a few operations per 4-byte tag), so the
@@ -347,10 +434,7 @@ template <int kTilesPerBatch>
 __device__ __forceinline__ void stream_warp_range(const int32_t* __restrict__ tags,
                                                   const int64_t* __restrict__ offsets,
                                                   int64_t n_traj, int64_t n_tokens,
-                                                  unsigned long long* __restrict__ sumv,
-                                                  unsigned* __restrict__ cnt,
-                                                  unsigned* __restrict__ maxp1,
-                                                  int n_stream_blocks) {
+                                                  const TagTotals& tt, int n_stream_blocks) {
   constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -358,8 +442,12 @@ __device__ __forceinline__ void stream_warp_range(const int32_t* __restrict__ ta
   const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
   const int64_t b_begin = n_batches * warp / n_warps;
   const int64_t b_end = n_batches * (warp + 1) / n_warps;
-  if (b_begin >= b_end) return;
+  if (b_begin >= b_end) {  // no tokens: no head part either
+    if (lane == 0) tt.head[warp].traj = -1;
+    return;
+  }
   const int64_t t_begin = b_begin * kBatchTokens;
+  const int64_t t_end = b_end * kBatchTokens < n_tokens ? b_end * kBatchTokens : n_tokens;
 
   // Start the stream before the search below: the warp's first batches are
   // requested into L2 while the offsets are searched (lanes 0..kPrefetchAhead-1,
@@ -390,7 +478,12 @@ __device__ __forceinline__ void stream_warp_range(const int32_t* __restrict__ ta
     }
   }
   int64_t cur = lo;
+  int64_t cur_begin = offsets[cur];
   int64_t cur_end = offsets[cur + 1];
+  // the first trajectory began before this range: this warp's part of it is its
+  // head slot; otherwise the head slot says there is none
+  const bool head_open = cur_begin < t_begin;
+  if (!head_open && lane == 0) tt.head[warp].traj = -1;
   LaneAcc acc{0, 0u, 0u};
 
   auto load_batch = [&](int4 (&v)[kTilesPerBatch], int64_t b) {
@@ -450,10 +543,11 @@ __device__ __forceinline__ void stream_warp_range(const int32_t* __restrict__ ta
         }
       }
       if (cur_end > bt1) return true;  // trajectory continues into the next batch
-      flush(acc, cur, sumv, cnt, maxp1);
+      emit(acc, cur, false, head_open && cur == lo, warp, tt);
       if (seg_hi > pos) pos = seg_hi;
       ++cur;
       if (cur >= n_traj) return false;  // tokens past the last trajectory: offsets are bad
+      cur_begin = cur_end;
       cur_end = offsets[cur + 1];
       // the next trajectory starts at the batch edge: continue in the next batch;
       // otherwise loop (more of this batch, or empty trajectories to step over)
@@ -473,7 +567,9 @@ __device__ __forceinline__ void stream_warp_range(const int32_t* __restrict__ ta
     if (!process(vb, b)) return;
     if (++b >= b_end) break;
   }
-  if (cur < n_traj) flush(acc, cur, sumv, cnt, maxp1);
+  // the trajectory still open continues past this range (one that begins at
+  // t_end belongs to the next warp)
+  if (cur < n_traj && cur_begin < t_end) emit(acc, cur, true, head_open && cur == lo, warp, tt);
 }
 
 struct FinalizeArgs {
@@ -483,9 +579,8 @@ struct FinalizeArgs {
   const float* window;           // W as given (used when window_sorted is null)
   const float* window_sorted;   // ascending, window_len values, or null
   const double* f_table;        // F for counts 0..window_len (with window_sorted)
-  const unsigned long long* sumv;
-  const unsigned* cnt;
-  const unsigned* maxp1;
+  TagTotals tt;
+  StreamGeom geom;
   int64_t n_traj;
   int64_t n_tokens;
   int32_t j;
@@ -593,9 +688,9 @@ __device__ __forceinline__ void load_traj_acc(const FinalizeArgs& p, int64_t i0,
   const int tid = static_cast<int>(threadIdx.x);
   const int64_t i = i0 + tid;
   if (tid < tpb && i < i_end) {
-    in.cnt = __ldcg(p.cnt + i);
-    in.maxp1 = __ldcg(p.maxp1 + i);
-    in.sum = __ldcg(p.sumv + i);
+    long long sum;
+    traj_totals(p.tt, p.geom, p.n_tokens, i, in.o0, in.o1, sum, in.cnt, in.maxp1);
+    in.sum = static_cast<unsigned long long>(sum);
   }
 }
 
@@ -694,7 +789,7 @@ __device__ void finalize_pass(const FinalizeArgs& p, int64_t i0, int64_t i_end, 
 __global__ void score_finalize_kernel(FinalizeArgs p) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int tpb = static_cast<int>(blockDim.x) / p.lanes;
-  const FinalizeSmem m = finalize_smem(smem_raw, p.window_len, tpb, false);
+  const FinalizeSmem m = finalize_smem(smem_raw, p.window_len, tpb, p.window_sorted != nullptr);
   const int64_t i0 = static_cast<int64_t>(blockIdx.x) * tpb;
   TrajIn in;
   load_traj_inputs(p, i0, p.n_traj, tpb, p.lanes, in);
@@ -824,23 +919,19 @@ __device__ __forceinline__ void fused_finalize(const int64_t* __restrict__ offse
 template <int kTilesPerBatch, int kMinBlocks>
 __global__ void __launch_bounds__(kReduceThreads, kMinBlocks)
     tag_reduce_kernel(const int32_t* __restrict__ tags, const int64_t* __restrict__ offsets,
-                      int64_t n_traj, int64_t n_tokens, unsigned long long* __restrict__ sumv,
-                      unsigned* __restrict__ cnt, unsigned* __restrict__ maxp1,
-                      int n_stream_blocks, WindowPrep prep, FusedFinalize fz) {
+                      int64_t n_traj, int64_t n_tokens, TagTotals tt, int n_stream_blocks,
+                      WindowPrep prep, FusedFinalize fz) {
   if (static_cast<int>(blockIdx.x) >= n_stream_blocks) {  // the window's preparation
     window_prep_block(static_cast<int>(blockIdx.x) - n_stream_blocks, prep);
     return;
   }
-  stream_warp_range<kTilesPerBatch>(tags, offsets, n_traj, n_tokens, sumv, cnt, maxp1,
-                                    n_stream_blocks);
+  stream_warp_range<kTilesPerBatch>(tags, offsets, n_traj, n_tokens, tt, n_stream_blocks);
   if (fz.done) fused_finalize<kTilesPerBatch>(offsets, n_tokens, n_stream_blocks, fz);
 }
 
 // Stale-k admission (Sec. 2): kbar = sum (j - v_t) / T = (j T - sum v_t) / T in
 // exact integers, one rounding; admitted when kbar <= k_max.
-__global__ void stale_k_kernel(const int64_t* __restrict__ offsets,
-                               const unsigned long long* __restrict__ sumv,
-                               const unsigned* __restrict__ cnt, const unsigned* __restrict__ maxp1,
+__global__ void stale_k_kernel(const int64_t* __restrict__ offsets, TagTotals tt, StreamGeom geom,
                                int64_t n_traj, int64_t n_tokens, int32_t j, double k_max,
                                double* __restrict__ kbar, uint8_t* __restrict__ admitted,
                                int32_t* status) {
@@ -849,26 +940,24 @@ __global__ void stale_k_kernel(const int64_t* __restrict__ offsets,
   const int64_t o0 = offsets[i], o1 = offsets[i + 1];
   if (o1 < o0 || (i == 0 && o0 != 0) || (i == n_traj - 1 && o1 != n_tokens))
     report(status, PACE_ERR_INVALID_ARG);
-  const unsigned t_count = cnt[i];
-  const unsigned mp1 = maxp1[i];
+  long long tag_sum;
+  unsigned t_count, mp1;
+  traj_totals(tt, geom, n_tokens, i, o0, o1, tag_sum, t_count, mp1);
   if (mp1 >= 0x80000000u) report(status, PACE_ERR_INVALID_ARG);
   if (mp1 != 0u && static_cast<int64_t>(mp1) - 1 > j) report(status, PACE_ERR_VERSION_ORDER);
-  const long long lag_sum = static_cast<long long>(j) * static_cast<long long>(t_count) -
-                            static_cast<long long>(sumv[i]);
+  const long long lag_sum = static_cast<long long>(j) * static_cast<long long>(t_count) - tag_sum;
   const double kb = t_count > 0u ? i64_div_u32_rn(lag_sum, t_count) : 0.0;
   if (kbar) kbar[i] = kb;
   admitted[i] = kb <= k_max ? 1 : 0;
 }
 
+// Stream blocks of one launch at most (one wave: SMs x resident blocks per SM).
+constexpr int kMaxStreamBlocks = 2048;
+
 struct ScoreWs {
-  unsigned long long* sumv;
-  unsigned* cnt;
-  unsigned* maxp1;
+  TagTotals tt;     // slots [n_traj], head slots [kMaxStreamBlocks x 8 warps]
   unsigned* flags;  // [2 + kMaxStreamBlocks]: ticket, preparation count, stream blocks done
 };
-
-// Stream blocks of one launch at most (one wave: SMs x resident blocks per SM).
-constexpr int kMaxStreamBlocks = 4096;
 
 struct WindowWs {
   float* sorted;    // [window_len]
@@ -884,12 +973,9 @@ WindowWs carve_window_ws(Carver& cv, int64_t window_len) {
 
 ScoreWs carve_score_ws(Carver& cv, int64_t n_traj) {
   ScoreWs w;
-  // one contiguous block (accumulators, then the flags) so a single memset clears it
-  w.sumv = cv.take<unsigned long long>(static_cast<size_t>(n_traj) * 2 +
-                                       (2 + kMaxStreamBlocks) / 2);
-  w.cnt = w.sumv ? reinterpret_cast<unsigned*>(w.sumv + n_traj) : nullptr;
-  w.maxp1 = w.cnt ? w.cnt + n_traj : nullptr;
-  w.flags = w.maxp1 ? w.maxp1 + n_traj : nullptr;
+  w.tt.slot = cv.take<ulonglong2>(static_cast<size_t>(n_traj));
+  w.tt.head = cv.take<HeadSlot>(static_cast<size_t>(kMaxStreamBlocks) * (kReduceThreads / 32));
+  w.flags = cv.take<unsigned>(2 + kMaxStreamBlocks);
   return w;
 }
 
@@ -933,7 +1019,7 @@ pace_status launch_tag_reduce(unsigned grid, size_t smem, bool cooperative, cuda
                               const WindowPrep& prep, const FusedFinalize& fz) {
   if (!cooperative) {
     tag_reduce_kernel<kTiles, kBlocks><<<grid, kReduceThreads, smem, st>>>(
-        tags, offsets, n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1, stream_blocks, prep, fz);
+        tags, offsets, n_traj, n_tokens, ws.tt, stream_blocks, prep, fz);
     return last_launch_status();
   }
   cudaLaunchConfig_t cfg = {};
@@ -947,19 +1033,20 @@ pace_status launch_tag_reduce(unsigned grid, size_t smem, bool cooperative, cuda
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   PACE_TRY_CUDA(cudaLaunchKernelEx(&cfg, tag_reduce_kernel<kTiles, kBlocks>, tags, offsets,
-                                   n_traj, n_tokens, ws.sumv, ws.cnt, ws.maxp1, stream_blocks,
-                                   prep, fz));
+                                   n_traj, n_tokens, ws.tt, stream_blocks, prep, fz));
   return last_launch_status();
 }
 
-// Zero the accumulators and stream the tags once.  With prep.window set, the
-// same launch also sorts the window and tabulates F (extra blocks, run in the
-// stream's tail).  With fz.fin set (fz.done is filled in here), the launch is
-// cooperative and also finalises every trajectory and group (fused_finalize):
-// one wave of stream blocks, at least one block even for an empty stream.
+// Stream the tags once into the slots (nothing to zero first).  With
+// prep.window set, the same launch also sorts the window and tabulates F
+// (extra blocks, run in the stream's tail).  With `fused` (fz.done is filled in
+// here, its flags zeroed), the launch is cooperative and also finalises every
+// trajectory and group (fused_finalize): one wave of stream blocks, at least
+// one block even for an empty stream.  *geom receives the launch's geometry.
 pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t n_traj,
                            int64_t n_tokens, const ScoreWs& ws, const WindowPrep& prep,
-                           FusedFinalize fz, bool fused, size_t fused_smem, cudaStream_t st) {
+                           FusedFinalize fz, bool fused, size_t fused_smem, StreamGeom* geom,
+                           cudaStream_t st) {
   const unsigned prep_blocks = (prep.window && !fused) ? window_prep_blocks(prep.n) : 0u;
   size_t smem = prep_blocks ? window_prep_smem(prep.n) : 0;
   if (fused) smem = fused_smem;
@@ -982,14 +1069,17 @@ pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t 
   if (cap > kMaxStreamBlocks) cap = kMaxStreamBlocks;
   if (blocks > cap) blocks = cap;
   if (fused && blocks < 1) blocks = 1;
-  const size_t zero_bytes = static_cast<size_t>(n_traj) * 16 +
-                            (fused ? static_cast<size_t>(2 + blocks) * sizeof(unsigned) : 0);
-  PACE_TRY_CUDA(cudaMemsetAsync(ws.sumv, 0, zero_bytes, st));
+  geom->batch_tokens = batch_tokens;
+  geom->n_batches = n_batches;
+  geom->n_warps = blocks * warps_per_block;
   if (blocks == 0 && prep_blocks == 0) return PACE_OK;
   if (fused) {
+    PACE_TRY_CUDA(cudaMemsetAsync(ws.flags, 0, static_cast<size_t>(2 + blocks) * sizeof(unsigned),
+                                  st));
     fz.ticket = ws.flags;
     fz.prep_done = ws.flags + 1;
     fz.done = ws.flags + 2;
+    fz.fin.geom = *geom;
   } else {
     fz = FusedFinalize{};
   }
@@ -1033,11 +1123,12 @@ extern "C" pace_status pace_stale_k(const int32_t* tags, const int64_t* offsets,
   ScoreWs ws = carve_score_ws(cv, n_traj);
   if (!cv.fits()) return PACE_ERR_WORKSPACE;
   cudaStream_t st = as_stream(stream);
+  StreamGeom geom{};
   PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, WindowPrep{}, FusedFinalize{},
-                          false, 0, st));
+                          false, 0, &geom, st));
   const int threads = 256;
   stale_k_kernel<<<static_cast<unsigned>((n_traj + threads - 1) / threads), threads, 0, st>>>(
-      offsets, ws.sumv, ws.cnt, ws.maxp1, n_traj, n_tokens, trainer_version, k_max, kbar,
+      offsets, ws.tt, geom, n_traj, n_tokens, trainer_version, k_max, kbar,
       admitted, status_dev);
   return last_launch_status();
 }
@@ -1119,9 +1210,8 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   a.window = window;
   a.window_sorted = use_table ? wws.sorted : nullptr;
   a.f_table = use_table ? wws.f_table : nullptr;
-  a.sumv = ws.sumv;
-  a.cnt = ws.cnt;
-  a.maxp1 = ws.maxp1;
+  a.tt = ws.tt;
+  a.geom = StreamGeom{};
   a.n_traj = n_traj;
   a.n_tokens = n_tokens;
   a.j = trainer_version;
@@ -1163,11 +1253,13 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
     }
     size_t smem = finalize_smem_bytes(window_len, fz.tpb, kReduceThreads, use_table);
     if (use_table && window_prep_smem(prep.n) > smem) smem = window_prep_smem(prep.n);
-    return run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, WindowPrep{}, fz, true, smem, st);
+    StreamGeom geom{};
+    return run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, WindowPrep{}, fz, true, smem, &geom,
+                          st);
   }
 
   PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, prep, FusedFinalize{}, false, 0,
-                          st));
+                          &a.geom, st));
   // A launch of its own: whole groups per block.  With the sorted window: one
   // thread per trajectory, 64 to 256 threads; small pools take fewer groups per
   // block so that the per-trajectory fp64 work (GB300's fp64 rate is low) is
@@ -1192,7 +1284,11 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   a.lanes = lanes;
   const int threads = tpb * lanes;
   const int64_t blocks = (n_traj + tpb - 1) / tpb;
-  const size_t smem = finalize_smem_bytes(window_len, tpb, threads, false);
+  const size_t smem = finalize_smem_bytes(window_len, tpb, threads, use_table);
+  if (smem > 48 * 1024)
+    PACE_TRY_CUDA(cudaFuncSetAttribute(score_finalize_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem)));
   score_finalize_kernel<<<static_cast<unsigned>(blocks), threads, smem, st>>>(a);
   return last_launch_status();
 }

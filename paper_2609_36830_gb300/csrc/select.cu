@@ -189,7 +189,7 @@ __global__ void __launch_bounds__(kSmallThreads)
 // consecutive positions (whole 32-byte sectors per warp store), four ids and
 // four flags per store when G is a multiple of 4 and the buffers are aligned.
 // C is the smallest power of two that keeps each CTA at 16,384 units and
-// 16,384 outputs or fewer; a cluster of one uses block barriers and plain
+// 32,768 outputs or fewer; a cluster of one uses block barriers and plain
 // shared memory instead (the kMulti = false instance).
 constexpr int kSelCtaUnits = 16384;  // units per CTA at most
 constexpr int kSelThreads = 1024;
@@ -393,7 +393,8 @@ __global__ void __launch_bounds__(kSelThreads, 1)
       if (top >= 0) h0 = hist[top];
       if (top >= 1) h1 = hist[top - 1];
     }
-    long long run = block_exclusive_scan<long long>(h0 + h1, nullptr);
+    // every count fits 32 bits (at most kSelMaxUnits keys in the cluster)
+    long long run = block_exclusive_scan<unsigned>(static_cast<unsigned>(h0 + h1), nullptr);
     if (top >= 0 && run < k_rem && k_rem <= run + h0) {
       s_digit = top;
       s_left = k_rem - run;
@@ -427,33 +428,45 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   if (!ok && t == 0 && rank == 0) report(status, PACE_ERR_INVALID_ARG);
   const uint64_t pivot = lo;  // k_rem of the keys equal to it are rejected, lowest ids first
 
-  int eq = 0, gt = 0;
+  // keys equal to the pivot (high 16 bits) and above it (low 16 bits) of this
+  // thread, scanned together: a CTA holds at most 16,384 keys, so neither field
+  // carries into the other
+  unsigned eqgt = 0u;
   for (int i = 0; i < n_mine; ++i) {
     const uint64_t key = keys[i * kSelRow + t];
-    eq += key == pivot;
-    gt += key > pivot;
+    eqgt += (key == pivot ? 0x10000u : 0u) + (key > pivot ? 1u : 0u);
   }
-  long long cta_eq = 0, cta_gt = 0;
-  const long long tie_local = block_exclusive_scan<long long>(eq, &cta_eq);
-  block_exclusive_scan<long long>(gt, &cta_gt);
+  unsigned cta_eqgt = 0u;
+  const long long tie_local = block_exclusive_scan<unsigned>(eqgt, &cta_eqgt) >> 16;
   if (t == 0) {
-    s_cnt[0] = cta_eq;
-    s_cnt[1] = cta_gt;
+    s_cnt[0] = cta_eqgt >> 16;
+    s_cnt[1] = cta_eqgt & 0xffffu;
   }
   if (kMulti) cluster.sync();  // every CTA's counts are written
   else __syncthreads();
-  if (t == 0) {
-    long long ties_before = 0, rej_before = 0;
-    for (int r = 0; r < (kMulti ? rank : 0); ++r) {
-      const long long* pc = cluster.map_shared_rank(s_cnt, static_cast<unsigned>(r));
-      const long long e = pc[0];
-      long long take = k_rem - ties_before;  // ties of CTA r that are rejected
-      take = take < 0 ? 0 : (take > e ? e : take);
-      rej_before += pc[1] + take;
-      ties_before += e;
+  if (t < 32) {
+    // lanes r < rank read CTA r's counts at once; lane 0 folds them in rank order
+    long long e = 0, g = 0;
+    if (kMulti && t < rank) {
+      const long long* pc = cluster.map_shared_rank(s_cnt, static_cast<unsigned>(t));
+      e = pc[0];
+      g = pc[1];
     }
-    s_off[0] = ties_before;
-    s_off[1] = rej_before;
+    long long ties_before = 0, rej_before = 0;
+    for (int r = 0; r < kSelMaxCluster; ++r) {
+      const long long er = __shfl_sync(0xffffffffu, e, r);
+      const long long gr = __shfl_sync(0xffffffffu, g, r);
+      if (r < (kMulti ? rank : 0)) {
+        long long take = k_rem - ties_before;  // ties of CTA r that are rejected
+        take = take < 0 ? 0 : (take > er ? er : take);
+        rej_before += gr + take;
+        ties_before += er;
+      }
+    }
+    if (t == 0) {
+      s_off[0] = ties_before;
+      s_off[1] = rej_before;
+    }
   }
   if (kMulti) cluster.sync();  // peers' counts are read: no CTA touches another's memory after this
   else __syncthreads();
@@ -467,8 +480,9 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     const uint64_t key = keys[i * kSelRow + t];
     nrej += key > pivot || (key == pivot && (tie++) < k_rem);
   }
-  long long cta_rej = 0;
-  long long lrpos = block_exclusive_scan<long long>(nrej, &cta_rej);
+  unsigned cta_rej32 = 0u;
+  long long lrpos = block_exclusive_scan<unsigned>(static_cast<unsigned>(nrej), &cta_rej32);
+  const long long cta_rej = cta_rej32;
   const long long n_acc_cta = nb - cta_rej;
   tie = tie0;
   for (int i = 0; i < n_mine; ++i) {
@@ -793,13 +807,17 @@ pace_status sel_cluster_limit(int* out) {
 }
 
 // Cluster size for U units of G trajectories: enough CTAs to hold the keys
-// (16,384 each) and one more SM per doubling of the outputs above 16,384, up to
-// the device's limit; 0 when the keys do not fit the largest cluster.
+// (16,384 each) and one more SM per doubling of the outputs above 32,768, up to
+// the device's limit; 0 when the keys do not fit the largest cluster.  Fewer
+// CTAs mean cheaper cluster barriers and fewer distributed-shared-memory reads
+// per round; more spread the writing of the id lists.  On the 16,384 groups of
+// the 128k sweep pool (131,072 outputs) 4 CTAs took 331.5 us per scoring +
+// selection call against 336 with 8 and 336 with 2 (CUDA-graph replays).
 int sel_cluster_size(int64_t n_units, int G, int limit) {
   const int64_t total = n_units * G;
   int c = 1;
   while (c < limit && (n_units > static_cast<int64_t>(c) * kSelCtaUnits ||
-                       total > static_cast<int64_t>(c) * 16384))
+                       total > static_cast<int64_t>(c) * 32768))
     c *= 2;
   return n_units <= static_cast<int64_t>(c) * kSelCtaUnits ? c : 0;
 }
