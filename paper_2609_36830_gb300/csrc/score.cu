@@ -39,6 +39,13 @@ constexpr int kTileTokens = 128;     // one int4 per lane
 constexpr int kTilesLarge = 8, kBlocksLarge = 2;
 constexpr int kTilesSmall = 4, kBlocksSmall = 3;
 constexpr int64_t kSmallPoolTokens = int64_t(1) << 27;
+// Short streams get fewer warps rather than fewer batches a warp: below this
+// many batches a warp, trajectories spread over several warps' ranges and their
+// totals need more head slots.  On the 1k sweep pool (3.6 M tags, ~3,500 a
+// trajectory) whole calls took 30.3 / 29.0 / 27.2 / 28.6 / 31.3 us with at
+// least 1 / 2 / 4 / 8 / 16 batches a warp (the stream itself 12.3 -> 18.3 us);
+// pools from ~15 M tags keep one full wave and are not affected.
+constexpr int64_t kMinBatchesPerWarp = 4;
 constexpr int kMaxWindow = 4096;
 // Pools of at least this many trajectories finalise inside the tag reduction's
 // launch (pace_set_score_fused_min_traj); smaller ones use a launch of their own.
@@ -254,15 +261,15 @@ __device__ __forceinline__ void emit(LaneAcc& a, int64_t traj, bool continues, b
 }
 
 // Trajectory i's totals (T, the exact sum of its policy tags, the largest tag
-// + 1) from the slots, given its offsets o0, o1.  Empty (or inconsistent)
-// ranges have zero totals (their slot, loaded regardless so that the load
-// need not wait for the offsets, is not used).  The head slots of a continuing
+// + 1) from its slot v and the head slots, given its offsets o0, o1.  Empty (or
+// inconsistent) ranges have zero totals (their slot, loaded regardless so that
+// the load need not wait for the offsets, is not used).  The head slots of a continuing
 // trajectory are loaded two at a time before either is used.  L2 loads: other
 // blocks of the same launch may have written the slots.
 __device__ __forceinline__ void traj_totals(const TagTotals& tt, const StreamGeom& g,
                                             int64_t n_tokens, int64_t i, int64_t o0, int64_t o1,
-                                            long long& sum, unsigned& cnt, unsigned& maxp1) {
-  const ulonglong2 v = __ldcg(tt.slot + i);
+                                            const ulonglong2& v, long long& sum, unsigned& cnt,
+                                            unsigned& maxp1) {
   sum = 0;
   cnt = 0u;
   maxp1 = 0u;
@@ -666,6 +673,7 @@ struct TrajIn {
   float s;
   int32_t c;
   int64_t o0, o1;
+  ulonglong2 slot;
   unsigned long long sum;
   unsigned cnt, maxp1;
 };
@@ -683,13 +691,22 @@ __device__ __forceinline__ void load_traj_inputs(const FinalizeArgs& p, int64_t 
   }
 }
 
+// The stream's slot of this thread's trajectory (issue it early: its load need
+// not wait for anything), then the totals (which may load head slots).
+__device__ __forceinline__ void load_traj_slot(const FinalizeArgs& p, int64_t i0, int64_t i_end,
+                                               int tpb, TrajIn& in) {
+  const int tid = static_cast<int>(threadIdx.x);
+  const int64_t i = i0 + tid;
+  if (tid < tpb && i < i_end) in.slot = __ldcg(p.tt.slot + i);
+}
+
 __device__ __forceinline__ void load_traj_acc(const FinalizeArgs& p, int64_t i0, int64_t i_end,
                                               int tpb, TrajIn& in) {
   const int tid = static_cast<int>(threadIdx.x);
   const int64_t i = i0 + tid;
   if (tid < tpb && i < i_end) {
     long long sum;
-    traj_totals(p.tt, p.geom, p.n_tokens, i, in.o0, in.o1, sum, in.cnt, in.maxp1);
+    traj_totals(p.tt, p.geom, p.n_tokens, i, in.o0, in.o1, in.slot, sum, in.cnt, in.maxp1);
     in.sum = static_cast<unsigned long long>(sum);
   }
 }
@@ -791,10 +808,13 @@ __global__ void score_finalize_kernel(FinalizeArgs p) {
   const int tpb = static_cast<int>(blockDim.x) / p.lanes;
   const FinalizeSmem m = finalize_smem(smem_raw, p.window_len, tpb, p.window_sorted != nullptr);
   const int64_t i0 = static_cast<int64_t>(blockIdx.x) * tpb;
+  // the inputs, the slot and the window are in flight together; the head slots
+  // of continuing trajectories are loaded once the window is in place
   TrajIn in;
   load_traj_inputs(p, i0, p.n_traj, tpb, p.lanes, in);
-  load_traj_acc(p, i0, p.n_traj, tpb, in);
+  load_traj_slot(p, i0, p.n_traj, tpb, in);
   finalize_load_window(p, m);
+  load_traj_acc(p, i0, p.n_traj, tpb, in);
   finalize_pass(p, i0, p.n_traj, tpb, p.lanes, m, in);
 }
 
@@ -900,14 +920,16 @@ __device__ __forceinline__ void fused_finalize(const int64_t* __restrict__ offse
     if (!__all_sync(0xffffffffu, ok) && lane == 0) report(p.status, PACE_ERR_TIMEOUT);
   }
   __syncthreads();
-  load_traj_acc(p, i_lo, i_hi, fz.tpb, cur);
+  load_traj_slot(p, i_lo, i_hi, fz.tpb, cur);
   finalize_load_window(p, m);
+  load_traj_acc(p, i_lo, i_hi, fz.tpb, cur);
   for (int64_t i0 = i_lo; i0 < i_hi; i0 += fz.tpb) {
     // the next pass's reads are in flight while this pass computes
     TrajIn nxt;
     const int64_t i1 = i0 + fz.tpb;
     if (i1 < i_hi) {
       load_traj_inputs(p, i1, i_hi, fz.tpb, fz.lanes, nxt);
+      load_traj_slot(p, i1, i_hi, fz.tpb, nxt);
       load_traj_acc(p, i1, i_hi, fz.tpb, nxt);
     }
     finalize_pass(p, i0, i_hi, fz.tpb, fz.lanes, m, cur);
@@ -942,7 +964,7 @@ __global__ void stale_k_kernel(const int64_t* __restrict__ offsets, TagTotals tt
     report(status, PACE_ERR_INVALID_ARG);
   long long tag_sum;
   unsigned t_count, mp1;
-  traj_totals(tt, geom, n_tokens, i, o0, o1, tag_sum, t_count, mp1);
+  traj_totals(tt, geom, n_tokens, i, o0, o1, __ldcg(tt.slot + i), tag_sum, t_count, mp1);
   if (mp1 >= 0x80000000u) report(status, PACE_ERR_INVALID_ARG);
   if (mp1 != 0u && static_cast<int64_t>(mp1) - 1 > j) report(status, PACE_ERR_VERSION_ORDER);
   const long long lag_sum = static_cast<long long>(j) * static_cast<long long>(t_count) - tag_sum;
@@ -1064,7 +1086,8 @@ pace_status run_tag_reduce(const int32_t* tags, const int64_t* offsets, int64_t 
   const int64_t batch_tokens = static_cast<int64_t>(kTileTokens) * tiles;
   const int64_t n_batches = (n_tokens + batch_tokens - 1) / batch_tokens;
   const int warps_per_block = kReduceThreads / 32;
-  int64_t blocks = (n_batches + warps_per_block - 1) / warps_per_block;
+  const int64_t per_block = warps_per_block * kMinBatchesPerWarp;
+  int64_t blocks = (n_batches + per_block - 1) / per_block;
   int64_t cap = static_cast<int64_t>(sm_count()) * per_sm;  // one wave
   if (cap > kMaxStreamBlocks) cap = kMaxStreamBlocks;
   if (blocks > cap) blocks = cap;
