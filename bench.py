@@ -47,17 +47,17 @@ PREFIX_WORKLOAD = "math7b"  # prefix rescoring and the backward are timed on the
 # DRAM bytes (read + written) per row in the loss of the LM-head kernel (rows read by index),
 # by (workload, vocabulary splits), from one-pass ncu captures (dram__bytes_read.sum +
 # dram__bytes_write.sum) of the current kernel on the MoE-shaped head.  4 splits: one wave
-# of 19,456 rows, 2.575841 GB read + 4.0 MB written; every round of items reads the
-# vocabulary once, so the bytes grow with the rows (a full 3,958,414-row launch of the
-# previous kernel read 133.1 KB per row, this wave 132.6 KB) and the wave's figure per row is
-# scaled by the launch's rows.  2 splits: a single wave is not proportional to a long launch
-# (the clusters of a split drift apart over it), so the figure is one full 3,958,414-row
-# launch, 289.62 GB read + 127.7 MB written.  Emptied whenever the kernel changes, until it
-# is captured again.  The tag reduction's per tag: 14.0656 GB read + 19.8 MB written for the
-# 3.5023 G tags of the 1M sweep pool.
-LMHEAD_DRAM_BYTES_PER_ROW = {("moe", 4): (2575841024 + 4003584) / 19456,
-                             ("moe", 2): (289.62e9 + 127.72e6) / 3958414}
-TAG_REDUCE_DRAM_BYTES_PER_TAG = (14065824512 + 19798528) / 3502330341
+# of 19,456 rows, 2.589991 GB read + 4.27 MB written; every round of items reads the
+# vocabulary once, so the bytes grow with the rows and the wave's figure per row is scaled by
+# the launch's rows.  2 splits: a single wave is not proportional to a long launch (the
+# clusters of a split drift apart over it), so the figure is one full 3,958,414-row launch,
+# 298.063 GB read + 129.3 MB written.  Emptied whenever the kernel changes, until it is
+# captured again.  The tag reduction's per tag: 219.96 MB read + 3.12 MB written for the
+# 54.93 M tags of the 16k sweep pool (the atomic-free kernel; its reads equal the algorithmic
+# bytes, so the figure per tag carries to the larger pools).
+LMHEAD_DRAM_BYTES_PER_ROW = {("moe", 4): (2589990656 + 4268800) / 19456,
+                             ("moe", 2): (298063478784 + 129295872) / 3958414}
+TAG_REDUCE_DRAM_BYTES_PER_TAG = (219963904 + 3123712) / 54929421
 SWEEP_N = 1048576
 SWEEP_SIZES = (1024, 16384, 131072, SWEEP_N)
 METRIC = "accepted tokens/sec (logprob+loss) and % bf16 tensor peak; pool scoring traj/s + HBM GB/s"
