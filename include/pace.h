@@ -112,8 +112,14 @@ PACE_API void pace_score_params_default(PaceScoreParams* p);
  * S = sum (c - v_t) summed exactly in integers (0 when T = 0); q = count of
  * window values <= s_pre (float32 compare) / |W|; integer powers by repeated
  * multiplication; no fused multiply-add anywhere.
+ * Launches: the tag stream (one wave, whose blocks also sort the window and
+ * tabulate F on pools of 8,192 trajectories and more) and a finalisation
+ * launch; from 2^18 trajectories (pace_set_score_fused_min_traj) the stream is
+ * a cooperative launch that also finalises, each block waiting (bounded) for
+ * the blocks that streamed its groups' tokens.
  * Device-side errors: PACE_ERR_VERSION_ORDER (v_t > c or c > j),
- * PACE_ERR_INVALID_ARG (tag < -1, c < 0, bad offsets), PACE_ERR_NAN_INPUT.
+ * PACE_ERR_INVALID_ARG (tag < -1, c < 0, bad offsets), PACE_ERR_NAN_INPUT,
+ * PACE_ERR_TIMEOUT (a bounded wait of the cooperative launch ran out).
  * Host errors: PACE_ERR_INVALID_ARG when n_traj is not a multiple of G or a
  * required pointer is NULL. */
 PACE_API pace_status pace_score_pool(const int32_t* tags, const int64_t* offsets,
@@ -125,8 +131,11 @@ PACE_API pace_status pace_score_pool(const int32_t* tags, const int64_t* offsets
                             void* stream);
 
 /* Workspace bytes pace_score_pool needs for a pool of n_traj trajectories and
- * a window of window_len values (the per-trajectory accumulators, the sorted
- * window and the table of F over every possible ECDF count). */
+ * a window of window_len values: a 16-byte slot per trajectory for the tag
+ * stream's totals, 512 KB of per-warp partial slots, the sorted window, the
+ * table of F over every possible ECDF count and a few KB of flags.  Its
+ * contents need no initialisation and are overwritten by every call; calls
+ * that overlap on the GPU need workspaces of their own. */
 PACE_API size_t pace_score_pool_workspace_size(int64_t n_traj, int64_t window_len);
 
 /* ------------------------------------------------------------------------ */
