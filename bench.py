@@ -230,7 +230,7 @@ def _sweep_scoring(steps, warmup, device, n_traj=SWEEP_N):
     g_ms = _timed(_capture(one, device).replay, steps, warmup, flush)
     assert int(status.item()) == 0, pace.status_string(int(status.item()))
     # algorithmic bytes of the tag reduction: every tag once, the offsets once,
-    # the 16-byte per-trajectory accumulators written once
+    # the 16-byte per-trajectory slots written once
     k_bytes = 4 * tok + 8 * (n + 1) + 16 * n
     fused = n >= L.pace_score_fused_min_traj_default()
     res = {"workload": f"sweep pool {n} trajectories, {tok} tags", "traj_per_s": n / (s_ms / 1e3),

@@ -558,8 +558,9 @@ PACE_API pace_status pace_set_lmhead_splits(int32_t splits);
  * tag stream is done, scores its own slice of the groups after bounded waits
  * for the blocks that streamed those groups' tokens (a cooperative launch, so
  * every block is resident and the waits end); most of the per-trajectory work
- * then hides in the stream's ragged tail.  Smaller pools finalise in a launch
- * of their own, which is faster there.  Results are identical either way.
+ * then hides in the stream's ragged tail.  Smaller pools, and every pool on a
+ * device without cooperative launches, finalise in a launch of their own,
+ * which is faster on small pools.  Results are identical either way.
  * From now on, in this process, the given threshold applies (0: every pool;
  * the default is pace_score_fused_min_traj_default(), 2^18).  Returns
  * PACE_ERR_INVALID_ARG for a negative min_traj. */

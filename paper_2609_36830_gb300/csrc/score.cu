@@ -55,6 +55,26 @@ std::atomic<int64_t>& fused_min_traj() {
   static std::atomic<int64_t> v{kFusedMinTrajDefault};
   return v;
 }
+
+// Whether the current device takes cooperative launches (cached per device);
+// where it does not, every pool finalises in a launch of its own.
+bool cooperative_launch_ok() {
+  constexpr int kMaxDevices = 64;
+  static std::atomic<int> cache[kMaxDevices];  // 0 unknown, 1 yes, 2 no
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return false;
+  int c = cache[dev].load();
+  if (c == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess) {
+      (void)cudaGetLastError();
+      v = 0;
+    }
+    c = v ? 1 : 2;
+    cache[dev].store(c);
+  }
+  return c == 1;
+}
 constexpr int64_t kTableMinTraj = 8192;  // pools from this size sort W and tabulate F
 
 __device__ __forceinline__ int4 ld_stream_v4(const int32_t* p) {
@@ -667,7 +687,7 @@ __device__ void finalize_load_window(const FinalizeArgs& p, const FinalizeSmem& 
 }
 
 // What one thread of a pass reads for its trajectory: the inputs (loadable any
-// time) and the accumulators of the stream (only once the stream blocks that
+// time) and the stream's totals from the slots (only once the stream blocks that
 // hold its tokens are done).
 struct TrajIn {
   float s;
@@ -853,7 +873,7 @@ __device__ __forceinline__ void fused_finalize(const int64_t* __restrict__ offse
   const int tid = static_cast<int>(threadIdx.x);
   const int S = n_stream_blocks;
   const int64_t blk = blockIdx.x;
-  __threadfence();  // this thread's accumulator atomics before the block's flag
+  __threadfence();  // this thread's slot stores before the block's flag
   __syncthreads();
   if (tid == 0) {
     __threadfence();
@@ -1251,7 +1271,7 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   a.unit_score = unit_score;
   a.status = status_dev;
 
-  if (G <= kReduceThreads && n_traj >= fused_min_traj().load()) {
+  if (G <= kReduceThreads && n_traj >= fused_min_traj().load() && cooperative_launch_ok()) {
     // Large pools whose groups fit one block: the finalisation runs inside the
     // tag reduction's launch, each stream block finalising its slice of the
     // groups in the stream's ragged tail, where most of the per-trajectory work
