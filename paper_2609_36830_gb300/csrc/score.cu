@@ -865,7 +865,6 @@ struct FusedFinalize {
 // tokens and the preparation are done.  Each block thus finalises in the tail
 // as soon as its neighbourhood of the stream is complete, and no launch of its
 // own is needed.
-template <int kTilesPerBatch>
 __device__ __forceinline__ void fused_finalize(const int64_t* __restrict__ offsets,
                                                int64_t n_tokens, int n_stream_blocks,
                                                const FusedFinalize& fz) {
@@ -912,13 +911,9 @@ __device__ __forceinline__ void fused_finalize(const int64_t* __restrict__ offse
     if (t1 < t0) {  // inconsistent offsets (reported by the pass): wait for every block
       b_hi = S - 1;
     } else if (t1 > t0) {
-      constexpr int64_t kBatchTokens = kTileTokens * kTilesPerBatch;
-      const int64_t n_batches = (n_tokens + kBatchTokens - 1) / kBatchTokens;
-      const int64_t n_warps = static_cast<int64_t>(S) * (kReduceThreads / 32);
-      const int64_t w0 = ((t0 / kBatchTokens + 1) * n_warps - 1) / n_batches;
-      const int64_t w1 = (((t1 - 1) / kBatchTokens + 1) * n_warps - 1) / n_batches;
-      b_lo = w0 / (kReduceThreads / 32);
-      b_hi = w1 / (kReduceThreads / 32);
+      const StreamGeom& g = p.geom;
+      b_lo = warp_of_batch(g, t0 / g.batch_tokens) / (kReduceThreads / 32);
+      b_hi = warp_of_batch(g, (t1 - 1) / g.batch_tokens) / (kReduceThreads / 32);
     }
     bool ok = true;
     const uint64_t start = global_timer_ns();
@@ -968,7 +963,7 @@ __global__ void __launch_bounds__(kReduceThreads, kMinBlocks)
     return;
   }
   stream_warp_range<kTilesPerBatch>(tags, offsets, n_traj, n_tokens, tt, n_stream_blocks);
-  if (fz.done) fused_finalize<kTilesPerBatch>(offsets, n_tokens, n_stream_blocks, fz);
+  if (fz.done) fused_finalize(offsets, n_tokens, n_stream_blocks, fz);
 }
 
 // Stale-k admission (Sec. 2): kbar = sum (j - v_t) / T = (j T - sum v_t) / T in
