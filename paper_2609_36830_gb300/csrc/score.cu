@@ -663,25 +663,30 @@ __device__ __forceinline__ FinalizeSmem finalize_smem(unsigned char* raw, int wi
 __device__ void finalize_load_window(const FinalizeArgs& p, const FinalizeSmem& m) {
   if (p.window_ready) {
     const bool sorted = p.window_sorted != nullptr;
+    const bool table = m.ftab && sorted;
     const int wpad = (p.window_len + 3) & ~3;
+    const int tlen = table ? p.window_len + 1 : 0;
+    const int span = wpad > tlen ? wpad : tlen;
     const float* src = sorted ? p.window_sorted : p.window;
     const int nb = static_cast<int>(blockDim.x);
-    for (int k0 = threadIdx.x; k0 < wpad; k0 += 4 * nb) {
+    // four window values and four table entries per thread in flight at once
+    for (int k0 = threadIdx.x; k0 < span; k0 += 4 * nb) {
       float w[4];
+      double f[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int k = k0 + j * nb;
         w[j] = k < p.window_len ? __ldcg(src + k) : __int_as_float(0x7fc00000);
+        f[j] = k < tlen ? __ldcg(p.f_table + k) : 0.0;
       }
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int k = k0 + j * nb;
         if (k < wpad) m.swin[k] = w[j];
+        if (k < tlen) m.ftab[k] = f[j];
         if (!sorted && k < p.window_len && isnan(w[j])) report(p.status, PACE_ERR_NAN_INPUT);
       }
     }
-    if (m.ftab && sorted)
-      for (int k = threadIdx.x; k <= p.window_len; k += nb) m.ftab[k] = __ldcg(p.f_table + k);
   }
   __syncthreads();
 }
@@ -1299,18 +1304,22 @@ extern "C" pace_status pace_score_pool(const int32_t* tags, const int64_t* offse
   PACE_TRY(run_tag_reduce(tags, offsets, n_traj, n_tokens, ws, prep, FusedFinalize{}, false, 0,
                           &a.geom, st));
   // A launch of its own: whole groups per block.  With the sorted window: one
-  // thread per trajectory, 64 to 256 threads; small pools take fewer groups per
-  // block so that the per-trajectory fp64 work (GB300's fp64 rate is low) is
-  // spread over about two blocks per SM instead of queueing on a few SMs.  With
-  // the direct count, up to 8 threads per trajectory share the count so its
-  // chain is 8 times shorter.
+  // thread per trajectory, 256 threads (whole groups) per block, so that one
+  // round of loads brings the window and the F table into shared memory.
+  // Otherwise small pools take fewer groups per block so that the
+  // per-trajectory fp64 work of F (GB300's fp64 rate is low) is spread over
+  // about two blocks per SM instead of queueing on a few SMs; with the direct
+  // count, up to 8 threads per trajectory share the count so its chain is 8
+  // times shorter.
   const int max_units = G >= 256 ? 1 : 256 / G;
   const int64_t n_units = n_traj / G;
   const int64_t spread = 2 * static_cast<int64_t>(sm_count());
   int64_t want = (n_units + spread - 1) / spread;
   int min_units = 1;
   int lanes = 1;
-  if (!use_table && window_ready) {
+  if (use_table) {
+    min_units = max_units;
+  } else if (window_ready) {
     lanes = 8;
   } else {
     min_units = G >= 64 ? 1 : (64 + G - 1) / G;
