@@ -565,6 +565,8 @@ PACE_API pace_status pace_set_lmhead_splits(int32_t splits);
  * the default is pace_score_fused_min_traj_default(), 2^18).  Returns
  * PACE_ERR_INVALID_ARG for a negative min_traj. */
 PACE_API pace_status pace_set_score_fused_min_traj(int64_t min_traj);
+
+/* The library's default for pace_set_score_fused_min_traj (2^18 trajectories). */
 PACE_API int64_t pace_score_fused_min_traj_default(void);
 
 /* Not part of the method: a measurement aid.  From now on, on the calling
