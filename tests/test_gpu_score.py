@@ -134,7 +134,7 @@ def _mk(lens, rng, j=50, tool=0.0):
 
 
 @pytest.mark.parametrize("case", ["empty_traj", "ragged", "one_long", "tiny_many", "all_tool",
-                                  "single", "huge_versions", "mixed_versions"])
+                                  "single", "huge_versions", "mixed_versions", "warp_aligned"])
 def test_edge_cases(case):
     """Pool shapes and tag ranges that take every path of the tag reduction: empty
     trajectories, boundaries at and off batch edges, tool tags, and versions at and
@@ -153,6 +153,14 @@ def test_edge_cases(case):
         lens = [10, 20, 30, 40]
     elif case in ("huge_versions", "mixed_versions"):
         lens = list(rng.integers(1, 5000, size=64))
+    elif case == "warp_aligned":
+        # trajectories of whole 512-tag batches, so every trajectory boundary is a
+        # batch edge, where warp ranges begin and end too (many coincide), with
+        # empty trajectories on the boundaries: each case of which warp writes a
+        # trajectory's slot and which warp's head slot continues it
+        lens = []
+        for i in range(48):
+            lens += [2048 * (1 + i % 3)] + [0] * (i % 2) + [512 * (1 + i % 5)] + [0] * (i % 3)
     else:
         lens = [1]
     lens = list(lens)
